@@ -1,0 +1,10 @@
+"""CPU oracle for VBQ (test infrastructure only).
+
+Only tests/, __graft_entry__.smoke() and bench.py's CPU baseline leg may
+import this package. The CUDA library and its Python binding never do.
+"""
+
+from .vbq_oracle import (  # noqa: F401
+    GROUP, WIDTHS, level, check_inputs, dequant, gemv, within_bound,
+    quantize_group, quantize, payload_bytes, scale_bytes, pack_lsb, unpack_lsb,
+)

@@ -1,0 +1,215 @@
+"""CPU oracle for VBQ per-group variable bit-width weights (fp64, numpy).
+
+TEST INFRASTRUCTURE. Only tests/, __graft_entry__.smoke() and bench.py's CPU
+baseline leg may import or call this module. The CUDA library never uses it,
+and this module imports nothing from the CUDA package.
+
+What it defines (paper: "Variable Bit-width Quantization", arXiv 2607.02893):
+
+* Groups: a weight matrix W (N x K, row-major) is cut into contiguous groups of
+  G = 64 weights along K (§3.1); group g of row n covers columns [64g, 64g+64).
+  Each group has its own width b in {1, 2, 4, 8} (§3.2, the candidate set) and
+  one scale s (§3.1), stored as FP16.
+* Quantiser, b >= 2 (§3.1, Eq. 1): s = max|w| / (2^(b-1) - 1) and
+  w_hat = s * clip(round(w / s), -(2^(b-1) - 1), 2^(b-1) - 1).
+* Quantiser, b = 1 (§3.1): w_hat = sign(w) * mean|w| over the group.
+* Packed storage: each group holds 64*b bits (§1, §6: "aligned byte
+  boundaries"), i.e. 8*b bytes, plus its scale.
+* The inference product (§6): y = W_hat x with the weights never widened in
+  memory; here simply the plain dense definition in fp64.
+
+Readings of points the paper leaves open (each also listed in the design notes):
+
+* Code encoding (never given in the paper): b >= 2 stores the integer
+  q in [-(2^(b-1)-1), 2^(b-1)-1] as offset binary u = q + 2^(b-1), so
+  L_b(u) = u - 2^(b-1). The code u = 0 (q = -2^(b-1)) is never produced by
+  the quantiser but is decoded by the same line. b = 1 stores u = 1 for
+  +mean|w| and u = 0 for -mean|w|, so L_1(u) = 2u - 1.
+* round() breaks ties to even (round-half-to-even).
+* sign(0) = +1 (one bit cannot encode zero).
+* The scale is computed in fp64, rounded to FP16 (round to nearest even),
+  and the codes are computed with the rounded scale; clip absorbs overshoot.
+  Scales above 65504 saturate to 65504.
+* An all-zero group (or one whose scale rounds to 0) gets s = 0 and codes
+  u = 2^(b-1) (b >= 2) or u = 1 (b = 1); it dequantises to zeros.
+* Activations are BF16; the reference product is exact-input fp64:
+  y[b, n] = sum_k f64(w_hat[n, k]) * f64(x[b, k]), with the error-scale term
+  A[b, n] = sum_k |w_hat[n, k] * x[b, k]|.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+
+GROUP = 64
+WIDTHS = (1, 2, 4, 8)
+FP16_MAX = 65504.0
+
+
+# ---------------------------------------------------------------------------
+# Level map (§3.1, Eq. 1 and the 1-bit sign rule; encoding as read above)
+# ---------------------------------------------------------------------------
+
+def level(b: int, u):
+    """Integer level L_b(u) of code u at width b (scalar or integer array)."""
+    u = np.asarray(u, dtype=np.int64)
+    if b == 1:
+        return 2 * u - 1
+    if b in (2, 4, 8):
+        return u - (1 << (b - 1))
+    raise ValueError(f"width {b} not in {WIDTHS}")
+
+
+def check_inputs(codes: np.ndarray, widths: np.ndarray, scales: np.ndarray) -> None:
+    n, k = codes.shape
+    if k % GROUP:
+        raise ValueError("K must be a multiple of 64")
+    if widths.shape != (n, k // GROUP) or scales.shape != (n, k // GROUP):
+        raise ValueError("widths/scales must be N x K/64")
+    if not np.isin(widths, WIDTHS).all():
+        raise ValueError("widths must be in {1,2,4,8}")
+    wide = np.repeat(widths.astype(np.int64), GROUP, axis=1)
+    if (codes.astype(np.int64) >= (np.int64(1) << wide)).any():
+        raise ValueError("code out of range for its group's width")
+
+
+def dequant(codes: np.ndarray, widths: np.ndarray, scales_fp16: np.ndarray) -> np.ndarray:
+    """Dense fp64 W_hat[n, k] = f64(s[n, k // 64]) * L_{b[n, k // 64]}(codes[n, k])."""
+    codes = np.asarray(codes, dtype=np.uint8)
+    widths = np.asarray(widths, dtype=np.uint8)
+    scales = np.asarray(scales_fp16, dtype=np.float16)
+    check_inputs(codes, widths, scales)
+    n, k = codes.shape
+    w = np.empty((n, k), dtype=np.float64)
+    for g in range(k // GROUP):
+        cols = slice(g * GROUP, (g + 1) * GROUP)
+        s = scales[:, g].astype(np.float64)
+        lv = np.zeros((n, GROUP), dtype=np.int64)
+        for b in WIDTHS:
+            rows = widths[:, g] == b
+            if rows.any():
+                lv[rows] = level(b, codes[rows, cols])
+        w[:, cols] = s[:, None] * lv.astype(np.float64)
+    return w
+
+
+def gemv(codes: np.ndarray, widths: np.ndarray, scales_fp16: np.ndarray, x: np.ndarray):
+    """y = W_hat x for a batch of activation rows.
+
+    x: (B, K) or (K,) float array holding the (BF16-representable) activations.
+    Returns (y, A), both (B, N) fp64, A[b, n] = sum_k |w_hat[n, k] * x[b, k]|.
+    """
+    w = dequant(codes, widths, scales_fp16)
+    x = np.atleast_2d(np.asarray(x, dtype=np.float64))
+    if x.shape[1] != w.shape[1]:
+        raise ValueError("x has the wrong length")
+    y = np.empty((x.shape[0], w.shape[0]), dtype=np.float64)
+    a = np.empty_like(y)
+    for bi in range(x.shape[0]):
+        prod = w * x[bi][None, :]
+        y[bi] = prod.sum(axis=1)
+        a[bi] = np.abs(prod).sum(axis=1)
+    return y, a
+
+
+def within_bound(y, y_ref, a_ref, rel: float = 2e-3, floor: float = 1e-5) -> np.ndarray:
+    """Acceptance test of a computed y: |y - y_ref| <= rel * A + floor, elementwise."""
+    return np.abs(np.asarray(y, np.float64) - y_ref) <= rel * a_ref + floor
+
+
+# ---------------------------------------------------------------------------
+# Quantiser (§3.1, Eq. 1 and the 1-bit absmean rule)
+# ---------------------------------------------------------------------------
+
+def _to_fp16_scale(s: float) -> np.float16:
+    if s > FP16_MAX:
+        return np.float16(FP16_MAX)
+    return np.float16(s)
+
+
+def quantize_group(w, b: int, fp16_scale: bool = True):
+    """Quantise one group of weights at width b.
+
+    Returns (codes uint8[len(w)], scale) where scale is np.float16 if
+    fp16_scale else the unrounded fp64 value.
+    """
+    w = np.asarray(w, dtype=np.float64)
+    if b == 1:
+        s = float(np.mean(np.abs(w)))
+        s_used = _to_fp16_scale(s) if fp16_scale else s
+        codes = (w >= 0).astype(np.uint8)          # sign(0) = +1
+        return codes, s_used
+    if b not in (2, 4, 8):
+        raise ValueError(f"width {b} not in {WIDTHS}")
+    qmax = (1 << (b - 1)) - 1
+    z = 1 << (b - 1)
+    m = float(np.max(np.abs(w))) if w.size else 0.0
+    s = m / qmax
+    s_used = _to_fp16_scale(s) if fp16_scale else s
+    sf = float(s_used)
+    if sf == 0.0:
+        return np.full(w.shape, z, dtype=np.uint8), s_used
+    q = np.clip(np.round(w / sf), -qmax, qmax).astype(np.int64)   # np.round: ties to even
+    return (q + z).astype(np.uint8), s_used
+
+
+def quantize(w: np.ndarray, widths: np.ndarray):
+    """Quantise an N x K matrix with per-group widths; returns (codes, scales_fp16)."""
+    w = np.asarray(w, dtype=np.float64)
+    n, k = w.shape
+    widths = np.asarray(widths, dtype=np.uint8)
+    if k % GROUP or widths.shape != (n, k // GROUP):
+        raise ValueError("bad shapes")
+    codes = np.empty((n, k), dtype=np.uint8)
+    scales = np.empty((n, k // GROUP), dtype=np.float16)
+    for r in range(n):
+        for g in range(k // GROUP):
+            c, s = quantize_group(w[r, g * GROUP:(g + 1) * GROUP], int(widths[r, g]))
+            codes[r, g * GROUP:(g + 1) * GROUP] = c
+            scales[r, g] = s
+    return codes, scales
+
+
+# ---------------------------------------------------------------------------
+# Storage accounting (§1, §6: each group packs 64*b bits plus its FP16 scale)
+# ---------------------------------------------------------------------------
+
+def payload_bytes(widths: np.ndarray) -> int:
+    """Packed code bytes: sum over groups of 64*b/8."""
+    return int(np.asarray(widths, dtype=np.int64).sum()) * GROUP // 8
+
+
+def scale_bytes(widths: np.ndarray) -> int:
+    return 2 * int(np.asarray(widths).size)
+
+
+def pack_lsb(codes: np.ndarray, widths: np.ndarray) -> bytes:
+    """Plain reference packing: groups in row-major order, each group's 64 codes
+    LSB-first into 8*b bytes. Used to check the storage accounting."""
+    out = bytearray()
+    n, k = codes.shape
+    for r in range(n):
+        for g in range(k // GROUP):
+            b = int(widths[r, g])
+            acc = 0
+            for i in range(GROUP):
+                acc |= int(codes[r, g * GROUP + i]) << (i * b)
+            out += acc.to_bytes(8 * b, "little")
+    return bytes(out)
+
+
+def unpack_lsb(buf: bytes, widths: np.ndarray) -> np.ndarray:
+    n, g = widths.shape
+    codes = np.empty((n, g * GROUP), dtype=np.uint8)
+    pos = 0
+    for r in range(n):
+        for j in range(g):
+            b = int(widths[r, j])
+            acc = int.from_bytes(buf[pos:pos + 8 * b], "little")
+            pos += 8 * b
+            mask = (1 << b) - 1
+            for i in range(GROUP):
+                codes[r, j * GROUP + i] = (acc >> (i * b)) & mask
+    if pos != len(buf):
+        raise ValueError("trailing bytes")
+    return codes

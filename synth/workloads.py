@@ -1,0 +1,113 @@
+"""Workload descriptions: matrix shapes and per-group bit-width distributions.
+
+Shapes follow the decoder families of the paper's inference study (§6,
+Table 2: a ~131M TinyStories decoder, ~1B and ~9B models) as plain linear
+stacks: per layer Q, K, V, O, gate, up, down, then the LM head. W is stored
+N x K (output features x input features); groups of 64 run along K.
+
+Bit-width distributions are probabilities over widths (1, 2, 4, 8):
+  * main:  the adaptive-search allocation of §5.1 (most groups at 1 bit),
+           p = (0.69, 0.15, 0.11, 0.05), mean 1.83 bits;
+  * mlp0:  the first block's MLP, which keeps more precision (§5.1, §3.4),
+           p = (0.40, 0.30, 0.22, 0.08), mean 2.50 bits;
+  * head:  the LM head, mostly 1 bit (§5.1), p = (0.96, 0.025, 0.01, 0.005),
+           mean 1.09 bits.
+"""
+
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import List, Tuple
+
+WIDTHS = (1, 2, 4, 8)
+
+DIST_MAIN = (0.69, 0.15, 0.11, 0.05)
+DIST_MLP0 = (0.40, 0.30, 0.22, 0.08)
+DIST_HEAD = (0.96, 0.025, 0.01, 0.005)
+DIST_ALL1 = (1.0, 0.0, 0.0, 0.0)
+DIST_ALL2 = (0.0, 1.0, 0.0, 0.0)
+DIST_ALL4 = (0.0, 0.0, 1.0, 0.0)
+DIST_ALL8 = (0.0, 0.0, 0.0, 1.0)
+
+SWEEP_DISTS = {
+    "all1": DIST_ALL1, "all2": DIST_ALL2, "all4": DIST_ALL4, "all8": DIST_ALL8,
+    "mixed": DIST_MAIN,
+}
+
+
+@dataclass(frozen=True)
+class MatrixSpec:
+    """One weight matrix of a workload: W is n x k, groups of 64 along k."""
+    name: str
+    n: int
+    k: int
+    dist: Tuple[float, float, float, float]
+    seed_path: Tuple[int, ...]   # (config_id, layer, proj_id) for the seed sequence
+
+
+@dataclass
+class Workload:
+    name: str
+    config_id: int
+    batch: int
+    mats: List[MatrixSpec] = field(default_factory=list)
+
+    @property
+    def weights(self) -> int:
+        return sum(m.n * m.k for m in self.mats)
+
+
+def _stack(config_id: int, d_model: int, n_layers: int, d_q: int, d_kv: int,
+           d_ff: int, vocab: int) -> List[MatrixSpec]:
+    mats: List[MatrixSpec] = []
+    for layer in range(n_layers):
+        mlp = DIST_MLP0 if layer == 0 else DIST_MAIN
+        projs = [
+            ("q", d_q, d_model, DIST_MAIN),
+            ("k", d_kv, d_model, DIST_MAIN),
+            ("v", d_kv, d_model, DIST_MAIN),
+            ("o", d_model, d_q, DIST_MAIN),
+            ("gate", d_ff, d_model, mlp),
+            ("up", d_ff, d_model, mlp),
+            ("down", d_model, d_ff, mlp),
+        ]
+        for pid, (pname, n, k, dist) in enumerate(projs):
+            mats.append(MatrixSpec(f"l{layer}.{pname}", n, k, dist, (config_id, layer, pid)))
+    mats.append(MatrixSpec("head", vocab, d_model, DIST_HEAD, (config_id, n_layers, 0)))
+    return mats
+
+
+def workload(name: str, batch: int = 1) -> Workload:
+    """Named workloads.
+
+    single768   one 768 x 768 GEMV, main distribution.
+    stack131m   d_model 768, 12 layers, MLP 2048, head 32000 (85 GEMVs).
+    stack1b     d_model 2048, 22 layers, Q/O 2048, K/V 256, MLP 5632, head 32000 (155 GEMVs).
+    stack9b     d_model 4096, 32 layers, Q/O 4096, K/V 1024, MLP 14336, head 128256 (225 GEMVs).
+    sweep:<n>:<dist>  one n x n GEMV, dist in all1/all2/all4/all8/mixed.
+    """
+    if name == "single768":
+        return Workload(name, 0, batch, [MatrixSpec("w", 768, 768, DIST_MAIN, (0, 0, 0))])
+    if name == "stack131m":
+        return Workload(name, 1, batch, _stack(1, 768, 12, 768, 768, 2048, 32000))
+    if name == "stack1b":
+        return Workload(name, 2, batch, _stack(2, 2048, 22, 2048, 256, 5632, 32000))
+    if name == "stack9b":
+        return Workload(name, 3, batch, _stack(3, 4096, 32, 4096, 1024, 14336, 128256))
+    if name.startswith("sweep:"):
+        _, n, dist = name.split(":")
+        n = int(n)
+        didx = list(SWEEP_DISTS).index(dist)
+        return Workload(name, 4, batch,
+                        [MatrixSpec(f"sweep{n}.{dist}", n, n, SWEEP_DISTS[dist], (4, n, didx))])
+    raise KeyError(name)
+
+
+def workload_names() -> List[str]:
+    return ["single768", "stack131m", "stack1b", "stack9b"]
+
+
+def sweep_points() -> List[Tuple[int, int, str]]:
+    """(n, batch, dist) of the roofline sweep: 3 sizes x 5 batches x 5 distributions."""
+    return [(n, b, d) for n in (4096, 8192, 16384) for b in (1, 2, 4, 8, 16)
+            for d in SWEEP_DISTS]

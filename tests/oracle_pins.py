@@ -1,0 +1,216 @@
+"""Checks that pin the CPU oracle to the paper and to plain mathematics.
+
+Each pin takes the oracle module as an argument so that the same checks can
+be run against deliberately broken copies of it (see test_oracle.py): every
+plausible mistake must trip at least one pin.
+"""
+
+from __future__ import annotations
+
+import os
+from fractions import Fraction
+
+import numpy as np
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+class PinFailed(AssertionError):
+    pass
+
+
+def _check(cond, msg):
+    if not cond:
+        raise PinFailed(msg)
+
+
+def load_eq1_examples():
+    rows = []
+    with open(os.path.join(GOLDEN, "eq1_examples.txt")) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            name, b, pairs, sbits, codes, zcode = [p.strip() for p in line.split("|")]
+            idx, vals = [], []
+            for tok in pairs.split():
+                i, v = tok.split(":")
+                idx.append(int(i))
+                vals.append(float(v))
+            rows.append(dict(name=name, b=int(b), idx=idx, vals=vals,
+                             sbits=int(sbits, 16),
+                             codes=[int(c) for c in codes.split()], zcode=int(zcode)))
+    return rows
+
+
+def pin_eq1_golden(O):
+    """Hand-worked Eq. 1 / 1-bit examples: scale bits and codes."""
+    for ex in load_eq1_examples():
+        w = np.zeros(64)
+        w[ex["idx"]] = ex["vals"]
+        codes, s = O.quantize_group(w, ex["b"])
+        _check(int(np.float16(s).view(np.uint16)) == ex["sbits"],
+               f"{ex['name']}: scale bits {int(np.float16(s).view(np.uint16)):04x} != {ex['sbits']:04x}")
+        exp = np.full(64, ex["zcode"], dtype=np.int64)
+        exp[ex["idx"]] = ex["codes"]
+        _check(np.array_equal(codes.astype(np.int64), exp), f"{ex['name']}: codes {codes} != {exp}")
+
+
+def pin_level_grid(O):
+    """Eq. 1's reconstruction grid: integer, uniform step 1, symmetric, zero at the
+    midpoint code; the quantiser's codes 1 .. 2^b-1 span -qmax .. qmax. 1 bit: +-1."""
+    for b in (2, 4, 8):
+        qmax = (1 << (b - 1)) - 1
+        z = 1 << (b - 1)
+        lv = [int(O.level(b, u)) for u in range(1 << b)]
+        _check(lv[z] == 0, f"b={b}: midpoint code is not the zero level")
+        _check(all(lv[u + 1] - lv[u] == 1 for u in range(len(lv) - 1)), f"b={b}: grid step")
+        _check(lv[1] == -qmax and lv[(1 << b) - 1] == qmax, f"b={b}: emitted range")
+        _check(all(lv[z + k] == -lv[z - k] for k in range(1, qmax + 1)), f"b={b}: symmetry")
+    _check(int(O.level(1, 1)) == 1 and int(O.level(1, 0)) == -1, "1-bit polarity")
+
+
+def pin_grid_roundtrip(O, seed=1):
+    """Weights already on an Eq. 1 grid (power-of-two scale, a group containing
+    +-qmax) are reproduced exactly by quantise -> dequantise; a constant-magnitude
+    group at 1 bit too."""
+    rng = np.random.default_rng(seed)
+    for b in (1, 2, 4, 8):
+        n, k = 3, 128
+        widths = np.full((n, k // 64), b, dtype=np.uint8)
+        if b == 1:
+            mag = 2.0 ** rng.integers(-8, 2, size=(n, k // 64))
+            sign = np.where(rng.random((n, k)) < 0.5, -1.0, 1.0)
+            w = sign * np.repeat(mag, 64, axis=1)
+        else:
+            qmax = (1 << (b - 1)) - 1
+            q = rng.integers(-qmax, qmax + 1, size=(n, k))
+            q[:, ::64] = qmax                          # each group contains +qmax
+            s = 2.0 ** rng.integers(-10, 0, size=(n, k // 64))
+            w = np.repeat(s, 64, axis=1) * q
+        codes, scales = O.quantize(w, widths)
+        _check(np.array_equal(O.dequant(codes, widths, scales), w), f"b={b}: grid roundtrip")
+
+
+def pin_quantizer_invariants(O, seed=2):
+    rng = np.random.default_rng(seed)
+    for b in (2, 4, 8):
+        qmax = (1 << (b - 1)) - 1
+        for _ in range(20):
+            w = rng.normal(0, rng.uniform(0.01, 3.0), size=64)
+            codes, s = O.quantize_group(w, b)
+            q = codes.astype(np.int64) - (1 << (b - 1))
+            _check(np.all(np.abs(q) <= qmax), f"b={b}: |q| > qmax")
+            sf = float(s)
+            err = np.abs(w - sf * q)
+            _check(np.all(err <= sf / 2 * (1 + 1e-9) + 1e-12), f"b={b}: error above s/2")
+            imax = int(np.argmax(np.abs(w)))
+            _check(abs(int(q[imax])) == qmax, f"b={b}: max-magnitude weight not at +-qmax")
+            # idempotence: quantising the reconstruction gives the same codes and scale
+            wh = sf * q
+            c2, s2 = O.quantize_group(wh, b)
+            _check(np.array_equal(c2, codes) and float(s2) == sf, f"b={b}: not idempotent")
+    for _ in range(10):
+        w = rng.normal(0, 1, size=64)
+        codes, s = O.quantize_group(w, 1)
+        _check(np.array_equal(codes, (w >= 0).astype(np.uint8)), "1-bit codes != sign")
+        _check(float(s) == float(np.float16(np.mean(np.abs(w)))), "1-bit scale != mean|w|")
+
+
+def pin_group_size_one(O, seed=3):
+    """§3.1: with one weight per group every width reconstructs w exactly
+    (unrounded scale)."""
+    rng = np.random.default_rng(seed)
+    for w0 in rng.normal(0, 1, size=50):
+        for b in (1, 2, 4, 8):
+            codes, s = O.quantize_group(np.array([w0]), b, fp16_scale=False)
+            wh = s * int(O.level(b, int(codes[0])))
+            _check(abs(wh - w0) <= 4e-16 * abs(w0), f"b={b}: G=1 not exact ({wh} vs {w0})")
+
+
+def pin_integer_gemv(O, seed=4):
+    """All-8-bit, unit scales, small integer x: y is an exact integer product,
+    checked against an int64 matmul; and with power-of-two scales and mixed
+    widths against exact rational arithmetic on a tiny case."""
+    rng = np.random.default_rng(seed)
+    n, k = 37, 256
+    codes = rng.integers(0, 256, size=(n, k)).astype(np.uint8)
+    widths = np.full((n, k // 64), 8, dtype=np.uint8)
+    scales = np.ones((n, k // 64), dtype=np.float16)
+    x = rng.integers(-8, 9, size=(2, k))
+    y, a = O.gemv(codes, widths, scales, x.astype(np.float64))
+    exp = (codes.astype(np.int64) - 128) @ x.T.astype(np.int64)
+    _check(np.array_equal(y, exp.T.astype(np.float64)), "integer all-8-bit GEMV")
+    _check(np.array_equal(a, (np.abs(codes.astype(np.int64) - 128) @ np.abs(x.T)).T.astype(np.float64)),
+           "integer all-8-bit bound term")
+
+
+def pin_exact_rational(O, seed=5):
+    """Tiny mixed-width case: the fp64 product equals the exact rational sum of
+    the dequantised weights times x to within fp64 rounding."""
+    rng = np.random.default_rng(seed)
+    n, k = 5, 192
+    widths = rng.choice(np.array([1, 2, 4, 8], np.uint8), size=(n, k // 64))
+    codes = (rng.integers(0, 256, size=(n, k)) & ((1 << np.repeat(widths, 64, axis=1).astype(np.int64)) - 1)).astype(np.uint8)
+    scales = (np.abs(rng.normal(0, 0.02, size=(n, k // 64))) + 1e-4).astype(np.float16)
+    x = rng.normal(0, 1, size=k).astype(np.float32)
+    w = O.dequant(codes, widths, scales)
+    y, _ = O.gemv(codes, widths, scales, x)
+    for r in range(n):
+        exact = sum((Fraction(float(w[r, j])) * Fraction(float(x[j])) for j in range(k)), Fraction(0))
+        mag = sum(abs(Fraction(float(w[r, j])) * Fraction(float(x[j]))) for j in range(k))
+        _check(abs(Fraction(float(y[0, r])) - exact) <= mag * Fraction(1, 2 ** 45), f"row {r}: fp64 sum")
+    # one-hot activations pick out single dequantised weights: checks group indexing
+    for j in (0, 63, 64, 130, 191):
+        e = np.zeros(k)
+        e[j] = 1.0
+        yj, _ = O.gemv(codes, widths, scales, e)
+        g = j // 64
+        for r in range(n):
+            b = int(widths[r, g])
+            expect = float(scales[r, g]) * int(O.level(b, int(codes[r, j])))
+            _check(yj[0, r] == expect, f"one-hot column {j} row {r}")
+
+
+def pin_enumerated_codes(O):
+    """Brute force over every code at every position of one group: with a one-hot
+    x the product returns s * level, and for each width the 2^b results form the
+    uniform grid s * (-2^(b-1) .. 2^(b-1)-1) (b >= 2) or {-s, +s} (b = 1)."""
+    s = np.float16(0.375)
+    for b in (1, 2, 4, 8):
+        ncode = 1 << b
+        z = (1 << (b - 1)) if b > 1 else 1
+        n = ncode * 64
+        codes = np.full((n, 64), z, dtype=np.uint8)
+        for pos in range(64):
+            for u in range(ncode):
+                codes[pos * ncode + u, pos] = u
+        widths = np.full((n, 1), b, dtype=np.uint8)
+        scales = np.full((n, 1), s, dtype=np.float16)
+        for pos in (0, 1, 31, 63):
+            e = np.zeros(64)
+            e[pos] = 1.0
+            y, _ = O.gemv(codes, widths, scales, e)
+            got = y[0, pos * ncode:(pos + 1) * ncode]
+            if b == 1:
+                _check(list(got) == [-0.375, 0.375], f"b=1 pos {pos}: {got}")
+            else:
+                expect = [0.375 * (u - (1 << (b - 1))) for u in range(ncode)]
+                _check(list(got) == expect, f"b={b} pos {pos}")
+
+
+def pin_payload_accounting(O, seed=6):
+    rng = np.random.default_rng(seed)
+    n, k = 7, 320
+    widths = rng.choice(np.array([1, 2, 4, 8], np.uint8), size=(n, k // 64))
+    codes = (rng.integers(0, 256, size=(n, k)) & ((1 << np.repeat(widths, 64, axis=1).astype(np.int64)) - 1)).astype(np.uint8)
+    buf = O.pack_lsb(codes, widths)
+    _check(len(buf) == sum(64 * int(b) // 8 for b in widths.ravel()), "packed length")
+    _check(O.payload_bytes(widths) == len(buf), "payload_bytes")
+    _check(O.scale_bytes(widths) == 2 * n * (k // 64), "scale bytes")
+    _check(np.array_equal(O.unpack_lsb(buf, widths), codes), "pack/unpack roundtrip")
+
+
+ALL_PINS = [pin_eq1_golden, pin_level_grid, pin_grid_roundtrip, pin_quantizer_invariants,
+            pin_group_size_one, pin_integer_gemv, pin_exact_rational, pin_enumerated_codes,
+            pin_payload_accounting]

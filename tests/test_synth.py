@@ -1,0 +1,107 @@
+"""Seeded input generators: determinism, ranges, and the paper's printed
+distribution figures. CPU only."""
+
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+from synth import gen, workloads
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _paper_numbers():
+    out = {}
+    with open(os.path.join(GOLDEN, "paper_numbers.txt")) as f:
+        for line in f:
+            if line.startswith("#") or not line.strip():
+                continue
+            name, val, _ = [p.strip() for p in line.split("|")]
+            out[name] = val
+    return out
+
+
+def _mean_bits(dist):
+    return sum(p * b for p, b in zip(dist, (1, 2, 4, 8)))
+
+
+def test_distribution_means_match_paper():
+    pn = _paper_numbers()
+    assert abs(_mean_bits(synth.DIST_HEAD) - float(pn["head_mean_bits"])) < 0.005
+    assert abs(_mean_bits(synth.DIST_MLP0) - float(pn["mlp0_mean_bits"])) < 0.05
+    assert abs(synth.DIST_MAIN[0] - float(pn["one_bit_fraction"])) < 1e-9
+    tiers = [t.split(":") for t in pn["recipe_head_tiers"].split()]
+    recipe_mean = sum(float(f) * int(b) for f, b in tiers)
+    assert abs(recipe_mean - float(pn["recipe_head_mean_bits"])) < 1e-9
+    for d in (synth.DIST_MAIN, synth.DIST_MLP0, synth.DIST_HEAD):
+        assert abs(sum(d) - 1.0) < 1e-12
+
+
+def test_stack_shapes():
+    w = synth.workload("stack9b")
+    assert len(w.mats) == 32 * 7 + 1
+    assert abs(w.weights / 7.5e9 - 1) < 0.01
+    w1 = synth.workload("stack131m")
+    assert len(w1.mats) == 85 and abs(w1.weights / 1.10e8 - 1) < 0.01
+    w2 = synth.workload("stack1b")
+    assert len(w2.mats) == 155 and abs(w2.weights / 1.03e9 - 1) < 0.01
+    assert len(synth.sweep_points()) == 75
+    for m in w.mats + w1.mats + w2.mats:
+        assert m.k % 64 == 0
+
+
+def test_fmix32_tensor_matches_reference():
+    # the int64-tensor formulation must equal the plain 32-bit definition
+    key = gen.code_key((9, 9, 9))
+    idx = np.array([0, 1, 2, 12345, 2**31 - 1, 2**32 - 1], dtype=np.int64)
+    t = torch.from_numpy(idx)
+    h = gen._fmix32_t((gen._mul32(t, gen._WEYL) + key) & gen._M32)
+    ref = [gen.fmix32_py((int(i) * gen._WEYL + key) & gen._M32) for i in idx]
+    assert h.tolist() == ref
+    # published fmix32 fixed point: fmix32(0) == 0
+    assert gen.fmix32_py(0) == 0
+
+
+def test_codes_in_range_and_uniform():
+    spec = synth.workload("single768").mats[0]
+    inp = gen.matrix_inputs(spec, 1)
+    codes = gen.codes_torch(inp["widths"], inp["key"], spec.k).numpy()
+    wide = np.repeat(inp["widths"].astype(np.int64), 64, axis=1)
+    assert (codes.astype(np.int64) < (1 << wide)).all()
+    one = codes[wide == 1]
+    assert abs(one.mean() - 0.5) < 0.01
+    eight = codes[wide == 8]
+    assert abs(eight.mean() - 127.5) < 3
+    # a row subset reproduces the same rows
+    sub = gen.codes_torch(inp["widths"], inp["key"], spec.k, row0=100, nrows=7).numpy()
+    assert np.array_equal(sub, codes[100:107])
+
+
+def test_generators_deterministic():
+    spec = synth.workload("stack131m").mats[3]
+    a = gen.matrix_inputs(spec, 2)
+    b = gen.matrix_inputs(spec, 2)
+    for k in ("widths", "scales", "x_bits"):
+        assert np.array_equal(a[k], b[k])
+    assert a["key"] == b["key"]
+    c = gen.matrix_inputs(spec, 1)
+    assert np.array_equal(c["x_bits"][0], a["x_bits"][0])
+
+
+def test_bf16_rounding_matches_torch():
+    rng = np.random.default_rng(0)
+    v = rng.normal(0, 1, size=10000).astype(np.float32)
+    v[:4] = [1.0 + 2**-8, 1.0 + 3 * 2**-8, -0.0, 3.0e38]      # ties and edges
+    bits = gen.f32_to_bf16_bits(v)
+    ref = torch.from_numpy(v).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(bits, ref)
+    assert np.array_equal(gen.bf16_bits_to_f32(bits), torch.from_numpy(v).to(torch.bfloat16).float().numpy())
+
+
+def test_scales_fp16_positive():
+    rng = gen.rng_for((0, 0, 0))
+    s = gen.draw_scales(100, 10, rng)
+    assert s.dtype == np.float16 and (s > 0).all()
