@@ -1,0 +1,145 @@
+/*
+ * vbq.h — C ABI of the VBQ packed-weight GEMV library for GB300 (sm_103a).
+ *
+ * VBQ ("Variable Bit-width Quantization", arXiv 2607.02893) stores a weight
+ * matrix W (N x K, row-major) as contiguous groups of 64 weights along K
+ * (§3.1). Each group g of row n has its own width b[n][g] in {1, 2, 4, 8}
+ * (§3.2, the candidate set) and one FP16 scale s[n][g] (§3.1). A group
+ * holds 64 integer codes u of b bits each; its weights are s * L_b(u) with
+ *     L_1(u) = 2u - 1                       (sign times the absmean scale, §3.1)
+ *     L_b(u) = u - 2^(b-1)   for b >= 2     (the symmetric grid of Eq. 1)
+ * (the paper fixes the values, not the bit encoding; offset binary is this
+ * library's encoding and code 0 of a b >= 2 group decodes to -2^(b-1)).
+ *
+ * The library implements the inference step of §6: a fused dequantise-and-
+ * multiply y = W x that streams the packed codes and never writes wide
+ * weights to memory, for one activation vector (vbq_gemv) or a small batch
+ * of 2..16 (vbq_gemm_small). Activations are BF16, accumulation and outputs
+ * FP32.
+ *
+ * Conventions for every call:
+ *   - Pointers documented as "device" point to CUDA device memory of the
+ *     current device; "host" pointers to host memory.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream). Work is enqueued on it and the call returns without waiting,
+ *     unless the call says otherwise.
+ *   - Every call returns a vbq_status_t. Arguments are validated before any
+ *     work is enqueued; on an error nothing is enqueued and outputs are
+ *     untouched. Nothing aborts or throws across the ABI. vbq_last_error()
+ *     gives a human-readable detail of the calling thread's last error.
+ *   - Device arrays must be 16-byte aligned (VBQ_ERR_ALIGN otherwise).
+ */
+#ifndef VBQ_H
+#define VBQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int vbq_status_t;
+
+enum {
+    VBQ_OK              = 0,
+    VBQ_ERR_ARG         = -1,  /* null pointer, bad flag or bad count          */
+    VBQ_ERR_SHAPE       = -2,  /* N < 1, K < 64 or K not a multiple of 64      */
+    VBQ_ERR_WIDTH       = -3,  /* a bit-width outside {1, 2, 4, 8}              */
+    VBQ_ERR_CODE_RANGE  = -4,  /* a code >= 2^b of its group                    */
+    VBQ_ERR_ALIGN       = -5,  /* a device pointer not 16-byte aligned          */
+    VBQ_ERR_CUDA        = -6,  /* a CUDA runtime call or launch failed          */
+    VBQ_ERR_UNSUPPORTED = -7,  /* batch outside 1..16, or a size over a limit   */
+    VBQ_ERR_TIMEOUT     = -8,  /* a bounded device wait gave up                 */
+    VBQ_ERR_NOMEM       = -9   /* device or host allocation failed              */
+};
+
+/* Opaque packed matrix: host descriptor plus one device allocation. */
+typedef struct vbq_layout vbq_layout;
+
+/*
+ * vbq_pack — build the packed device layout of one matrix (§6: the export
+ * step that turns per-group codes into packed storage; §3.1 groups of 64).
+ *
+ *   codes        N x K uint8, row-major; codes[n*K + k] < 2^b of its group.
+ *   bitwidths    N x (K/64) uint8, each in {1, 2, 4, 8}.
+ *   scales_fp16  N x (K/64) IEEE half bit patterns.
+ *   N, K         rows and columns of W; K % 64 == 0 (callers zero-pad K, as
+ *                the paper pads MLP intermediates, §6).
+ *   src_on_device  0: the three arrays are host memory; 1: device memory.
+ *   stream       stream for the device work.
+ *   out          receives the new layout on VBQ_OK.
+ *
+ * Validates shape, widths and code ranges (VBQ_ERR_SHAPE / _WIDTH /
+ * _CODE_RANGE) before building anything. The layout owns its device memory
+ * until vbq_free. This call synchronises `stream` (it reads back counts to
+ * size the allocation) and may allocate temporary device memory.
+ */
+vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths,
+                      const uint16_t* scales_fp16, int64_t N, int64_t K,
+                      int src_on_device, void* stream, vbq_layout** out);
+
+/*
+ * vbq_packed_bytes — storage of a layout in bytes (§1, §6 storage accounting).
+ *   payload  packed codes: sum over groups of 64*b/8 (exactly; no padding).
+ *   scales   2 bytes per group.
+ *   meta     everything else the layout keeps on the device (width map, item
+ *            offsets, alignment padding).
+ * Any output pointer may be NULL.
+ */
+vbq_status_t vbq_packed_bytes(const vbq_layout* layout, size_t* payload,
+                              size_t* scales, size_t* meta);
+
+/* vbq_layout_shape — N and K of a layout (either pointer may be NULL). */
+vbq_status_t vbq_layout_shape(const vbq_layout* layout, int64_t* N, int64_t* K);
+
+/*
+ * vbq_dequant — unpack a layout back to per-group form (inverse of vbq_pack;
+ * the weights of §3.1 rebuilt from storage). All outputs are device arrays
+ * and any of them may be NULL:
+ *   codes_out      N x K uint8 codes (bit-exact copy of what was packed).
+ *   bitwidths_out  N x (K/64) uint8 widths.
+ *   scales_out     N x (K/64) FP16 bit patterns.
+ *   w_out          N x K float: s * L_b(u).
+ */
+vbq_status_t vbq_dequant(const vbq_layout* layout, uint8_t* codes_out,
+                         uint8_t* bitwidths_out, uint16_t* scales_out,
+                         float* w_out, void* stream);
+
+/*
+ * vbq_gemv — y = W x for one activation vector (§6, fused dequantise-and-
+ * multiply; batch 1 decode).
+ *   x  device, K BF16 bit patterns.
+ *   y  device, N floats; overwritten.
+ * Per output, |y - y_exact| stays within 2e-3 * sum_k |w_nk x_k| + 1e-5.
+ * The summation order is not fixed: results can differ in the last bits
+ * between calls. Calls on different streams may run concurrently on the same
+ * layout.
+ */
+vbq_status_t vbq_gemv(const vbq_layout* layout, const uint16_t* x, float* y,
+                      void* stream);
+
+/*
+ * vbq_gemm_small — Y = X W^T for a small batch (§6 product for B = 1..16).
+ *   X  device, B x K BF16 bit patterns, row-major.
+ *   Y  device, B x N floats, row-major; overwritten.
+ *   B  1..16 (VBQ_ERR_UNSUPPORTED otherwise).
+ * Same accuracy statement as vbq_gemv.
+ */
+vbq_status_t vbq_gemm_small(const vbq_layout* layout, const uint16_t* X, float* Y,
+                            int B, void* stream);
+
+/* vbq_free — release a layout and its device memory (NULL is accepted). */
+vbq_status_t vbq_free(vbq_layout* layout);
+
+/* vbq_status_string — static name of a status code. */
+const char* vbq_status_string(vbq_status_t status);
+
+/* vbq_last_error — detail of the calling thread's last failed call ("" if none). */
+const char* vbq_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VBQ_H */

@@ -1,0 +1,10 @@
+"""VBQ packed variable-bit-width GEMV for GB300 (sm_103a).
+
+The compute lives in libvbq.so (CUDA kernels behind the C ABI of
+include/vbq.h); this package is its thin Python binding.
+"""
+
+from .vbq import (  # noqa: F401
+    Layout, VbqError, load, vbq_pack, vbq_packed_bytes, vbq_layout_shape, vbq_dequant,
+    vbq_gemv, vbq_gemm_small, vbq_free, vbq_status_string, SIGNATURES, LIB_PATH,
+)

@@ -1,0 +1,305 @@
+// vbq_api.cu — the C ABI declared in include/vbq.h: argument validation,
+// layout planning and allocation, and kernel dispatch on the caller's stream.
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <vector>
+
+#include "../../include/vbq.h"
+#include "vbq_kernels.h"
+
+struct vbq_layout {
+    vbq::LayoutView view;     // device pointers and shape, passed to kernels
+    void* base = nullptr;     // the one device allocation
+    size_t alloc_bytes = 0;
+    size_t payload_bytes = 0, scale_bytes = 0, meta_bytes = 0;
+    int device = 0;
+};
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+vbq_status_t fail(vbq_status_t st, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return st;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Device buffers that vbq_pack frees on every exit path.
+struct TempBuffers {
+    std::vector<void*> ptrs;
+    ~TempBuffers() {
+        for (void* p : ptrs) cudaFree(p);
+    }
+    cudaError_t alloc(void** p, size_t bytes) {
+        cudaError_t e = cudaMalloc(p, bytes);
+        if (e == cudaSuccess) ptrs.push_back(*p);
+        return e;
+    }
+};
+
+#define VBQ_CUDA(call)                                                                     \
+    do {                                                                                   \
+        cudaError_t e_ = (call);                                                           \
+        if (e_ != cudaSuccess)                                                             \
+            return fail(e_ == cudaErrorMemoryAllocation ? VBQ_ERR_NOMEM : VBQ_ERR_CUDA,    \
+                        "%s: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__, __LINE__); \
+    } while (0)
+
+// Columns per slab: the largest C in {32, 16, 8, 4} that still gives at least
+// two units per SM; fewer columns if the matrix is narrower.
+int choose_slab_columns(int64_t nrb, int G, int sms) {
+    int C = 4;
+    for (int cand : {32, 16, 8}) {
+        int64_t S = (G + cand - 1) / cand;
+        if (nrb * S >= 2LL * sms) { C = cand; break; }
+    }
+    return std::min(C, G);
+}
+
+vbq_status_t check_layout(const vbq_layout* L) {
+    if (!L) return fail(VBQ_ERR_ARG, "layout is NULL");
+    if (!L->base) return fail(VBQ_ERR_ARG, "layout has no device storage");
+    return VBQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* vbq_status_string(vbq_status_t st) {
+    switch (st) {
+        case VBQ_OK: return "VBQ_OK";
+        case VBQ_ERR_ARG: return "VBQ_ERR_ARG";
+        case VBQ_ERR_SHAPE: return "VBQ_ERR_SHAPE";
+        case VBQ_ERR_WIDTH: return "VBQ_ERR_WIDTH";
+        case VBQ_ERR_CODE_RANGE: return "VBQ_ERR_CODE_RANGE";
+        case VBQ_ERR_ALIGN: return "VBQ_ERR_ALIGN";
+        case VBQ_ERR_CUDA: return "VBQ_ERR_CUDA";
+        case VBQ_ERR_UNSUPPORTED: return "VBQ_ERR_UNSUPPORTED";
+        case VBQ_ERR_TIMEOUT: return "VBQ_ERR_TIMEOUT";
+        case VBQ_ERR_NOMEM: return "VBQ_ERR_NOMEM";
+        default: return "VBQ_ERR_UNKNOWN";
+    }
+}
+
+const char* vbq_last_error(void) { return g_err; }
+
+vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint16_t* scales_fp16,
+                      int64_t N, int64_t K, int src_on_device, void* stream, vbq_layout** out) {
+    g_err[0] = 0;
+    if (!out) return fail(VBQ_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    if (!codes || !bitwidths || !scales_fp16) return fail(VBQ_ERR_ARG, "codes, bitwidths and scales must be non-NULL");
+    if (src_on_device != 0 && src_on_device != 1) return fail(VBQ_ERR_ARG, "src_on_device must be 0 or 1");
+    if (N < 1 || K < vbq::GROUP || K % vbq::GROUP != 0)
+        return fail(VBQ_ERR_SHAPE, "need N >= 1 and K a positive multiple of 64 (N=%lld K=%lld)",
+                    (long long)N, (long long)K);
+    if (N > (1LL << 31) - 1 || K / vbq::GROUP > (1LL << 20))
+        return fail(VBQ_ERR_UNSUPPORTED, "N or K too large (N=%lld K=%lld)", (long long)N, (long long)K);
+    if (src_on_device && !(aligned16(codes) && aligned16(bitwidths) && aligned16(scales_fp16)))
+        return fail(VBQ_ERR_ALIGN, "device inputs must be 16-byte aligned");
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int64_t G = K / vbq::GROUP;
+    const size_t ncodes = (size_t)N * (size_t)K, ngroups = (size_t)N * (size_t)G;
+    TempBuffers tmp;
+
+    const uint8_t* d_codes = codes;
+    const uint8_t* d_widths = bitwidths;
+    const uint16_t* d_scales = scales_fp16;
+    if (!src_on_device) {
+        void *pc, *pw, *ps;
+        VBQ_CUDA(tmp.alloc(&pc, ncodes));
+        VBQ_CUDA(tmp.alloc(&pw, ngroups));
+        VBQ_CUDA(tmp.alloc(&ps, ngroups * 2));
+        VBQ_CUDA(cudaMemcpyAsync(pc, codes, ncodes, cudaMemcpyHostToDevice, s));
+        VBQ_CUDA(cudaMemcpyAsync(pw, bitwidths, ngroups, cudaMemcpyHostToDevice, s));
+        VBQ_CUDA(cudaMemcpyAsync(ps, scales_fp16, ngroups * 2, cudaMemcpyHostToDevice, s));
+        d_codes = static_cast<uint8_t*>(pc);
+        d_widths = static_cast<uint8_t*>(pw);
+        d_scales = static_cast<uint16_t*>(ps);
+    }
+
+    // 1. validation on the device
+    void* d_err;
+    VBQ_CUDA(tmp.alloc(&d_err, sizeof(uint32_t)));
+    VBQ_CUDA(cudaMemsetAsync(d_err, 0, sizeof(uint32_t), s));
+    VBQ_CUDA(vbq::launch_validate(d_codes, d_widths, N, K, static_cast<uint32_t*>(d_err), s));
+    uint32_t h_err = 0;
+    VBQ_CUDA(cudaMemcpyAsync(&h_err, d_err, sizeof(uint32_t), cudaMemcpyDeviceToHost, s));
+    VBQ_CUDA(cudaStreamSynchronize(s));
+    if (h_err & 1u) return fail(VBQ_ERR_WIDTH, "a bit-width is not in {1,2,4,8}");
+    if (h_err & 2u) return fail(VBQ_ERR_CODE_RANGE, "a code is >= 2^b for its group's width");
+
+    // 2. plan: row blocks x slabs, per-unit item counts
+    int dev = 0, sms = 0;
+    VBQ_CUDA(cudaGetDevice(&dev));
+    VBQ_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    const int64_t nrb = (N + vbq::RB - 1) / vbq::RB;
+    const int C = choose_slab_columns(nrb, (int)G, sms);
+    const int64_t S = (G + C - 1) / C;
+    const int64_t units = nrb * S;
+    if (units > (1LL << 31) - 2) return fail(VBQ_ERR_UNSUPPORTED, "too many units");
+    void* d_counts;
+    VBQ_CUDA(tmp.alloc(&d_counts, (size_t)units * 4 * sizeof(uint32_t)));
+    VBQ_CUDA(vbq::launch_count(d_widths, N, (int)G, C, (int)S, (int)nrb, static_cast<uint32_t*>(d_counts), s));
+    std::vector<uint32_t> counts((size_t)units * 4);
+    VBQ_CUDA(cudaMemcpyAsync(counts.data(), d_counts, counts.size() * sizeof(uint32_t),
+                             cudaMemcpyDeviceToHost, s));
+    VBQ_CUDA(cudaStreamSynchronize(s));
+    std::vector<uint32_t> ustart(((size_t)units + 1) * 4);
+    uint64_t items[4] = {0, 0, 0, 0};
+    for (int64_t u = 0; u < units; ++u)
+        for (int w = 0; w < 4; ++w) {
+            ustart[u * 4 + w] = (uint32_t)items[w];
+            items[w] += counts[u * 4 + w];
+        }
+    for (int w = 0; w < 4; ++w) {
+        if (items[w] > 0xffffffffull) return fail(VBQ_ERR_UNSUPPORTED, "too many groups of one width");
+        ustart[units * 4 + w] = (uint32_t)items[w];
+    }
+    uint64_t total_items = items[0] + items[1] + items[2] + items[3];
+    if (total_items != ngroups) return fail(VBQ_ERR_CUDA, "item count mismatch (%llu vs %llu)",
+                                            (unsigned long long)total_items, (unsigned long long)ngroups);
+
+    // 3. one device allocation, sub-buffers 256-byte aligned
+    const size_t A = 256;
+    size_t off = 0;
+    const size_t map_off = off;
+    off = round_up(off + (size_t)units * C * vbq::MAP_WORDS * 4, A);
+    const size_t ustart_off = off;
+    off = round_up(off + ustart.size() * 4, A);
+    size_t pay_off[4], sc_off[4];
+    size_t payload_bytes = 0, scale_bytes = 0;
+    for (int w = 0; w < 4; ++w) {
+        pay_off[w] = off;
+        const size_t pb = (size_t)items[w] * 8 * (1u << w);
+        payload_bytes += pb;
+        off = round_up(off + pb + 64, A);      // 64 bytes of slack after each stream
+    }
+    for (int w = 0; w < 4; ++w) {
+        sc_off[w] = off;
+        scale_bytes += (size_t)items[w] * 2;
+        off = round_up(off + (size_t)items[w] * 2 + 16, A);
+    }
+    const size_t alloc_bytes = off;
+
+    vbq_layout* L = new (std::nothrow) vbq_layout();
+    if (!L) return fail(VBQ_ERR_NOMEM, "host allocation failed");
+    cudaError_t e = cudaMalloc(&L->base, alloc_bytes);
+    if (e != cudaSuccess) {
+        delete L;
+        return fail(VBQ_ERR_NOMEM, "cudaMalloc(%zu): %s", alloc_bytes, cudaGetErrorString(e));
+    }
+    auto bail = [&](vbq_status_t st, const char* what, cudaError_t err) {
+        cudaFree(L->base);
+        delete L;
+        return fail(st, "%s: %s", what, cudaGetErrorString(err));
+    };
+    uint8_t* base = static_cast<uint8_t*>(L->base);
+    L->alloc_bytes = alloc_bytes;
+    L->payload_bytes = payload_bytes;
+    L->scale_bytes = scale_bytes;
+    L->meta_bytes = alloc_bytes - payload_bytes - scale_bytes;
+    L->device = dev;
+    vbq::LayoutView& V = L->view;
+    V.map = reinterpret_cast<uint32_t*>(base + map_off);
+    V.ustart = reinterpret_cast<uint32_t*>(base + ustart_off);
+    uint8_t* pay[4];
+    uint16_t* sc[4];
+    for (int w = 0; w < 4; ++w) {
+        pay[w] = base + pay_off[w];
+        sc[w] = reinterpret_cast<uint16_t*>(base + sc_off[w]);
+        V.payload[w] = pay[w];
+        V.scales[w] = sc[w];
+    }
+    V.N = N;
+    V.K = K;
+    V.G = (int)G;
+    V.C = C;
+    V.S = (int)S;
+    V.nrb = (int)nrb;
+    V.units = (int)units;
+
+    if ((e = cudaMemsetAsync(L->base, 0, alloc_bytes, s)) != cudaSuccess) return bail(VBQ_ERR_CUDA, "memset", e);
+    if ((e = cudaMemcpyAsync(const_cast<uint32_t*>(V.ustart), ustart.data(), ustart.size() * 4,
+                             cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return bail(VBQ_ERR_CUDA, "ustart copy", e);
+    if ((e = vbq::launch_scatter(d_codes, d_widths, d_scales, V, const_cast<uint32_t*>(V.map), pay, sc, s)) !=
+        cudaSuccess)
+        return bail(VBQ_ERR_CUDA, "scatter launch", e);
+    if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return bail(VBQ_ERR_CUDA, "pack", e);
+    *out = L;
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_packed_bytes(const vbq_layout* L, size_t* payload, size_t* scales, size_t* meta) {
+    vbq_status_t st = check_layout(L);
+    if (st) return st;
+    if (payload) *payload = L->payload_bytes;
+    if (scales) *scales = L->scale_bytes;
+    if (meta) *meta = L->meta_bytes;
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_layout_shape(const vbq_layout* L, int64_t* N, int64_t* K) {
+    vbq_status_t st = check_layout(L);
+    if (st) return st;
+    if (N) *N = L->view.N;
+    if (K) *K = L->view.K;
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_dequant(const vbq_layout* L, uint8_t* codes_out, uint8_t* bitwidths_out,
+                         uint16_t* scales_out, float* w_out, void* stream) {
+    g_err[0] = 0;
+    vbq_status_t st = check_layout(L);
+    if (st) return st;
+    if (!aligned16(codes_out) || !aligned16(bitwidths_out) || !aligned16(scales_out) || !aligned16(w_out))
+        return fail(VBQ_ERR_ALIGN, "outputs must be 16-byte aligned");
+    if (!codes_out && !bitwidths_out && !scales_out && !w_out) return VBQ_OK;
+    VBQ_CUDA(vbq::launch_dequant(L->view, codes_out, bitwidths_out, scales_out, w_out,
+                                 static_cast<cudaStream_t>(stream)));
+    return VBQ_OK;
+}
+
+static vbq_status_t run_product(const vbq_layout* L, const uint16_t* X, float* Y, int B, void* stream) {
+    g_err[0] = 0;
+    vbq_status_t st = check_layout(L);
+    if (st) return st;
+    if (!X || !Y) return fail(VBQ_ERR_ARG, "x and y must be non-NULL");
+    if (B < 1 || B > vbq::MAX_BATCH) return fail(VBQ_ERR_UNSUPPORTED, "batch %d outside 1..16", B);
+    if (!aligned16(X) || !aligned16(Y)) return fail(VBQ_ERR_ALIGN, "x and y must be 16-byte aligned");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (L->view.S > 1)
+        VBQ_CUDA(cudaMemsetAsync(Y, 0, (size_t)B * (size_t)L->view.N * sizeof(float), s));
+    VBQ_CUDA(vbq::launch_gemv(L->view, X, Y, B, s));
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_gemv(const vbq_layout* L, const uint16_t* x, float* y, void* stream) {
+    return run_product(L, x, y, 1, stream);
+}
+
+vbq_status_t vbq_gemm_small(const vbq_layout* L, const uint16_t* X, float* Y, int B, void* stream) {
+    return run_product(L, X, Y, B, stream);
+}
+
+vbq_status_t vbq_free(vbq_layout* L) {
+    if (!L) return VBQ_OK;
+    cudaError_t e = L->base ? cudaFree(L->base) : cudaSuccess;
+    delete L;
+    if (e != cudaSuccess) return fail(VBQ_ERR_CUDA, "cudaFree: %s", cudaGetErrorString(e));
+    return VBQ_OK;
+}
+
+}  // extern "C"

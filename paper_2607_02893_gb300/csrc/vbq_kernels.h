@@ -1,0 +1,26 @@
+// vbq_kernels.h — launchers of the library's CUDA kernels (internal; called by
+// the C ABI in vbq_api.cu). Each returns the cudaError_t of its launch.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+#include "vbq_common.cuh"
+
+namespace vbq {
+
+// Pack-time kernels (vbq_pack.cu).
+cudaError_t launch_validate(const uint8_t* codes, const uint8_t* widths, int64_t N, int64_t K,
+                            uint32_t* err_flags, cudaStream_t s);
+cudaError_t launch_count(const uint8_t* widths, int64_t N, int G, int C, int S, int nrb,
+                         uint32_t* counts, cudaStream_t s);
+cudaError_t launch_scatter(const uint8_t* codes, const uint8_t* widths, const uint16_t* scales,
+                           const LayoutView& L, uint32_t* map, uint8_t* const payload[4],
+                           uint16_t* const scales_out[4], cudaStream_t s);
+cudaError_t launch_dequant(const LayoutView& L, uint8_t* codes_out, uint8_t* widths_out,
+                           uint16_t* scales_out, float* w_out, cudaStream_t s);
+
+// Products (vbq_gemv.cu). Y is B x N; `accumulate` means Y was zeroed and
+// units add into it (more than one slab per row).
+cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s);
+
+}  // namespace vbq

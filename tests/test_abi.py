@@ -1,0 +1,87 @@
+"""The C-ABI library: it loads, exports every symbol the header declares, and
+rejects bad arguments on the host before touching the GPU. CPU only."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2607_02893_gb300 as vbq
+from paper_2607_02893_gb300 import vbq as binding
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "vbq.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_02893_gb300 import build
+    build.build()
+    return vbq.load()
+
+
+def header_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(vbq_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = header_functions()
+    for required in ("vbq_pack", "vbq_dequant", "vbq_gemv", "vbq_gemm_small", "vbq_free"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = header_functions()
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, f"missing exports: {missing}"
+    assert set(names) == set(binding.SIGNATURES), "binding and header disagree"
+
+
+def test_status_strings(lib):
+    assert vbq.vbq_status_string(0) == "VBQ_OK"
+    for code, name in binding.STATUS_NAMES.items():
+        assert vbq.vbq_status_string(code) == name
+    assert vbq.vbq_status_string(-1234) == "VBQ_ERR_UNKNOWN"
+
+
+def _pack_raw(lib, codes, widths, scales, n, k, on_dev):
+    out = ctypes.c_void_p(12345)
+    st = lib.vbq_pack(codes, widths, scales, n, k, on_dev, None, ctypes.byref(out))
+    return st, out.value
+
+
+def test_pack_rejects_bad_arguments_on_host(lib):
+    buf = ctypes.create_string_buffer(64)
+    p = ctypes.addressof(buf)
+    assert lib.vbq_pack(p, p, p, 1, 64, 0, None, None) == -1          # out NULL
+    st, out = _pack_raw(lib, None, p, p, 1, 64, 0)
+    assert st == -1 and out is None                                      # codes NULL, out cleared
+    assert _pack_raw(lib, p, p, p, 1, 64, 2)[0] == -1                   # bad flag
+    assert _pack_raw(lib, p, p, p, 0, 64, 0)[0] == -2                   # N < 1
+    assert _pack_raw(lib, p, p, p, 4, 65, 0)[0] == -2                   # K % 64
+    assert _pack_raw(lib, p, p, p, 4, 0, 0)[0] == -2
+    assert _pack_raw(lib, p + 1, p, p, 4, 64, 1)[0] == -5               # misaligned device ptr
+    assert b"16-byte" in lib.vbq_last_error()
+
+
+def test_calls_reject_null_layout(lib):
+    assert lib.vbq_gemv(None, None, None, None) == -1
+    assert lib.vbq_gemm_small(None, None, None, 4, None) == -1
+    assert lib.vbq_dequant(None, None, None, None, None, None) == -1
+    assert lib.vbq_packed_bytes(None, None, None, None) == -1
+    assert lib.vbq_layout_shape(None, None, None) == -1
+    assert lib.vbq_free(None) == 0
+
+
+def test_binding_raises_typed_errors(lib):
+    with pytest.raises(vbq.VbqError) as ei:
+        vbq.vbq_pack(0, 0, 0, N=4, K=64, src_on_device=0)
+    assert ei.value.name == "VBQ_ERR_ARG"
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(RuntimeError, match="not built"):
+        binding.load(str(tmp_path / "libvbq.so"))

@@ -1,0 +1,201 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Codes, widths and scales must round-trip bit-exactly; every product output
+must satisfy |y - y_ref| <= 2e-3 * sum_k |w_nk x_k| + 1e-5 against the fp64
+oracle (the accuracy bound the library states)."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2607_02893_gb300 as vbq
+import synth
+from vbq_cases import Matrix, bits_to_i16, scales_to_i16
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2607_02893_gb300 import build
+    build.build()
+    vbq.load()
+    torch.cuda.init()
+
+
+def _pack(m: Matrix):
+    return vbq.vbq_pack(*m.device_args(DEV))
+
+
+def _gemv(layout, m: Matrix, batch=1):
+    x = bits_to_i16(m.x_bits[:batch]).to(DEV)
+    y = torch.full((batch, m.n), float("nan"), dtype=torch.float32, device=DEV)
+    if batch == 1:
+        vbq.vbq_gemv(layout, x[0], y[0])
+    else:
+        vbq.vbq_gemm_small(layout, x, y, batch)
+    torch.cuda.synchronize()
+    return y.cpu().numpy()
+
+
+def _assert_bound(y, m: Matrix, batch=1, rows=None):
+    codes = m.codes.cpu().numpy() if rows is None else m.rows_codes_cpu(rows)
+    widths = m.widths if rows is None else m.widths[rows]
+    scales = m.scales if rows is None else m.scales[rows]
+    y_ref, a_ref = oracle.gemv(codes, widths, scales, m.x()[:batch])
+    got = y if rows is None else y[:, rows]
+    ok = oracle.within_bound(got, y_ref, a_ref)
+    if not ok.all():
+        bad = np.argwhere(~ok)[:5]
+        detail = [(int(b), int(r), float(got[b, r]), float(y_ref[b, r]), float(a_ref[b, r])) for b, r in bad]
+        raise AssertionError(f"{int((~ok).sum())} outputs outside the bound; first: {detail}")
+
+
+SHAPES = [(768, 768), (1, 64), (129, 832), (300, 4096), (1000, 2048), (257, 64 * 37), (128, 64 * 33)]
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: f"{s[0]}x{s[1]}")
+def test_roundtrip_bitexact(shape):
+    n, k = shape
+    m = Matrix(n, k, seed_path=(99, n, k))
+    layout = _pack(m)
+    g = k // 64
+    codes = torch.full((n, k), 255, dtype=torch.uint8, device=DEV)
+    widths = torch.zeros((n, g), dtype=torch.uint8, device=DEV)
+    scales = torch.zeros((n, g), dtype=torch.int16, device=DEV)
+    w = torch.full((n, k), float("nan"), dtype=torch.float32, device=DEV)
+    vbq.vbq_dequant(layout, codes, widths, scales, w)
+    torch.cuda.synchronize()
+    assert torch.equal(codes.cpu(), m.codes.cpu())
+    assert np.array_equal(widths.cpu().numpy(), m.widths)
+    assert np.array_equal(scales.cpu().numpy().view(np.uint16), m.scales.view(np.uint16))
+    w_ref = oracle.dequant(m.codes.numpy(), m.widths, m.scales)
+    assert np.array_equal(w.cpu().numpy().astype(np.float64), w_ref)
+    payload, sc, meta = vbq.vbq_packed_bytes(layout)
+    assert payload == oracle.payload_bytes(m.widths)
+    assert sc == oracle.scale_bytes(m.widths)
+    assert vbq.vbq_layout_shape(layout) == (n, k)
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: f"{s[0]}x{s[1]}")
+@pytest.mark.parametrize("dist", ["main", "mlp0", "head"])
+def test_gemv_parity(shape, dist):
+    n, k = shape
+    d = {"main": synth.DIST_MAIN, "mlp0": synth.DIST_MLP0, "head": synth.DIST_HEAD}[dist]
+    m = Matrix(n, k, dist=d, seed_path=(98, n, k))
+    layout = _pack(m)
+    _assert_bound(_gemv(layout, m), m)
+
+
+@pytest.mark.parametrize("batch", [2, 3, 4, 5, 8, 13, 16])
+def test_gemm_small_parity(batch):
+    m = Matrix(513, 1024, seed_path=(97, batch, 0), batch=16)
+    layout = _pack(m)
+    _assert_bound(_gemv(layout, m, batch), m, batch)
+
+
+@pytest.mark.parametrize("b", [1, 2, 4, 8])
+def test_single_width(b):
+    d = tuple(1.0 if w == b else 0.0 for w in (1, 2, 4, 8))
+    m = Matrix(384, 4096, dist=d, seed_path=(96, b, 0), batch=4)
+    layout = _pack(m)
+    _assert_bound(_gemv(layout, m), m)
+    _assert_bound(_gemv(layout, m, 4), m, 4)
+
+
+def test_integer_all8_exact():
+    rng = np.random.default_rng(5)
+    n, k = 200, 1024
+    codes = rng.integers(0, 256, size=(n, k)).astype(np.uint8)
+    widths = np.full((n, k // 64), 8, np.uint8)
+    scales = np.ones((n, k // 64), np.float16)
+    xi = rng.integers(-8, 9, size=(3, k))
+    layout = vbq.vbq_pack(torch.from_numpy(codes).to(DEV), torch.from_numpy(widths).to(DEV),
+                          scales_to_i16(scales).to(DEV))
+    x_bits = bits_to_i16(((xi.astype(np.float32).view(np.uint32)) >> 16).astype(np.uint16)).to(DEV)
+    y = torch.empty((3, n), dtype=torch.float32, device=DEV)
+    vbq.vbq_gemm_small(layout, x_bits, y, 3)
+    y1 = torch.empty(n, dtype=torch.float32, device=DEV)
+    vbq.vbq_gemv(layout, x_bits[0], y1)
+    exp = ((codes.astype(np.int64) - 128) @ xi.T).T
+    assert np.array_equal(y.cpu().numpy().astype(np.int64), exp)
+    assert np.array_equal(y1.cpu().numpy().astype(np.int64), exp[0])
+
+
+@pytest.mark.parametrize("b", [2, 4, 8])
+def test_all_zero_level(b):
+    n, k = 256, 2048
+    codes = np.full((n, k), 1 << (b - 1), np.uint8)
+    widths = np.full((n, k // 64), b, np.uint8)
+    m = Matrix(n, k, seed_path=(95, b, 0))
+    layout = vbq.vbq_pack(torch.from_numpy(codes).to(DEV), torch.from_numpy(widths).to(DEV),
+                          scales_to_i16(m.scales).to(DEV))
+    x = bits_to_i16(m.x_bits).to(DEV)
+    y = torch.empty(n, dtype=torch.float32, device=DEV)
+    vbq.vbq_gemv(layout, x[0], y)
+    assert float(y.abs().max()) <= 1e-5
+
+
+def test_one_hot_exact():
+    m = Matrix(640, 1024, seed_path=(94, 0, 0))
+    layout = _pack(m)
+    w_ref = oracle.dequant(m.codes.numpy(), m.widths, m.scales)
+    for j in (0, 1, 63, 64, 511, 1023):
+        xb = np.zeros(1024, np.uint16)
+        xb[j] = 0x3F80                       # bf16 1.0
+        x = bits_to_i16(xb).to(DEV)
+        y = torch.empty(640, dtype=torch.float32, device=DEV)
+        vbq.vbq_gemv(layout, x, y)
+        torch.cuda.synchronize()
+        assert np.array_equal(y.cpu().numpy().astype(np.float64), w_ref[:, j])
+
+
+def test_host_source_pack_matches_device_source():
+    m = Matrix(300, 1536, seed_path=(93, 0, 0))
+    l_dev = _pack(m)
+    l_host = vbq.vbq_pack(m.codes, torch.from_numpy(m.widths), scales_to_i16(m.scales),
+                          src_on_device=0)
+    y1 = _gemv(l_dev, m)
+    y2 = _gemv(l_host, m)
+    _assert_bound(y2, m)
+    assert vbq.vbq_packed_bytes(l_dev) == vbq.vbq_packed_bytes(l_host)
+    c = torch.empty((m.n, m.k), dtype=torch.uint8, device=DEV)
+    vbq.vbq_dequant(l_host, codes_out=c)
+    torch.cuda.synchronize()
+    assert torch.equal(c.cpu(), m.codes)
+    assert np.isfinite(y1).all()
+
+
+def test_pack_rejects_bad_widths_and_codes():
+    m = Matrix(64, 256, seed_path=(92, 0, 0))
+    codes, widths, scales = m.device_args(DEV)
+    bad_w = widths.clone()
+    bad_w[3, 1] = 3
+    with pytest.raises(vbq.VbqError) as e:
+        vbq.vbq_pack(codes, bad_w, scales)
+    assert e.value.name == "VBQ_ERR_WIDTH"
+    bad_c = codes.clone()
+    w1 = (widths == 1).nonzero()[0]
+    bad_c[int(w1[0]), int(w1[1]) * 64 + 5] = 2
+    with pytest.raises(vbq.VbqError) as e:
+        vbq.vbq_pack(bad_c, widths, scales)
+    assert e.value.name == "VBQ_ERR_CODE_RANGE"
+    layout = vbq.vbq_pack(codes, widths, scales)
+    x = torch.zeros(256, dtype=torch.int16, device=DEV)
+    y = torch.zeros(64, dtype=torch.float32, device=DEV)
+    with pytest.raises(vbq.VbqError) as e:
+        vbq.vbq_gemm_small(layout, x, y, 17)
+    assert e.value.name == "VBQ_ERR_UNSUPPORTED"
+    with pytest.raises(vbq.VbqError) as e:
+        vbq.vbq_gemv(layout, x[1:], y)
+    assert e.value.name == "VBQ_ERR_ALIGN"
+
+
+def test_empty_output_dequant_is_noop():
+    m = Matrix(64, 128, seed_path=(91, 0, 0))
+    layout = _pack(m)
+    vbq.vbq_dequant(layout)
+    torch.cuda.synchronize()
