@@ -1,0 +1,454 @@
+"""Benchmark: batch-1 VBQ decode GEMV over a synthetic decoder linear stack.
+
+One step = one token through every linear layer of the stack (per layer Q, K,
+V, O, gate, up, down, then the LM head), each a packed VBQ GEMV run by
+libvbq.so on one stream, replayed from a CUDA graph. Weights are
+random-but-seeded (synthetic) with the per-projection width distributions of
+the workload; every GEMV has its own resident BF16 activation vector.
+
+Printed JSON line (rank 0):
+  value         algorithmic HBM GB/s of the whole step: sum over GEMVs of
+                (packed payload + FP16 scales + x + y bytes) / step time.
+  roofline      the GEMV kernel (the only kernel of the step): per-launch
+                algorithmic bytes / CUDA-event launch duration, against the
+                measured copy bandwidth.
+  e2e           the same metric with the step's activations copied in from
+                pinned host memory and the head's logits copied back, inside
+                the timed region.
+  cpu_baseline  the CPU oracle (numpy fp64) on a bounded row sample of the
+                same stack.
+
+`--impl reference` times the CPU oracle alone on the same workload (rank 0).
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = ("batch-1 decode GEMV achieved HBM GB/s (% of ~8 TB/s) and layer-stack tokens/s")
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=300)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default="stack9b")
+    p.add_argument("--batch", type=int, default=1)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--event-ring", type=int, default=4)
+    return p.parse_args()
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def algorithmic_bytes(widths: np.ndarray, n: int, k: int, batch: int) -> int:
+    """Packed payload + FP16 scales + BF16 x + FP32 y bytes of one product."""
+    payload = int(widths.astype(np.int64).sum()) * 8
+    return payload + 2 * widths.size + 2 * k * batch + 4 * n * batch
+
+
+# ---------------------------------------------------------------------------
+# clocks sampler (nvidia-smi during the timed region)
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, smax, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = max(smax, float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle leg
+# ---------------------------------------------------------------------------
+
+ORACLE_WEIGHTS_PER_S = 2.5e7     # rough single-core rate of the numpy oracle, for sizing samples
+
+
+def oracle_block(spec, batch: int, rows: int, seed: int):
+    """Time the oracle on a random contiguous block of `rows` rows of one matrix.
+
+    Returns (seconds, algorithmic bytes of the block)."""
+    import oracle
+    from synth import gen
+    rng = np.random.default_rng(seed)
+    inp = gen.matrix_inputs(spec, batch)
+    r = max(1, min(rows, spec.n))
+    row0 = int(rng.integers(0, spec.n - r + 1))
+    codes = gen.codes_torch(inp["widths"], inp["key"], spec.k, row0=row0, nrows=r,
+                            device="cpu").numpy()
+    w, s = inp["widths"][row0:row0 + r], inp["scales"][row0:row0 + r]
+    x = gen.bf16_bits_to_f32(inp["x_bits"])
+    t0 = time.perf_counter()
+    oracle.gemv(codes, w, s, x)
+    return time.perf_counter() - t0, algorithmic_bytes(w, r, spec.k, batch)
+
+
+def oracle_leg(work, batch: int, budget_s: float, seed: int = 0):
+    """The oracle on one row block of every matrix, about `budget_s` seconds in all."""
+    per_mat_weights = budget_s * ORACLE_WEIGHTS_PER_S / len(work.mats)
+    t, nb, rows_done = 0.0, 0, 0
+    for i, spec in enumerate(work.mats):
+        rows = max(1, int(per_mat_weights / spec.k))
+        dt, b = oracle_block(spec, batch, rows, seed + i)
+        t += dt
+        nb += b
+        rows_done += min(rows, spec.n)
+    frac = rows_done / sum(m.n for m in work.mats)
+    return t, nb, frac
+
+
+# ---------------------------------------------------------------------------
+# GPU leg
+# ---------------------------------------------------------------------------
+
+def setup_stack(work, batch, dev):
+    import torch
+    import paper_2607_02893_gb300 as vbq
+    from synth import gen
+    layouts, xs, ys, nbytes, host_x = [], [], [], [], []
+    for spec in work.mats:
+        inp = gen.matrix_inputs(spec, batch)
+        wd = torch.from_numpy(inp["widths"]).to(dev)
+        codes = gen.codes_torch(wd, inp["key"], spec.k, device=dev)
+        sc = torch.from_numpy(inp["scales"].view(np.uint16).astype(np.int16)).to(dev)
+        layouts.append(vbq.vbq_pack(codes, wd, sc))
+        del codes, wd, sc
+        xb = inp["x_bits"].astype(np.uint16).view(np.int16)
+        host_x.append(xb)
+        xs.append(torch.from_numpy(xb.copy()).to(dev))
+        ys.append(torch.empty((batch, spec.n), dtype=torch.float32, device=dev))
+        nbytes.append(algorithmic_bytes(inp["widths"], spec.n, spec.k, batch))
+    torch.cuda.synchronize()
+    return layouts, xs, ys, nbytes, host_x
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import paper_2607_02893_gb300 as vbq
+    import synth
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    vbq.load()
+    work = synth.workload(args.workload, args.batch)
+    B = args.batch
+    layouts, xs, ys, nbytes, host_x = setup_stack(work, B, dev)
+    step_bytes = sum(nbytes)
+    stream = torch.cuda.Stream(device=dev)
+
+    def launch_all(events=None):
+        for i, lay in enumerate(layouts):
+            if events is not None:
+                events[i][0].record(stream)
+            if B == 1:
+                vbq.vbq_gemv(lay, xs[i][0], ys[i][0], stream=stream)
+            else:
+                vbq.vbq_gemm_small(lay, xs[i], ys[i], B, stream=stream)
+            if events is not None:
+                events[i][1].record(stream)
+
+    # warm the kernels (sets function attributes outside capture)
+    with torch.cuda.stream(stream):
+        launch_all()
+    torch.cuda.synchronize()
+
+    # the step captured once as a CUDA graph
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        launch_all()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            graph.replay()
+    torch.cuda.synchronize()
+
+    # --- timed region: device-resident inputs --------------------------------
+    clocks = ClockSampler(int(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0])
+                          if "CUDA_VISIBLE_DEVICES" in os.environ else local_rank)
+    clocks.start()
+    time.sleep(0.3)
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            graph.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+
+    # --- per-launch kernel durations: the same steps launched eagerly with a
+    # CUDA event pair around every GEMV on its stream ---------------------------
+    ring = max(1, args.event_ring)
+    events = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in layouts] for _ in range(ring)]
+    with torch.cuda.stream(stream):
+        for r in range(ring):
+            launch_all(events[r])
+    torch.cuda.synchronize()
+    durs = [ev[i][0].elapsed_time(ev[i][1]) for ev in events for i in range(len(layouts))]
+    kernel_ms_per_step = sum(durs) / ring
+
+    # --- e2e: host activations in, head logits out ------------------------------
+    pinned_x = torch.from_numpy(np.concatenate([h.reshape(-1) for h in host_x])).pin_memory()
+    dev_x_flat = torch.empty_like(pinned_x, device=dev)
+    head_out = torch.empty(ys[-1].shape, dtype=torch.float32).pin_memory()
+    offs = np.cumsum([0] + [h.size for h in host_x])
+    xs_views = [dev_x_flat[offs[i]:offs[i + 1]].view(xs[i].shape) for i in range(len(xs))]
+    g_e2e = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_e2e, stream=stream):
+        for i, lay in enumerate(layouts):
+            if B == 1:
+                vbq.vbq_gemv(lay, xs_views[i][0], ys[i][0], stream=stream)
+            else:
+                vbq.vbq_gemm_small(lay, xs_views[i], ys[i], B, stream=stream)
+    h2d = pinned_x.numel() * 2
+    d2h = head_out.numel() * 4
+    e2e_steps = max(3, args.steps // 4)
+    for i in range(3):
+        with torch.cuda.stream(stream):
+            dev_x_flat.copy_(pinned_x, non_blocking=True)
+            g_e2e.replay()
+            head_out.copy_(ys[-1], non_blocking=True)
+    torch.cuda.synchronize()
+    barrier()
+    t0 = time.perf_counter()
+    for i in range(e2e_steps):
+        with torch.cuda.stream(stream):
+            dev_x_flat.copy_(pinned_x, non_blocking=True)
+            g_e2e.replay()
+            head_out.copy_(ys[-1], non_blocking=True)
+        stream.synchronize()
+        _ = float(head_out[0, 0])          # the result is read on the host every step
+    e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
+    barrier()
+
+    ms_max, e2e_max = ms, e2e_ms
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_max, e2e_max = float(t[0]), float(t[1])
+
+    gbs = step_bytes * world / (ms_max * 1e-3) / 1e9
+    tok_s = B * world / (ms_max * 1e-3)
+    peak, peak_kind = measured_peak()
+    kernel_gbs = step_bytes / (kernel_ms_per_step * 1e-3) / 1e9
+    launches = len(layouts)
+    result = {
+        "metric": METRIC,
+        "value": round(gbs, 1),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_max, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic",
+        "config": {
+            "workload": args.workload,
+            "batch": B,
+            "gemvs_per_step": launches,
+            "weights": work.weights,
+            "algorithmic_bytes_per_step": step_bytes,
+            "tokens_per_s": round(tok_s, 1),
+            "pct_of_nominal_8TBs": round(100 * gbs / world / NOMINAL_HBM_GBS, 2),
+            "l2": "inputs larger than L2: each step streams the whole packed stack once",
+            "activations": "BF16 N(0,1), one resident vector per GEMV",
+        },
+        "roofline": {
+            "bound": "hbm",
+            "kernel": "gemv_kernel<1> (vbq_gemv)",
+            "achieved": round(kernel_gbs, 1),
+            "peak": peak,
+            "peak_kind": peak_kind,
+            "unit": "GB/s",
+            "frac": round(kernel_gbs / peak, 4),
+            "traffic": None,
+            "launches_timed": launches * ring,
+            "avg_launch_us": round(kernel_ms_per_step * 1e3 / launches, 3),
+        },
+        "e2e": {
+            "value": round(step_bytes * world / (e2e_max * 1e-3) / 1e9, 1),
+            "unit": "GB/s",
+            "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h),
+            "tokens_per_s": round(B * world / (e2e_max * 1e-3), 1),
+        },
+        "gpu_launches": launches * args.steps,
+        "clocks": clk,
+    }
+    return result, work
+
+
+def run_reference(args):
+    """The CPU oracle as the reference arm: step s runs the oracle on a random
+    row block of matrix s mod M, sized so that the whole run takes a few minutes."""
+    import synth
+    work = synth.workload(args.workload, args.batch)
+    budget_per_step = min(2.0, 150.0 / max(1, args.steps + args.warmup))
+    t, nbytes, rows_seen = 0.0, 0, 0
+    for s in range(args.warmup + args.steps):
+        spec = work.mats[s % len(work.mats)]
+        rows = max(1, int(budget_per_step * ORACLE_WEIGHTS_PER_S / spec.k))
+        dt, nb = oracle_block(spec, args.batch, rows, seed=1000 + s)
+        if s >= args.warmup:
+            t += dt
+            nbytes += nb
+            rows_seen += min(rows, spec.n)
+    gbs = nbytes / t / 1e9
+    token_bytes = sum(algorithmic_bytes_est(m, args.batch) for m in work.mats)
+    ms_per_step = token_bytes / (gbs * 1e9) * 1e3          # one full token at that rate
+    sample = (f"per step one random contiguous row block (about {budget_per_step:.2f} s of work) of one "
+              f"matrix, cycling through the {len(work.mats)} matrices; {rows_seen} rows in all")
+    return {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": round(gbs, 4),
+        "unit": "GB/s",
+        "n_gpus": 1,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": args.workload, "batch": args.batch,
+                   "tokens_per_s": round(args.batch / (ms_per_step * 1e-3), 6)},
+        "cpu_baseline": {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": round(gbs, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def algorithmic_bytes_est(spec, batch: int) -> int:
+    """Algorithmic bytes of one matrix from its drawn widths."""
+    from synth import gen
+    rng = gen.rng_for(spec.seed_path)
+    widths = gen.draw_widths(spec.n, spec.k // 64, spec.dist, rng)
+    return algorithmic_bytes(widths, spec.n, spec.k, batch)
+
+
+def main():
+    args = parse()
+    if args.warmup < 3:
+        args.warmup = 3
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args)), flush=True)
+        return
+
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    result, work = run_ours(args, rank, world, local_rank)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        t, nb, frac = oracle_leg(work, args.batch, budget_s=12.0)
+        result["cpu_baseline"] = {
+            "value": round(nb / t / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": f"one random contiguous row block of each of the {len(work.mats)} matrices "
+                      f"({frac * 100:.3f}% of all rows), {t:.1f} s of numpy fp64 on one host core",
+        }
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+        dist.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -54,17 +54,6 @@ struct TempBuffers {
                         "%s: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__, __LINE__); \
     } while (0)
 
-// Columns per slab: the largest C in {32, 16, 8, 4} that still gives at least
-// two units per SM; fewer columns if the matrix is narrower.
-int choose_slab_columns(int64_t nrb, int G, int sms) {
-    int C = 4;
-    for (int cand : {32, 16, 8}) {
-        int64_t S = (G + cand - 1) / cand;
-        if (nrb * S >= 2LL * sms) { C = cand; break; }
-    }
-    return std::min(C, G);
-}
-
 vbq_status_t check_layout(const vbq_layout* L) {
     if (!L) return fail(VBQ_ERR_ARG, "layout is NULL");
     if (!L->base) return fail(VBQ_ERR_ARG, "layout has no device storage");
@@ -140,58 +129,71 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     if (h_err & 1u) return fail(VBQ_ERR_WIDTH, "a bit-width is not in {1,2,4,8}");
     if (h_err & 2u) return fail(VBQ_ERR_CODE_RANGE, "a code is >= 2^b for its group's width");
 
-    // 2. plan: row blocks x slabs, per-unit item counts
+    // 2. plan: row blocks x slabs. Take the widest slab (C in 16..1) that gives
+    // at least three units per SM and whose largest unit blob fits a stage.
     int dev = 0, sms = 0;
     VBQ_CUDA(cudaGetDevice(&dev));
     VBQ_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     const int64_t nrb = (N + vbq::RB - 1) / vbq::RB;
-    const int C = choose_slab_columns(nrb, (int)G, sms);
-    const int64_t S = (G + C - 1) / C;
-    const int64_t units = nrb * S;
-    if (units > (1LL << 31) - 2) return fail(VBQ_ERR_UNSUPPORTED, "too many units");
-    void* d_counts;
-    VBQ_CUDA(tmp.alloc(&d_counts, (size_t)units * 4 * sizeof(uint32_t)));
-    VBQ_CUDA(vbq::launch_count(d_widths, N, (int)G, C, (int)S, (int)nrb, static_cast<uint32_t*>(d_counts), s));
-    std::vector<uint32_t> counts((size_t)units * 4);
-    VBQ_CUDA(cudaMemcpyAsync(counts.data(), d_counts, counts.size() * sizeof(uint32_t),
-                             cudaMemcpyDeviceToHost, s));
-    VBQ_CUDA(cudaStreamSynchronize(s));
-    std::vector<uint32_t> ustart(((size_t)units + 1) * 4);
-    uint64_t items[4] = {0, 0, 0, 0};
-    for (int64_t u = 0; u < units; ++u)
-        for (int w = 0; w < 4; ++w) {
-            ustart[u * 4 + w] = (uint32_t)items[w];
-            items[w] += counts[u * 4 + w];
+    std::vector<uint32_t> counts;
+    std::vector<vbq::UnitHeader> headers;
+    int C = 0;
+    int64_t S = 0, units = 0;
+    uint32_t max16 = 0;
+    void* d_counts = nullptr;
+    for (int cand : {16, 8, 4, 2, 1}) {
+        if (cand > G && cand != 1) continue;
+        const int64_t Sc = (G + cand - 1) / cand, uc = nrb * Sc;
+        const bool last = (cand == 1);
+        if (!last && uc < 3LL * sms) continue;        // too few units for the GPU: narrower slabs
+        if (uc > (1LL << 31) - 2) return fail(VBQ_ERR_UNSUPPORTED, "too many units");
+        void* dc = nullptr;
+        VBQ_CUDA(tmp.alloc(&dc, (size_t)uc * 4 * sizeof(uint32_t)));
+        VBQ_CUDA(vbq::launch_count(d_widths, N, (int)G, cand, (int)nrb, (int)uc, static_cast<uint32_t*>(dc), s));
+        std::vector<uint32_t> cnt((size_t)uc * 4);
+        VBQ_CUDA(cudaMemcpyAsync(cnt.data(), dc, cnt.size() * sizeof(uint32_t), cudaMemcpyDeviceToHost, s));
+        VBQ_CUDA(cudaStreamSynchronize(s));
+        std::vector<vbq::UnitHeader> hd((size_t)uc);
+        uint32_t m16 = 0;
+        for (int64_t u = 0; u < uc; ++u) {
+            hd[u] = vbq::make_header(&cnt[u * 4], cand);
+            m16 = std::max<uint32_t>(m16, hd[u].size16);
         }
-    for (int w = 0; w < 4; ++w) {
-        if (items[w] > 0xffffffffull) return fail(VBQ_ERR_UNSUPPORTED, "too many groups of one width");
-        ustart[units * 4 + w] = (uint32_t)items[w];
+        if (m16 * 16u > vbq::MAX_BLOB_BYTES && !last) continue;
+        if (m16 * 16u > vbq::MAX_BLOB_BYTES) return fail(VBQ_ERR_UNSUPPORTED, "unit blob too large");
+        C = cand; S = Sc; units = uc; max16 = m16;
+        counts.swap(cnt);
+        headers.swap(hd);
+        d_counts = dc;
+        break;
     }
-    uint64_t total_items = items[0] + items[1] + items[2] + items[3];
+    if (C == 0) return fail(VBQ_ERR_UNSUPPORTED, "no slab width fits");
+    (void)d_counts;
+    uint64_t real_items[4] = {0, 0, 0, 0};
+    std::vector<uint32_t> blob_off((size_t)units + 1);
+    uint64_t off16 = 0;
+    for (int64_t u = 0; u < units; ++u) {
+        blob_off[u] = (uint32_t)off16;
+        off16 += headers[u].size16;
+        for (int w = 0; w < 4; ++w) real_items[w] += counts[u * 4 + w];
+        if (off16 > 0xffffffffull) return fail(VBQ_ERR_UNSUPPORTED, "layout too large");
+    }
+    blob_off[units] = (uint32_t)off16;
+    const uint64_t total_items = real_items[0] + real_items[1] + real_items[2] + real_items[3];
     if (total_items != ngroups) return fail(VBQ_ERR_CUDA, "item count mismatch (%llu vs %llu)",
                                             (unsigned long long)total_items, (unsigned long long)ngroups);
+    size_t payload_bytes = 0;
+    for (int w = 0; w < 4; ++w) payload_bytes += (size_t)real_items[w] * 8 * (1u << w);
+    const size_t scale_bytes = (size_t)ngroups * 2;
 
-    // 3. one device allocation, sub-buffers 256-byte aligned
-    const size_t A = 256;
-    size_t off = 0;
-    const size_t map_off = off;
-    off = round_up(off + (size_t)units * C * vbq::MAP_WORDS * 4, A);
-    const size_t ustart_off = off;
-    off = round_up(off + ustart.size() * 4, A);
-    size_t pay_off[4], sc_off[4];
-    size_t payload_bytes = 0, scale_bytes = 0;
-    for (int w = 0; w < 4; ++w) {
-        pay_off[w] = off;
-        const size_t pb = (size_t)items[w] * 8 * (1u << w);
-        payload_bytes += pb;
-        off = round_up(off + pb + 64, A);      // 64 bytes of slack after each stream
-    }
-    for (int w = 0; w < 4; ++w) {
-        sc_off[w] = off;
-        scale_bytes += (size_t)items[w] * 2;
-        off = round_up(off + (size_t)items[w] * 2 + 16, A);
-    }
-    const size_t alloc_bytes = off;
+    // 3. one device allocation: blob area (+ slack), then the blob offsets
+    const size_t blob_bytes = (size_t)off16 * 16 + 256;
+    const size_t off_at = round_up(blob_bytes, 256);
+    const size_t alloc_bytes = off_at + blob_off.size() * 4;
+    void* d_headers = nullptr;
+    VBQ_CUDA(tmp.alloc(&d_headers, headers.size() * sizeof(vbq::UnitHeader)));
+    VBQ_CUDA(cudaMemcpyAsync(d_headers, headers.data(), headers.size() * sizeof(vbq::UnitHeader),
+                             cudaMemcpyHostToDevice, s));
 
     vbq_layout* L = new (std::nothrow) vbq_layout();
     if (!L) return fail(VBQ_ERR_NOMEM, "host allocation failed");
@@ -212,16 +214,8 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     L->meta_bytes = alloc_bytes - payload_bytes - scale_bytes;
     L->device = dev;
     vbq::LayoutView& V = L->view;
-    V.map = reinterpret_cast<uint32_t*>(base + map_off);
-    V.ustart = reinterpret_cast<uint32_t*>(base + ustart_off);
-    uint8_t* pay[4];
-    uint16_t* sc[4];
-    for (int w = 0; w < 4; ++w) {
-        pay[w] = base + pay_off[w];
-        sc[w] = reinterpret_cast<uint16_t*>(base + sc_off[w]);
-        V.payload[w] = pay[w];
-        V.scales[w] = sc[w];
-    }
+    V.blobs = base;
+    V.blob_off = reinterpret_cast<uint32_t*>(base + off_at);
     V.N = N;
     V.K = K;
     V.G = (int)G;
@@ -229,13 +223,14 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     V.S = (int)S;
     V.nrb = (int)nrb;
     V.units = (int)units;
+    V.max_blob16 = (int)max16;
 
     if ((e = cudaMemsetAsync(L->base, 0, alloc_bytes, s)) != cudaSuccess) return bail(VBQ_ERR_CUDA, "memset", e);
-    if ((e = cudaMemcpyAsync(const_cast<uint32_t*>(V.ustart), ustart.data(), ustart.size() * 4,
-                             cudaMemcpyHostToDevice, s)) != cudaSuccess)
-        return bail(VBQ_ERR_CUDA, "ustart copy", e);
-    if ((e = vbq::launch_scatter(d_codes, d_widths, d_scales, V, const_cast<uint32_t*>(V.map), pay, sc, s)) !=
+    if ((e = cudaMemcpyAsync(base + off_at, blob_off.data(), blob_off.size() * 4, cudaMemcpyHostToDevice, s)) !=
         cudaSuccess)
+        return bail(VBQ_ERR_CUDA, "offset copy", e);
+    if ((e = vbq::launch_scatter(d_codes, d_widths, d_scales, static_cast<const vbq::UnitHeader*>(d_headers), V,
+                                 base, s)) != cudaSuccess)
         return bail(VBQ_ERR_CUDA, "scatter launch", e);
     if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return bail(VBQ_ERR_CUDA, "pack", e);
     *out = L;

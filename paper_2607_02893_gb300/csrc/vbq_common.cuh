@@ -1,29 +1,31 @@
 // vbq_common.cuh — device layout of a packed VBQ matrix, shared by the CUDA
-// kernels of this library (pack, dequant, GEMV).
+// kernels of this library (pack, dequant, products).
 //
-// Layout (chosen for GB300; the paper fixes only "64*b bits per group on byte
-// boundaries", §1 and §6):
+// Layout (chosen for GB300; the paper fixes only "64*b bits per group, packed
+// on byte boundaries", §1 and §6):
 //
 //   * Rows are cut into row blocks of RB = 128 rows; the K/64 group columns
-//     into slabs of C columns (C in 4..32, chosen per matrix at pack time so
-//     that there are enough blocks for every SM). A (row block, slab) pair is
-//     a "unit", numbered u = rb * S + s with S = slabs per row.
-//   * For each unit a width map holds a 2-bit width code per (column, row):
-//     code w means b = 1 << w. Column c of unit u occupies 8 32-bit words
-//     map[(u*C + c)*8 + j], word j holding rows 16j .. 16j+15 (2 bits each,
-//     row r at bits 2*(r%16)).
-//   * Each width b has its own item stream. An item is one group (64 codes)
-//     of width b; within a unit the items of width b are ordered by
-//     (column, row), and units follow each other in unit order. Item i of
-//     width index w starts at byte 8*b*i of payload[w] and its FP16 scale is
-//     scales[w][i]. ustart[u*4 + w] is the index of the unit's first item of
-//     width index w (ustart has units+1 rows; the last row holds the totals).
-//   * Inside an item, code j of the group (column 64*col + j) occupies bits
-//     [j*b, j*b + b) of the item's little-endian bytes.
-//
-// The map gives, per unit, every item's (column, row) without storing row or
-// column indices per item: kernels rebuild the item list of a unit in shared
-// memory from the map (build_item_list below).
+//     into slabs of C columns (C in 1..16, chosen per matrix at pack time). A
+//     (row block, slab) pair is a "unit", numbered slab-major:
+//     u = s * nrb + rb, so consecutive units share the same activations.
+//   * Every unit is one contiguous, 16-byte aligned blob (so a kernel can copy
+//     it into shared memory in one sweep):
+//         UnitHeader (48 bytes)
+//         payload of width index w = 0..3 (b = 1 << w), each padded to 16 bytes
+//         FP16 scales of each width, each padded to 16 bytes
+//         row bytes of each width (row within the row block), padded to 16
+//         column ends: uint16 cend[w][c] = index (within width w) of the
+//         first item after column c
+//     Blob u starts at byte 16 * blob_off[u] of the layout's blob area.
+//   * Within a unit the groups ("items") of one width are ordered by
+//     (column, row); item i of width index w has its 8*b payload bytes at
+//     payload_w + 8*b*i, its scale at scales_w[i], its row at rows_w[i].
+//   * Item formats (code j = the group's weight at column 64*col + j):
+//       b = 1: 8 bytes, bit j of the little-endian 64-bit word is code j;
+//       b = 2: 16 bytes as two bit planes: bytes 0-7 hold bit 0 of every code
+//              (bit j = code j's low bit), bytes 8-15 bit 1;
+//       b = 4: 32 bytes, code j at bits [4j, 4j+4) (little-endian);
+//       b = 8: 64 bytes, byte j is code j.
 #pragma once
 
 #include <cstdint>
@@ -34,20 +36,33 @@ namespace vbq {
 
 constexpr int RB = 128;          // rows per row block
 constexpr int GROUP = 64;        // weights per group (§3.1)
-constexpr int MAX_C = 32;        // max group columns per slab
-constexpr int MAP_WORDS = RB / 16;   // map words per column
+constexpr int MAX_C = 16;        // max group columns per slab
 constexpr int MAX_BATCH = 16;
+constexpr int MAX_UNIT_ITEMS = RB * MAX_C;
+constexpr uint32_t MAX_BLOB_BYTES = 23 * 1024;   // a unit blob fits one shared-memory stage
+
+struct UnitHeader {
+    uint16_t n[4];        // items per width index
+    uint16_t pay16[4];    // payload offsets within the blob, in 16-byte units
+    uint16_t sc16[4];     // scale offsets
+    uint16_t row16[4];    // row-byte offsets
+    uint16_t cc16;        // column-end offset (uint16 [4][C])
+    uint16_t size16;      // blob size in 16-byte units
+    uint16_t pad[6];
+};
+static_assert(sizeof(UnitHeader) == 48, "header is 48 bytes");
 
 struct LayoutView {
-    const uint32_t* map;
-    const uint32_t* ustart;
-    const uint8_t* payload[4];
-    const uint16_t* scales[4];
+    const uint8_t* blobs;       // blob area
+    const uint32_t* blob_off;   // units + 1 offsets, in 16-byte units
     int64_t N, K;
     int G, C, S, nrb, units;
+    int max_blob16;             // largest blob, in 16-byte units
 };
 
 __host__ __device__ inline int width_of(int w) { return 1 << w; }
+__host__ __device__ inline int unit_rb(const LayoutView& L, int u) { return u % L.nrb; }
+__host__ __device__ inline int unit_slab(const LayoutView& L, int u) { return u / L.nrb; }
 
 // Rows and columns actually present in unit (rb, s).
 __host__ __device__ inline int unit_rows(const LayoutView& L, int rb) {
@@ -59,83 +74,104 @@ __host__ __device__ inline int unit_cols(const LayoutView& L, int s) {
     return c < L.C ? c : L.C;
 }
 
-// Shared-memory item list of one unit. list[i] = (column << 8) | row, with
-// the items of width index w at [wbase[w], wbase[w] + wcount[w]) in
-// (column, row) order. colbase must have room for MAX_C * 4 ints.
-struct ItemList {
-    uint16_t* list;
-    int* colbase;     // [MAX_C][4] scratch
-    int* wcount;      // [4]
-    int* wbase;       // [4]
-};
+// Sizes of the blob parts, given the item counts of a unit.
+__host__ __device__ inline uint32_t pad16(uint32_t bytes) { return (bytes + 15u) / 16u; }
 
-// Rebuild the item list of a unit from its width map (already in shared memory
-// as map_s[c*8 + j]). All threads of the block must call it; blockDim.x must be
-// a multiple of 32.
-__device__ inline void build_item_list(const uint32_t* map_s, int rows, int cols, ItemList il) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
-    // pass 1: per (column, width) counts
-    for (int c = warp; c < cols; c += nwarps) {
-        int cnt0 = 0, cnt1 = 0, cnt2 = 0, cnt3 = 0;
-        for (int chunk = 0; chunk < RB / 32; ++chunk) {
-            int r = chunk * 32 + lane;
-            uint32_t code = (map_s[c * MAP_WORDS + (r >> 4)] >> (2 * (r & 15))) & 3u;
-            bool valid = r < rows;
-            cnt0 += __popc(__ballot_sync(0xffffffffu, valid && code == 0));
-            cnt1 += __popc(__ballot_sync(0xffffffffu, valid && code == 1));
-            cnt2 += __popc(__ballot_sync(0xffffffffu, valid && code == 2));
-            cnt3 += __popc(__ballot_sync(0xffffffffu, valid && code == 3));
+__host__ __device__ inline UnitHeader make_header(const uint32_t n[4], int C) {
+    UnitHeader h{};
+    uint32_t off = sizeof(UnitHeader) / 16;
+    for (int w = 0; w < 4; ++w) { h.n[w] = (uint16_t)n[w]; h.pay16[w] = (uint16_t)off; off += pad16(n[w] * 8u * (1u << w)); }
+    for (int w = 0; w < 4; ++w) { h.sc16[w] = (uint16_t)off; off += pad16(n[w] * 2u); }
+    for (int w = 0; w < 4; ++w) { h.row16[w] = (uint16_t)off; off += pad16(n[w]); }
+    h.cc16 = (uint16_t)off;
+    off += pad16(8u * (uint32_t)C);
+    h.size16 = (uint16_t)off;
+    return h;
+}
+
+// ---------------------------------------------------------------------------
+// Item formats: pack 64 codes (64 bytes, one per code) into an item, and back.
+// ---------------------------------------------------------------------------
+
+template <int B>
+__device__ __forceinline__ void pack_item(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst) {
+    uint32_t cw[16];
+    const uint4* p = reinterpret_cast<const uint4*>(src);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint4 v = p[q];
+        cw[4 * q] = v.x; cw[4 * q + 1] = v.y; cw[4 * q + 2] = v.z; cw[4 * q + 3] = v.w;
+    }
+    auto code = [&](int j) -> uint32_t { return (cw[j >> 2] >> (8 * (j & 3))) & 0xffu; };
+    if (B == 1 || B == 2) {
+        uint64_t plane[2] = {0, 0};
+#pragma unroll
+        for (int j = 0; j < GROUP; ++j) {
+            const uint64_t c = code(j);
+            plane[0] |= (c & 1ull) << j;
+            if (B == 2) plane[1] |= ((c >> 1) & 1ull) << j;
         }
-        if (lane == 0) {
-            il.colbase[c * 4 + 0] = cnt0;
-            il.colbase[c * 4 + 1] = cnt1;
-            il.colbase[c * 4 + 2] = cnt2;
-            il.colbase[c * 4 + 3] = cnt3;
+        if (B == 1) {
+            *reinterpret_cast<uint2*>(dst) = make_uint2((uint32_t)plane[0], (uint32_t)(plane[0] >> 32));
+        } else {
+            *reinterpret_cast<uint4*>(dst) = make_uint4((uint32_t)plane[0], (uint32_t)(plane[0] >> 32),
+                                                        (uint32_t)plane[1], (uint32_t)(plane[1] >> 32));
+        }
+    } else if (B == 4) {
+        uint32_t o[8];
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+            uint32_t w = 0;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) w |= code(8 * t + i) << (4 * i);
+            o[t] = w;
+        }
+        uint4* d = reinterpret_cast<uint4*>(dst);
+        d[0] = make_uint4(o[0], o[1], o[2], o[3]);
+        d[1] = make_uint4(o[4], o[5], o[6], o[7]);
+    } else {
+        uint4* d = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) d[q] = make_uint4(cw[4 * q], cw[4 * q + 1], cw[4 * q + 2], cw[4 * q + 3]);
+    }
+}
+
+// Code j of an item of width B held in 2*B words.
+template <int B>
+__device__ __forceinline__ uint32_t item_code(const uint32_t* w, int j) {
+    if (B == 1) return (w[j >> 5] >> (j & 31)) & 1u;
+    if (B == 2) return ((w[j >> 5] >> (j & 31)) & 1u) | (((w[2 + (j >> 5)] >> (j & 31)) & 1u) << 1);
+    if (B == 4) return (w[j >> 3] >> (4 * (j & 7))) & 0xfu;
+    return (w[j >> 2] >> (8 * (j & 3))) & 0xffu;
+}
+
+// Load an item of width B (8-byte aligned for B = 1, 16-byte otherwise) into 2*B words.
+template <int B>
+__device__ __forceinline__ void load_item(const uint8_t* __restrict__ src, uint32_t* w) {
+    if (B == 1) {
+        uint2 v = *reinterpret_cast<const uint2*>(src);
+        w[0] = v.x; w[1] = v.y;
+    } else {
+#pragma unroll
+        for (int q = 0; q < B / 2; ++q) {
+            uint4 v = reinterpret_cast<const uint4*>(src)[q];
+            w[4 * q] = v.x; w[4 * q + 1] = v.y; w[4 * q + 2] = v.z; w[4 * q + 3] = v.w;
         }
     }
-    __syncthreads();
-    if (threadIdx.x < 4) {
-        int w = threadIdx.x, tot = 0;
-        for (int c = 0; c < cols; ++c) tot += il.colbase[c * 4 + w];
-        il.wcount[w] = tot;
-    }
-    __syncthreads();
-    if (threadIdx.x < 4) {
-        int w = threadIdx.x, base = 0;
-        for (int v = 0; v < w; ++v) base += il.wcount[v];
-        il.wbase[w] = base;
-        for (int c = 0; c < cols; ++c) {
-            int n = il.colbase[c * 4 + w];
-            il.colbase[c * 4 + w] = base;
-            base += n;
-        }
-    }
-    __syncthreads();
-    // pass 2: scatter (column, row) entries
-    const uint32_t lt = (1u << lane) - 1u;
-    for (int c = warp; c < cols; c += nwarps) {
-        int run0 = il.colbase[c * 4 + 0], run1 = il.colbase[c * 4 + 1];
-        int run2 = il.colbase[c * 4 + 2], run3 = il.colbase[c * 4 + 3];
-        for (int chunk = 0; chunk < RB / 32; ++chunk) {
-            int r = chunk * 32 + lane;
-            uint32_t code = (map_s[c * MAP_WORDS + (r >> 4)] >> (2 * (r & 15))) & 3u;
-            bool valid = r < rows;
-            uint32_t m0 = __ballot_sync(0xffffffffu, valid && code == 0);
-            uint32_t m1 = __ballot_sync(0xffffffffu, valid && code == 1);
-            uint32_t m2 = __ballot_sync(0xffffffffu, valid && code == 2);
-            uint32_t m3 = __ballot_sync(0xffffffffu, valid && code == 3);
-            if (valid) {
-                int pos;
-                if (code == 0) pos = run0 + __popc(m0 & lt);
-                else if (code == 1) pos = run1 + __popc(m1 & lt);
-                else if (code == 2) pos = run2 + __popc(m2 & lt);
-                else pos = run3 + __popc(m3 & lt);
-                il.list[pos] = (uint16_t)((c << 8) | r);
-            }
-            run0 += __popc(m0); run1 += __popc(m1); run2 += __popc(m2); run3 += __popc(m3);
-        }
-    }
-    __syncthreads();
+}
+
+// Level L_b(u): 2u - 1 for b = 1, u - 2^(b-1) otherwise.
+template <int B>
+__device__ __forceinline__ int level_of(uint32_t u) {
+    return B == 1 ? (int)(2 * u) - 1 : (int)u - (1 << (B - 1));
+}
+
+// Column of item i of width w, given its column-end table cend (C entries,
+// nondecreasing) and a lower bound c0 on the answer.
+__device__ __forceinline__ int column_of(const uint16_t* cend, int cols, int c0, int i) {
+    int c = c0;
+    while (c < cols - 1 && (int)cend[c] <= i) ++c;
+    return c;
 }
 
 }  // namespace vbq

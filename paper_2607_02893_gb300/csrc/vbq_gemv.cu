@@ -1,43 +1,400 @@
 // vbq_gemv.cu — fused dequantise-and-multiply y = W x over the packed layout
-// (§6: "loads the packed low-bit bytes for a group, expands them ... in
-// registers using the per-group scale, and accumulates the matrix-vector
-// product").
+// (§6: load the packed low-bit bytes of a group, expand them in registers with
+// the group's scale, accumulate the matrix-vector product; the wide weights
+// never reach memory).
 //
-// One block per unit (row block x slab). The block stages the slab's x in
-// shared memory as fp32, rebuilds the unit's item list from the width map,
-// then each thread takes whole items: it loads the item's 8*b bytes, expands
-// each code to its level, accumulates level * x in fp32, applies the group
-// scale once, and adds the group's contribution to the row's shared-memory
-// partial sum. Row partials go to y directly (one slab per row) or are added
-// into a zeroed y (several slabs).
+// Batch 1 (gemv1_kernel): a persistent grid of three blocks per SM. Block p
+// owns a contiguous range of units in slab-major order, so consecutive units
+// share their activations. Unit blobs stream into two shared-memory stages
+// with cp.async (the next unit loads while the current one is computed).
+// Per slab the block stages x as fp32 and builds, for every 4 consecutive
+// weights of a group column, the 16 subset sums of their activations (a
+// lookup table indexed by 4 code bits). Per unit, the four widths are split
+// into warp tasks:
+//   b = 1  one table lookup per 4 weights: S = sum of x over set bits, and
+//          the group's dot product is 2S - X (L_1(u) = 2u - 1, X = sum of x);
+//   b = 2  the two bit planes use the same tables: S0 + 2 S1 - 2X;
+//   b = 4  codes are masked in place and read as exact denormal floats
+//          against activations pre-scaled per code slot (packed f32x2 FMAs);
+//          8X (summed in the same order) is subtracted for the zero level;
+//   b = 8  same with a byte permute and 2^23 + 128.
+// X is summed from the tables in the same order as the lookups, so a group
+// whose codes are all at the zero level contributes exactly 0. Each group's
+// fp32 dot product is scaled once by its FP16 scale and added to its row's
+// shared-memory partial; a unit's rows then go to y directly (one slab per
+// row) or are added into a zeroed y (several slabs).
+//
+// Batch 2..16 (gemm_kernel<NB>): one block per unit, one thread per group,
+// plain fp32 FMAs per code and per activation row.
 #include "vbq_kernels.h"
 
 namespace vbq {
 namespace {
 
-constexpr int GEMV_THREADS = 256;
+constexpr int THREADS = 256;
+constexpr int WARPS = THREADS / 32;
+constexpr int XQ = 20;                   // floats per 16-code quarter of x (16 + 4 pad: quarters use other banks)
+constexpr int XH = 36;                   // floats per 32-code half of the pre-scaled x (32 + 4 pad)
+constexpr int LUT_COL_BYTES = 1088;      // 16 tables x 64 bytes + 64: neighbouring columns use other banks
+constexpr int STAGE_BYTES = MAX_BLOB_BYTES;   // holds the largest unit blob (the packer guarantees it)
+
+struct __align__(16) Tables {
+    uint8_t lut[MAX_C * LUT_COL_BYTES];  // column c, nibble j, entry m at c*1088 + j*64 + m*4
+    float xs[MAX_C * 4 * XQ];            // x as fp32; quarter (c, q) at (c*4 + q) * XQ
+    float x4s[MAX_C * 2 * XH];           // x pre-scaled per 4-bit nibble slot (see dot4_half); half (c, h) at (c*2 + h) * XH
+    float2 x4z[MAX_C][2];                // per column and half: sums of x * 2^-100, even / odd codes
+    float xlut[MAX_C];                   // per column: sum of the all-ones entries, in lookup order
+    float ys[2][RB];                     // row partials of the current and the previous unit
+};
+
+constexpr size_t GEMV1_SMEM = 128 /* alignment slack */ + 2 * STAGE_BYTES + sizeof(Tables);
+// three blocks per SM: 3 x (GEMV1_SMEM + 1 KB reserved per block) must fit in 228 KB
+static_assert(3 * (GEMV1_SMEM + 1024) <= 228 * 1024, "three blocks per SM");
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+template <int OFF>
+__device__ __forceinline__ float lds_f32(uint32_t addr) {
+    float v;
+    asm("ld.shared.f32 %0, [%1+%2];" : "=f"(v) : "r"(addr), "n"(OFF));
+    return v;
+}
+
+__device__ __forceinline__ float4 lds_f32x4(uint32_t addr) {
+    float4 v;
+    asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint32_t lds_u8(uint32_t addr) {
+    uint32_t v;
+    asm("ld.shared.u8 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ uint32_t lds_u16(uint32_t addr) {
+    uint32_t v;
+    asm("ld.shared.u16 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ float lds_f32r(uint32_t addr) {
+    float v;
+    asm("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ float2 lds_f32x2(uint32_t addr) {
+    float2 v;
+    asm("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint4 lds_u32x4(uint32_t addr) {
+    uint4 v;
+    asm("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
+__device__ __forceinline__ float2 f2(float a, float b) { return make_float2(a, b); }
+
+// Byte offset of nibble I (0..7) of w, scaled by 4 (a table entry is 4 bytes).
+template <int I>
+__device__ __forceinline__ uint32_t nib4(uint32_t w) {
+    return (I == 0 ? (w << 2) : (w >> (4 * I - 2))) & 0x3Cu;
+}
+
+// Sum over the 16 nibbles of a 64-bit bit plane (words lo, hi) of the table
+// entries they select; tb = shared address of the column's tables. The 16
+// lookups are added as a balanced tree (pairs, then pairs of pairs), the same
+// tree that builds xlut.
+__device__ __forceinline__ float tree16(const float* v) {
+    const float a0 = v[0] + v[1], a1 = v[2] + v[3], a2 = v[4] + v[5], a3 = v[6] + v[7];
+    const float a4 = v[8] + v[9], a5 = v[10] + v[11], a6 = v[12] + v[13], a7 = v[14] + v[15];
+    return ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
+}
+
+__device__ __forceinline__ float plane_sum(uint32_t tb, uint32_t lo, uint32_t hi) {
+    float v[16];
+    v[0] = lds_f32<0>(nib4<0>(lo) | tb);
+    v[1] = lds_f32<64>(nib4<1>(lo) | tb);
+    v[2] = lds_f32<128>(nib4<2>(lo) | tb);
+    v[3] = lds_f32<192>(nib4<3>(lo) | tb);
+    v[4] = lds_f32<256>(nib4<4>(lo) | tb);
+    v[5] = lds_f32<320>(nib4<5>(lo) | tb);
+    v[6] = lds_f32<384>(nib4<6>(lo) | tb);
+    v[7] = lds_f32<448>(nib4<7>(lo) | tb);
+    v[8] = lds_f32<512>(nib4<0>(hi) | tb);
+    v[9] = lds_f32<576>(nib4<1>(hi) | tb);
+    v[10] = lds_f32<640>(nib4<2>(hi) | tb);
+    v[11] = lds_f32<704>(nib4<3>(hi) | tb);
+    v[12] = lds_f32<768>(nib4<4>(hi) | tb);
+    v[13] = lds_f32<832>(nib4<5>(hi) | tb);
+    v[14] = lds_f32<896>(nib4<6>(hi) | tb);
+    v[15] = lds_f32<960>(nib4<7>(hi) | tb);
+    return tree16(v);
+}
+
+// 4-bit, half a group per lane (32 codes: four words of LSB-first nibbles).
+// Codes are masked in place: (w & 0xF << 4i) read as a float is exactly
+// u * 2^(4i - 149) for nibbles whose top bit is at most bit 23 (a set bit 23 is
+// the implicit leading one of a normal number, which keeps the value linear in
+// u). The top two nibbles are shifted down first. Activations come pre-scaled
+// per nibble slot (x4s[j] = x_j * 2^(49 - e_j), e_j the slot's shift), so each
+// product is exactly u * x * 2^-100. Two f32x2 chains (words 0, 2 and 1, 3)
+// add even codes in .x and odd codes in .y; x4z holds the same sums of x.
+__device__ __forceinline__ float2 dot4_half(uint4 v, uint32_t xa) {
+    float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
+    const uint32_t words[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+        const uint32_t w = words[t], w2 = w >> 24;
+        const float4 xa4 = lds_f32x4(xa + t * 32), xb4 = lds_f32x4(xa + t * 32 + 16);
+        float2& c = (t & 1) ? cb : ca;
+        c = __ffma2_rn(f2(__uint_as_float(w & 0xFu), __uint_as_float(w & 0xF0u)), f2(xa4.x, xa4.y), c);
+        c = __ffma2_rn(f2(__uint_as_float(w & 0xF00u), __uint_as_float(w & 0xF000u)), f2(xa4.z, xa4.w), c);
+        c = __ffma2_rn(f2(__uint_as_float(w & 0xF0000u), __uint_as_float(w & 0xF00000u)), f2(xb4.x, xb4.y), c);
+        c = __ffma2_rn(f2(__uint_as_float(w2 & 0xFu), __uint_as_float(w2 & 0xF0u)), f2(xb4.z, xb4.w), c);
+    }
+    return __fadd2_rn(ca, cb);
+}
+
+// 8-bit, a quarter group per lane (16 codes): codes expand to exact floats
+// 2^23 + u by a byte permute, 2^23 + 128 is subtracted exactly, packed f32x2
+// FMAs accumulate in two chains.
+__device__ __forceinline__ float dot8_quarter(uint4 v, uint32_t xa) {
+    const float2 off = f2(-8388736.f, -8388736.f);          // -(2^23 + 128)
+    const uint32_t M = 0x4B000000u;
+    float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
+    const uint32_t words[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+        const uint32_t w = words[t];
+        const float4 x4 = lds_f32x4(xa + t * 16);
+        const float2 l0 = __fadd2_rn(f2(__uint_as_float(__byte_perm(w, M, 0x7540)),
+                                        __uint_as_float(__byte_perm(w, M, 0x7541))), off);
+        const float2 l1 = __fadd2_rn(f2(__uint_as_float(__byte_perm(w, M, 0x7542)),
+                                        __uint_as_float(__byte_perm(w, M, 0x7543))), off);
+        ca = __ffma2_rn(l0, f2(x4.x, x4.y), ca);
+        cb = __ffma2_rn(l1, f2(x4.z, x4.w), cb);
+    }
+    return (ca.x + ca.y) + (cb.x + cb.y);
+}
+
+// Copy unit u's blob into the stage at shared address dst (each thread its
+// 16-byte chunks).
+__device__ __forceinline__ void issue_unit(const LayoutView& L, int u, uint32_t dst) {
+    const uint32_t o0 = L.blob_off[u], o1 = L.blob_off[u + 1];
+    const uint8_t* src = L.blobs + (int64_t)o0 * 16;
+    for (uint32_t i = threadIdx.x; i < o1 - o0; i += THREADS) cp_async16(dst + i * 16, src + (int64_t)i * 16);
+}
+
+__device__ __forceinline__ float half_bits(uint32_t bits) { return __half2float(__ushort_as_half((uint16_t)bits)); }
+
+// Column of a task's first item i0: the number of columns ending at or before
+// it (lane l < cols holds the end of column l).
+__device__ __forceinline__ int task_first_column(const uint16_t* cend, int cols, int i0, int lane) {
+    const bool ended = lane < cols && (int)cend[lane] <= i0;
+    const int c0 = __popc(__ballot_sync(0xffffffffu, ended));
+    return c0 < cols ? c0 : cols - 1;
+}
+
+__global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
+                                                           float* __restrict__ y) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    // stages and tables on a 128-byte boundary: lookups OR a nibble offset into table addresses
+    unsigned char* base = smem_raw + ((128u - (smem_u32(smem_raw) & 127u)) & 127u);
+    Tables& T = *reinterpret_cast<Tables*>(base + 2 * STAGE_BYTES);
+    const uint32_t stage0 = smem_u32(base);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int P = gridDim.x, p = blockIdx.x;
+    const int u_begin = (int)((int64_t)L.units * p / P), u_end = (int)((int64_t)L.units * (p + 1) / P);
+    if (u_begin >= u_end) return;
+
+    issue_unit(L, u_begin, stage0);
+    cp_async_commit();
+    if (u_begin + 1 < u_end) issue_unit(L, u_begin + 1, stage0 + STAGE_BYTES);
+    cp_async_commit();
+    for (int i = tid; i < 2 * RB; i += THREADS) (&T.ys[0][0])[i] = 0.f;
+
+    const uint32_t lut0 = smem_u32(T.lut), xs0 = smem_u32(T.xs), x4s0 = smem_u32(T.x4s);
+    const uint32_t x4z0 = smem_u32(T.x4z), xlut0 = smem_u32(T.xlut);
+    int cur_slab = -1;
+    for (int k = u_begin; k < u_end; ++k) {
+        const int buf = (k - u_begin) & 1;
+        const unsigned char* blob = base + buf * STAGE_BYTES;
+        const uint32_t sblob = stage0 + buf * STAGE_BYTES;
+        const int s = unit_slab(L, k), rb = unit_rb(L, k);
+        const int cols = unit_cols(L, s);
+        float* ys = T.ys[buf];
+
+        if (s != cur_slab) {            // activations of a new slab: x, tables, X sums
+            const int64_t k0 = (int64_t)s * L.C * GROUP;
+            __syncthreads();            // nobody still reads the old tables
+            for (int i = tid; i < cols * 32; i += THREADS) {
+                const uint32_t two = __ldg(reinterpret_cast<const uint32_t*>(x + k0) + i);
+                const float xa = __uint_as_float(two << 16), xb = __uint_as_float(two & 0xFFFF0000u);
+                const int kk = 2 * i, c = kk >> 6, jj = kk & 63;
+                *reinterpret_cast<float2*>(&T.xs[(c * 4 + (jj >> 4)) * XQ + (jj & 15)]) = f2(xa, xb);
+                // 4-bit slot shifts: nibble slots 0..5 of a word keep their place, 6 and 7 come down by 24
+                const int slot = jj & 7, e = slot < 6 ? 4 * slot : 4 * (slot - 6);
+                *reinterpret_cast<float2*>(&T.x4s[(c * 2 + (jj >> 5)) * XH + (jj & 31)]) =
+                    f2(xa * __uint_as_float((uint32_t)(127 + 49 - e) << 23),
+                       xb * __uint_as_float((uint32_t)(127 + 49 - e - 4) << 23));
+            }
+            __syncthreads();
+            for (int pj = tid; pj < cols * 16; pj += THREADS) {
+                const int c = pj >> 4, j = pj & 15;
+                const float4 xv = *reinterpret_cast<const float4*>(&T.xs[(c * 4 + (j >> 2)) * XQ + 4 * (j & 3)]);
+                const float t3 = xv.x + xv.y, t12 = xv.w + xv.z;
+                float4* dst = reinterpret_cast<float4*>(T.lut + c * LUT_COL_BYTES + j * 64);
+                dst[0] = make_float4(0.f, xv.x, xv.y, t3);
+                dst[1] = make_float4(xv.z, xv.z + xv.x, xv.z + xv.y, xv.z + t3);
+                dst[2] = make_float4(xv.w, xv.w + xv.x, xv.w + xv.y, xv.w + t3);
+                dst[3] = make_float4(t12, t12 + xv.x, t12 + xv.y, t12 + t3);
+            }
+            __syncthreads();
+            if (tid < cols) {
+                const float* t = reinterpret_cast<const float*>(T.lut + tid * LUT_COL_BYTES);
+                float v[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) v[j] = t[j * 16 + 15];
+                T.xlut[tid] = tree16(v);
+                // X for the 4-bit zero level, summed as dot4_half accumulates
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                    float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
+                    for (int t = 0; t < 4; ++t) {
+                        float2& cc = (t & 1) ? cb : ca;
+                        for (int e = 0; e < 8; e += 2) {
+                            const int j = 32 * hh + 8 * t + e;
+                            const float* xq = &T.xs[(tid * 4 + (j >> 4)) * XQ + (j & 15)];
+                            cc = __ffma2_rn(f2(xq[0], xq[1]), f2(0x1p-100f, 0x1p-100f), cc);
+                        }
+                    }
+                    T.x4z[tid][hh] = __fadd2_rn(ca, cb);
+                }
+            }
+            cur_slab = s;
+        }
+
+        cp_async_wait_1();              // this thread's copies of unit k have landed
+        __syncthreads();                // ... and everyone's
+        const UnitHeader h = *reinterpret_cast<const UnitHeader*>(blob);
+        const int n[4] = {h.n[0], h.n[1], h.n[2], h.n[3]};
+
+        // warp tasks: 64 one-bit groups (two per lane), 32 two-bit groups, 16
+        // four-bit groups (two lanes each), 8 eight-bit groups (four lanes each)
+        const int t1 = (n[0] + 63) >> 6, t2 = (n[1] + 31) >> 5, t4 = (n[2] + 15) >> 4, t8 = (n[3] + 7) >> 3;
+        const int ntask = t1 + t2 + t4 + t8;
+        const uint16_t* cend = reinterpret_cast<const uint16_t*>(blob + h.cc16 * 16);
+        for (int t = warp; t < ntask; t += WARPS) {
+            if (t < t4) {                                   // 4-bit: two lanes per group, one half each
+                // lanes l and l+16 share group l%16; the half is swizzled so that a
+                // quarter-warp reads 8 distinct 16-byte bank groups
+                const int e = lane & 15, hh = ((e >> 2) + (lane >> 4)) & 1;
+                const int i0 = t * 16, i = i0 + e;
+                const uint16_t* ce = cend + 2 * L.C;
+                const int c0 = task_first_column(ce, cols, i0, lane);
+                float part = 0.f;
+                if (i < n[2]) {
+                    const uint4 v = lds_u32x4(sblob + h.pay16[2] * 16 + i * 32 + hh * 16);
+                    const int c = column_of(ce, cols, c0, i);
+                    const float2 acc = dot4_half(v, x4s0 + (c * 2 + hh) * XH * 4);
+                    const float2 z = lds_f32x2(x4z0 + (c * 2 + hh) * 8);
+                    part = (acc.x - 8.f * z.x) + (acc.y - 8.f * z.y);
+                }
+                part += __shfl_xor_sync(0xffffffffu, part, 16);
+                if (i < n[2] && lane < 16) {
+                    const int r = lds_u8(sblob + h.row16[2] * 16 + i);
+                    atomicAdd(&ys[r], (half_bits(lds_u16(sblob + h.sc16[2] * 16 + 2 * i)) * 0x1p100f) * part);
+                }
+            } else if (t < t4 + t8) {                       // 8-bit: four lanes per group, one quarter each
+                // lane 8k + e takes quarter ((e >> 1) + k) % 4 of group e: a quarter-warp
+                // reads 8 distinct 16-byte bank groups
+                const int e = lane & 7, q = ((e >> 1) + (lane >> 3)) & 3;
+                const int i0 = (t - t4) * 8, i = i0 + e;
+                const uint16_t* ce = cend + 3 * L.C;
+                const int c0 = task_first_column(ce, cols, i0, lane);
+                float part = 0.f;
+                if (i < n[3]) {
+                    const uint4 v = lds_u32x4(sblob + h.pay16[3] * 16 + i * 64 + q * 16);
+                    const int c = column_of(ce, cols, c0, i);
+                    part = dot8_quarter(v, xs0 + (c * 4 + q) * XQ * 4);
+                }
+                part += __shfl_xor_sync(0xffffffffu, part, 8);
+                part += __shfl_xor_sync(0xffffffffu, part, 16);
+                if (i < n[3] && lane < 8) {
+                    const int r = lds_u8(sblob + h.row16[3] * 16 + i);
+                    atomicAdd(&ys[r], half_bits(lds_u16(sblob + h.sc16[3] * 16 + 2 * i)) * part);
+                }
+            } else if (t < t4 + t8 + t2) {                  // 2-bit: one group per lane
+                const int i0 = (t - t4 - t8) * 32, i = i0 + lane;
+                const uint16_t* ce = cend + L.C;
+                const int c0 = task_first_column(ce, cols, i0, lane);
+                if (i < n[1]) {
+                    const uint4 pl = lds_u32x4(sblob + h.pay16[1] * 16 + i * 16);
+                    const int c = column_of(ce, cols, c0, i);
+                    const uint32_t tb = lut0 + c * LUT_COL_BYTES;
+                    const float s0 = plane_sum(tb, pl.x, pl.y);
+                    const float s1 = plane_sum(tb, pl.z, pl.w);
+                    const int r = lds_u8(sblob + h.row16[1] * 16 + i);
+                    atomicAdd(&ys[r], half_bits(lds_u16(sblob + h.sc16[1] * 16 + 2 * i)) *
+                                          (s0 + 2.f * (s1 - lds_f32r(xlut0 + 4 * c))));
+                }
+            } else {                                        // 1-bit: two groups per lane
+                const int i0 = (t - t4 - t8 - t2) * 64, i = i0 + 2 * lane;
+                const int c0 = task_first_column(cend, cols, i0, lane);
+                if (i < n[0]) {
+                    const uint4 v = lds_u32x4(sblob + h.pay16[0] * 16 + i * 8);
+                    const uint32_t rows2 = lds_u16(sblob + h.row16[0] * 16 + i);
+                    const uint32_t sc2 = *reinterpret_cast<const uint32_t*>(blob + h.sc16[0] * 16 + 2 * i);
+                    const int ca = column_of(cend, cols, c0, i);
+                    const float suma = plane_sum(lut0 + ca * LUT_COL_BYTES, v.x, v.y);
+                    if (i + 1 < n[0]) {
+                        const int cb = column_of(cend, cols, ca, i + 1);
+                        const float sumb = plane_sum(lut0 + cb * LUT_COL_BYTES, v.z, v.w);
+                        atomicAdd(&ys[rows2 >> 8], half_bits(sc2 >> 16) * (2.f * sumb - lds_f32r(xlut0 + 4 * cb)));
+                    }
+                    atomicAdd(&ys[rows2 & 0xff], half_bits(sc2) * (2.f * suma - lds_f32r(xlut0 + 4 * ca)));
+                }
+            }
+        }
+        __syncthreads();                // unit k done: its stage and ys[buf] are complete
+        if (k + 2 < u_end) issue_unit(L, k + 2, stage0 + buf * STAGE_BYTES);
+        cp_async_commit();
+        const int rows = unit_rows(L, rb);
+        float* dst = y + (int64_t)rb * RB;
+        for (int r = tid; r < RB; r += THREADS) {
+            const float v = ys[r];
+            ys[r] = 0.f;                // ready for unit k + 2 (the barrier at its start orders this)
+            if (r < rows) {
+                if (L.S == 1) dst[r] = v;
+                else atomicAdd(dst + r, v);
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Batch 2..16: one block per unit, one thread per group.
+// ---------------------------------------------------------------------------
 
 template <int B, int NB>
 __device__ __forceinline__ void dot_item(const uint8_t* __restrict__ src, const float* __restrict__ xs,
                                          int xstride, int nb, float* acc) {
-    uint64_t wv[B];
-    if (B == 1) {
-        wv[0] = __ldg(reinterpret_cast<const unsigned long long*>(src));
-    } else {
-        const uint4* p = reinterpret_cast<const uint4*>(src);
-#pragma unroll
-        for (int i = 0; i < B / 2; ++i) {
-            uint4 v = __ldg(p + i);
-            wv[2 * i] = (uint64_t)v.x | ((uint64_t)v.y << 32);
-            wv[2 * i + 1] = (uint64_t)v.z | ((uint64_t)v.w << 32);
-        }
-    }
-    constexpr uint32_t MASK = (1u << B) - 1u;
+    uint32_t w[2 * B];
+    load_item<B>(src, w);
 #pragma unroll
     for (int j = 0; j < GROUP; ++j) {
-        const int bit = j * B;
-        const uint32_t u = (uint32_t)(wv[bit >> 6] >> (bit & 63)) & MASK;
-        const float lv = (B == 1) ? (float)(int)(2 * u - 1) : (float)((int)u - (1 << (B - 1)));
+        const float lv = (float)level_of<B>(item_code<B>(w, j));
 #pragma unroll
         for (int q = 0; q < NB; ++q)
             if (q < nb) acc[q] = fmaf(lv, xs[q * xstride + j], acc[q]);
@@ -45,23 +402,20 @@ __device__ __forceinline__ void dot_item(const uint8_t* __restrict__ src, const 
 }
 
 template <int NB>
-__global__ void __launch_bounds__(GEMV_THREADS) gemv_kernel(LayoutView L, const uint16_t* __restrict__ X,
-                                                            float* __restrict__ Y, int nb) {
+__global__ void __launch_bounds__(THREADS) gemm_kernel(LayoutView L, const uint16_t* __restrict__ X,
+                                                       float* __restrict__ Y, int nb) {
     extern __shared__ float4 smem_f4[];
     float* xs = reinterpret_cast<float*>(smem_f4);                 // [NB][C*64]
-    __shared__ uint32_t map_s[MAX_C * MAP_WORDS];
-    __shared__ uint16_t list_s[RB * MAX_C];
-    __shared__ int colbase_s[MAX_C * 4];
-    __shared__ int wcount_s[4], wbase_s[4];
+    __shared__ UnitHeader h;
     __shared__ float ys[NB][RB];
 
-    const int u = blockIdx.x, rb = u / L.S, s = u % L.S;
+    const int u = blockIdx.x, rb = unit_rb(L, u), s = unit_slab(L, u);
     const int rows = unit_rows(L, rb), cols = unit_cols(L, s);
     const int xstride = L.C * GROUP;
     const int64_t k0 = (int64_t)s * L.C * GROUP;
+    const uint8_t* blob = L.blobs + (int64_t)L.blob_off[u] * 16;
 
-    for (int i = threadIdx.x; i < cols * MAP_WORDS; i += blockDim.x)
-        map_s[i] = L.map[(int64_t)u * L.C * MAP_WORDS + i];
+    if (threadIdx.x == 0) h = *reinterpret_cast<const UnitHeader*>(blob);
     for (int i = threadIdx.x; i < nb * cols * GROUP; i += blockDim.x) {
         const int q = i / (cols * GROUP), k = i - q * cols * GROUP;
         const uint32_t bits = X[(int64_t)q * L.K + k0 + k];
@@ -69,25 +423,24 @@ __global__ void __launch_bounds__(GEMV_THREADS) gemv_kernel(LayoutView L, const 
     }
     for (int i = threadIdx.x; i < NB * RB; i += blockDim.x) (&ys[0][0])[i] = 0.f;
     __syncthreads();
-    ItemList il{list_s, colbase_s, wcount_s, wbase_s};
-    build_item_list(map_s, rows, cols, il);
-
-    const int total = wbase_s[3] + wcount_s[3];
+    const uint16_t* cend = reinterpret_cast<const uint16_t*>(blob + h.cc16 * 16);
+    const int total = h.n[0] + h.n[1] + h.n[2] + h.n[3];
     for (int i = threadIdx.x; i < total; i += blockDim.x) {
-        const int w = (i >= wbase_s[3]) ? 3 : (i >= wbase_s[2]) ? 2 : (i >= wbase_s[1]) ? 1 : 0;
-        const uint32_t e = list_s[i];
-        const int c = e >> 8, r = e & 0xff;
-        const int64_t item = (int64_t)L.ustart[u * 4 + w] + (i - wbase_s[w]);
-        const float sf = __half2float(__ushort_as_half(L.scales[w][item]));
+        int w = 0, j = i;
+        while (w < 3 && j >= h.n[w]) { j -= h.n[w]; ++w; }
+        const int c = column_of(cend + w * L.C, cols, 0, j);
+        const int r = blob[h.row16[w] * 16 + j];
+        const float sf = __half2float(__ushort_as_half(reinterpret_cast<const uint16_t*>(blob + h.sc16[w] * 16)[j]));
+        const uint8_t* pay = blob + h.pay16[w] * 16;
         float acc[NB];
 #pragma unroll
         for (int q = 0; q < NB; ++q) acc[q] = 0.f;
         const float* xc = xs + c * GROUP;
         switch (w) {
-            case 0: dot_item<1, NB>(L.payload[0] + item * 8, xc, xstride, nb, acc); break;
-            case 1: dot_item<2, NB>(L.payload[1] + item * 16, xc, xstride, nb, acc); break;
-            case 2: dot_item<4, NB>(L.payload[2] + item * 32, xc, xstride, nb, acc); break;
-            default: dot_item<8, NB>(L.payload[3] + item * 64, xc, xstride, nb, acc); break;
+            case 0: dot_item<1, NB>(pay + j * 8, xc, xstride, nb, acc); break;
+            case 1: dot_item<2, NB>(pay + j * 16, xc, xstride, nb, acc); break;
+            case 2: dot_item<4, NB>(pay + j * 32, xc, xstride, nb, acc); break;
+            default: dot_item<8, NB>(pay + j * 64, xc, xstride, nb, acc); break;
         }
 #pragma unroll
         for (int q = 0; q < NB; ++q)
@@ -106,21 +459,39 @@ __global__ void __launch_bounds__(GEMV_THREADS) gemv_kernel(LayoutView L, const 
 template <int NB>
 cudaError_t launch_nb(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
     const size_t dyn = (size_t)NB * L.C * GROUP * sizeof(float);
-    static bool attr_set = false;           // per process; the attribute is per function
+    static bool attr_set = false;           // the attribute is per function; set once per process
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemv_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute(gemm_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)(NB * MAX_C * GROUP * sizeof(float)));
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    gemv_kernel<NB><<<L.units, GEMV_THREADS, dyn, s>>>(L, X, Y, B);
+    gemm_kernel<NB><<<L.units, THREADS, dyn, s>>>(L, X, Y, B);
+    return cudaGetLastError();
+}
+
+int g_sms = 0;
+
+cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(gemv1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)GEMV1_SMEM);
+        if (e != cudaSuccess) return e;
+        int dev = 0;
+        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+        if ((e = cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int grid = L.units < 3 * g_sms ? L.units : 3 * g_sms;
+    gemv1_kernel<<<grid, THREADS, GEMV1_SMEM, s>>>(L, x, y);
     return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
-    if (B <= 1) return launch_nb<1>(L, X, Y, B, s);
+    if (B <= 1) return launch_gemv1(L, X, Y, s);
     if (B <= 2) return launch_nb<2>(L, X, Y, B, s);
     if (B <= 4) return launch_nb<4>(L, X, Y, B, s);
     if (B <= 8) return launch_nb<8>(L, X, Y, B, s);

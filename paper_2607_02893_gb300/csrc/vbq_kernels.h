@@ -11,16 +11,15 @@ namespace vbq {
 // Pack-time kernels (vbq_pack.cu).
 cudaError_t launch_validate(const uint8_t* codes, const uint8_t* widths, int64_t N, int64_t K,
                             uint32_t* err_flags, cudaStream_t s);
-cudaError_t launch_count(const uint8_t* widths, int64_t N, int G, int C, int S, int nrb,
+cudaError_t launch_count(const uint8_t* widths, int64_t N, int G, int C, int nrb, int units,
                          uint32_t* counts, cudaStream_t s);
 cudaError_t launch_scatter(const uint8_t* codes, const uint8_t* widths, const uint16_t* scales,
-                           const LayoutView& L, uint32_t* map, uint8_t* const payload[4],
-                           uint16_t* const scales_out[4], cudaStream_t s);
+                           const UnitHeader* headers, const LayoutView& L, uint8_t* blobs, cudaStream_t s);
 cudaError_t launch_dequant(const LayoutView& L, uint8_t* codes_out, uint8_t* widths_out,
                            uint16_t* scales_out, float* w_out, cudaStream_t s);
 
-// Products (vbq_gemv.cu). Y is B x N; `accumulate` means Y was zeroed and
-// units add into it (more than one slab per row).
+// Products (vbq_gemv.cu). Y is B x N. When the layout has more than one slab
+// per row, units add into Y, which the caller must have zeroed.
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s);
 
 }  // namespace vbq
