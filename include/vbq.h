@@ -112,9 +112,14 @@ vbq_status_t vbq_dequant(const vbq_layout* layout, uint8_t* codes_out,
  *   x  device, K BF16 bit patterns.
  *   y  device, N floats; overwritten.
  * Per output, |y - y_exact| stays within 2e-3 * sum_k |w_nk x_k| + 1e-5.
- * The summation order is not fixed: results can differ in the last bits
- * between calls. Calls on different streams may run concurrently on the same
- * layout.
+ * Groups of one row block are summed in a varying order, so repeated calls can
+ * differ in the last bits. When a row spans several slabs of the layout, the
+ * call uses a split-K workspace
+ * owned by the layout: calls that share a layout must not overlap on the GPU
+ * (issue them on one stream, or order them with events). The kernel is
+ * launched with programmatic dependent launch: it may start loading weights
+ * before the previous kernel on the stream has finished, and reads x only
+ * after it has.
  */
 vbq_status_t vbq_gemv(const vbq_layout* layout, const uint16_t* x, float* y,
                       void* stream);
@@ -124,7 +129,8 @@ vbq_status_t vbq_gemv(const vbq_layout* layout, const uint16_t* x, float* y,
  *   X  device, B x K BF16 bit patterns, row-major.
  *   Y  device, B x N floats, row-major; overwritten.
  *   B  1..16 (VBQ_ERR_UNSUPPORTED otherwise).
- * Same accuracy statement as vbq_gemv.
+ * Same accuracy statement as vbq_gemv; the summation order is not fixed (results
+ * can differ in the last bits between calls). Y is zeroed on the stream first.
  */
 vbq_status_t vbq_gemm_small(const vbq_layout* layout, const uint16_t* X, float* Y,
                             int B, void* stream);

@@ -140,7 +140,6 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     int C = 0;
     int64_t S = 0, units = 0;
     uint32_t max16 = 0;
-    void* d_counts = nullptr;
     for (int cand : {16, 8, 4, 2, 1}) {
         if (cand > G && cand != 1) continue;
         const int64_t Sc = (G + cand - 1) / cand, uc = nrb * Sc;
@@ -164,11 +163,9 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
         C = cand; S = Sc; units = uc; max16 = m16;
         counts.swap(cnt);
         headers.swap(hd);
-        d_counts = dc;
         break;
     }
     if (C == 0) return fail(VBQ_ERR_UNSUPPORTED, "no slab width fits");
-    (void)d_counts;
     uint64_t real_items[4] = {0, 0, 0, 0};
     std::vector<uint32_t> blob_off((size_t)units + 1);
     uint64_t off16 = 0;
@@ -189,7 +186,8 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     // 3. one device allocation: blob area (+ slack), then the blob offsets
     const size_t blob_bytes = (size_t)off16 * 16 + 256;
     const size_t off_at = round_up(blob_bytes, 256);
-    const size_t alloc_bytes = off_at + blob_off.size() * 4;
+    const size_t ctl_at = round_up(off_at + blob_off.size() * 4, 256);
+    const size_t alloc_bytes = ctl_at + (2 + (size_t)nrb) * sizeof(uint32_t);
     void* d_headers = nullptr;
     VBQ_CUDA(tmp.alloc(&d_headers, headers.size() * sizeof(vbq::UnitHeader)));
     VBQ_CUDA(cudaMemcpyAsync(d_headers, headers.data(), headers.size() * sizeof(vbq::UnitHeader),
@@ -216,6 +214,7 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     vbq::LayoutView& V = L->view;
     V.blobs = base;
     V.blob_off = reinterpret_cast<uint32_t*>(base + off_at);
+    V.ctl = reinterpret_cast<uint32_t*>(base + ctl_at);
     V.N = N;
     V.K = K;
     V.G = (int)G;
@@ -275,7 +274,7 @@ static vbq_status_t run_product(const vbq_layout* L, const uint16_t* X, float* Y
     if (B < 1 || B > vbq::MAX_BATCH) return fail(VBQ_ERR_UNSUPPORTED, "batch %d outside 1..16", B);
     if (!aligned16(X) || !aligned16(Y)) return fail(VBQ_ERR_ALIGN, "x and y must be 16-byte aligned");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (L->view.S > 1)
+    if (B > 1 && L->view.S > 1)       // the batched kernel adds slab partials into a zeroed Y
         VBQ_CUDA(cudaMemsetAsync(Y, 0, (size_t)B * (size_t)L->view.N * sizeof(float), s));
     VBQ_CUDA(vbq::launch_gemv(L->view, X, Y, B, s));
     return VBQ_OK;

@@ -17,6 +17,13 @@
 //         column ends: uint16 cend[w][c] = index (within width w) of the
 //         first item after column c
 //     Blob u starts at byte 16 * blob_off[u] of the layout's blob area.
+//   * When a row has several slabs, the batch-1 product adds every slab's row
+//     partials into y with atomics, and y needs no zeroing by the caller: the
+//     block that owns slab 0 of a row block zeroes those rows first and then
+//     sets that row block's flag to the current call's epoch; blocks adding
+//     other slabs wait for the flag. The epoch lives on the device (the last
+//     block of a call advances it), so graph replays stay correct. Calls that
+//     share a layout must not overlap on the GPU.
 //   * Within a unit the groups ("items") of one width are ordered by
 //     (column, row); item i of width index w has its 8*b payload bytes at
 //     payload_w + 8*b*i, its scale at scales_w[i], its row at rows_w[i].
@@ -39,7 +46,7 @@ constexpr int GROUP = 64;        // weights per group (§3.1)
 constexpr int MAX_C = 16;        // max group columns per slab
 constexpr int MAX_BATCH = 16;
 constexpr int MAX_UNIT_ITEMS = RB * MAX_C;
-constexpr uint32_t MAX_BLOB_BYTES = 23 * 1024;   // a unit blob fits one shared-memory stage
+constexpr uint32_t MAX_BLOB_BYTES = 22 * 1024;   // a unit blob fits one shared-memory stage
 
 struct UnitHeader {
     uint16_t n[4];        // items per width index
@@ -55,6 +62,7 @@ static_assert(sizeof(UnitHeader) == 48, "header is 48 bytes");
 struct LayoutView {
     const uint8_t* blobs;       // blob area
     const uint32_t* blob_off;   // units + 1 offsets, in 16-byte units
+    uint32_t* ctl;              // [0] call epoch, [1] blocks finished in this call, [2 + rb] y-zeroed flags
     int64_t N, K;
     int G, C, S, nrb, units;
     int max_blob16;             // largest blob, in 16-byte units

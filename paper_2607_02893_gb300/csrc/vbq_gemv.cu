@@ -22,10 +22,12 @@
 // whose codes are all at the zero level contributes exactly 0. Each group's
 // fp32 dot product is scaled once by its FP16 scale and added to its row's
 // shared-memory partial; a unit's rows then go to y directly (one slab per
-// row) or are added into a zeroed y (several slabs).
+// row) or through the layout's split-K workspace (several slabs).
 //
 // Batch 2..16 (gemm_kernel<NB>): one block per unit, one thread per group,
 // plain fp32 FMAs per code and per activation row.
+#include <cstddef>
+
 #include "vbq_kernels.h"
 
 namespace vbq {
@@ -45,7 +47,14 @@ struct __align__(16) Tables {
     float2 x4z[MAX_C][2];                // per column and half: sums of x * 2^-100, even / odd codes
     float xlut[MAX_C];                   // per column: sum of the all-ones entries, in lookup order
     float ys[2][RB];                     // row partials of the current and the previous unit
+    unsigned long long bar[2];           // one mbarrier per stage
+    alignas(16) uint8_t colarr[MAX_UNIT_ITEMS + 64];   // column of every item of the current unit (16-byte stores)
+    uint32_t epoch;                      // this call's epoch (split-K y zeroing)
+    int flag_ok;
 };
+static_assert(offsetof(Tables, colarr) % 16 == 0, "colarr takes 16-byte stores");
+static_assert(offsetof(Tables, bar) % 8 == 0, "mbarriers are 8-byte aligned");
+static_assert(offsetof(Tables, lut) == 0, "tables start at the aligned base");
 
 constexpr size_t GEMV1_SMEM = 128 /* alignment slack */ + 2 * STAGE_BYTES + sizeof(Tables);
 // three blocks per SM: 3 x (GEMV1_SMEM + 1 KB reserved per block) must fit in 228 KB
@@ -97,11 +106,11 @@ __device__ __forceinline__ uint4 lds_u32x4(uint32_t addr) {
     return v;
 }
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(dst), "l"(src) : "memory");
+__device__ __forceinline__ uint32_t lds_u32(uint32_t addr) {
+    uint32_t v;
+    asm("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
 }
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
 
 __device__ __forceinline__ float2 f2(float a, float b) { return make_float2(a, b); }
 
@@ -188,22 +197,72 @@ __device__ __forceinline__ float dot8_quarter(uint4 v, uint32_t xa) {
     return (ca.x + ca.y) + (cb.x + cb.y);
 }
 
-// Copy unit u's blob into the stage at shared address dst (each thread its
-// 16-byte chunks).
-__device__ __forceinline__ void issue_unit(const LayoutView& L, int u, uint32_t dst) {
-    const uint32_t o0 = L.blob_off[u], o1 = L.blob_off[u + 1];
-    const uint8_t* src = L.blobs + (int64_t)o0 * 16;
-    for (uint32_t i = threadIdx.x; i < o1 - o0; i += THREADS) cp_async16(dst + i * 16, src + (int64_t)i * 16);
+__device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) {
+    return *reinterpret_cast<const volatile uint32_t*>(p);
+}
+__device__ __forceinline__ void st_volatile(uint32_t* p, uint32_t v) {
+    *reinterpret_cast<volatile uint32_t*>(p) = v;
 }
 
 __device__ __forceinline__ float half_bits(uint32_t bits) { return __half2float(__ushort_as_half((uint16_t)bits)); }
 
-// Column of a task's first item i0: the number of columns ending at or before
-// it (lane l < cols holds the end of column l).
-__device__ __forceinline__ int task_first_column(const uint16_t* cend, int cols, int i0, int lane) {
-    const bool ended = lane < cols && (int)cend[lane] <= i0;
-    const int c0 = __popc(__ballot_sync(0xffffffffu, ended));
-    return c0 < cols ? c0 : cols - 1;
+// ---------------------------------------------------------------------------
+// Unit blobs arrive by TMA bulk copy, completion tracked by one mbarrier per
+// stage. Every wait is bounded: after about a second the block records
+// VBQ_DEVICE_TIMEOUT in g_device_status and stops.
+// ---------------------------------------------------------------------------
+
+__device__ uint32_t g_device_status;
+constexpr uint32_t VBQ_DEVICE_TIMEOUT = 1u;
+constexpr unsigned long long WAIT_LIMIT_NS = 1000000000ull;
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_barrier_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+    return ok != 0;
+}
+// Wait until the barrier's phase with this parity completes; false on timeout.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (global_ns() - t0 > WAIT_LIMIT_NS) return false;
+    }
+    return true;
+}
+// One thread: expect `bytes` on the barrier and start the bulk copy.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(bar), "r"(bytes) : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void issue_unit(const LayoutView& L, int u, uint32_t dst, uint32_t bar) {
+    const uint32_t o0 = L.blob_off[u], o1 = L.blob_off[u + 1];
+    bulk_load(dst, L.blobs + (int64_t)o0 * 16, (o1 - o0) * 16, bar);
+}
+
+// Fill colarr[cb + a .. cb + e) with column c: bytes up to a 16-byte boundary,
+// 16-byte stores in between, bytes after.
+__device__ __forceinline__ void fill_run(uint32_t cb, int a, int e, int c) {
+    const uint32_t b4 = 0x01010101u * (uint32_t)c;
+    const int a16 = min((a + 15) & ~15, e), e16 = max(e & ~15, a16);
+    for (int i = a; i < a16; ++i) asm volatile("st.shared.u8 [%0], %1;" :: "r"(cb + i), "r"(c) : "memory");
+    for (int i = a16; i < e16; i += 16)
+        asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" :: "r"(cb + i), "r"(b4) : "memory");
+    for (int i = e16; i < e; ++i) asm volatile("st.shared.u8 [%0], %1;" :: "r"(cb + i), "r"(c) : "memory");
 }
 
 __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
@@ -218,21 +277,50 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
     const int u_begin = (int)((int64_t)L.units * p / P), u_end = (int)((int64_t)L.units * (p + 1) / P);
     if (u_begin >= u_end) return;
 
-    issue_unit(L, u_begin, stage0);
-    cp_async_commit();
-    if (u_begin + 1 < u_end) issue_unit(L, u_begin + 1, stage0 + STAGE_BYTES);
-    cp_async_commit();
+    const uint32_t bar0 = smem_u32(&T.bar[0]);
+    if (tid == 0) {
+        mbar_init(bar0, 1);
+        mbar_init(bar0 + 8, 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (tid == 0) {
+        issue_unit(L, u_begin, stage0, bar0);
+        if (u_begin + 1 < u_end) issue_unit(L, u_begin + 1, stage0 + STAGE_BYTES, bar0 + 8);
+    }
+    // Weights never depend on earlier work in the stream, so their first copies
+    // are in flight before this grid waits for its predecessor (programmatic
+    // dependent launch); x, y and the workspace are touched only after the wait.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (L.S > 1) {
+        // split-K: this call's epoch; zero y for the row blocks whose slab 0 this
+        // block owns (units u < nrb) and publish them
+        if (tid == 0) T.epoch = ld_volatile(L.ctl) + 1u;
+        const int z_end = min(u_end, L.nrb);
+        for (int u = u_begin; u < z_end; ++u) {
+            float* dst = y + (int64_t)u * RB;
+            const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
+            for (int r = tid; r < rows; r += THREADS) dst[r] = 0.f;
+        }
+        __syncthreads();
+        if (tid == 0 && u_begin < z_end) {
+            __threadfence();
+            for (int u = u_begin; u < z_end; ++u) st_volatile(L.ctl + 2 + u, T.epoch);
+        }
+    }
     for (int i = tid; i < 2 * RB; i += THREADS) (&T.ys[0][0])[i] = 0.f;
 
     const uint32_t lut0 = smem_u32(T.lut), xs0 = smem_u32(T.xs), x4s0 = smem_u32(T.x4s);
-    const uint32_t x4z0 = smem_u32(T.x4z), xlut0 = smem_u32(T.xlut);
+    const uint32_t x4z0 = smem_u32(T.x4z), xlut0 = smem_u32(T.xlut), cola = smem_u32(T.colarr);
+    int s = u_begin / L.nrb, rb = u_begin - s * L.nrb;
     int cur_slab = -1;
+    bool ok = true;
     for (int k = u_begin; k < u_end; ++k) {
-        const int buf = (k - u_begin) & 1;
+        const int j = k - u_begin, buf = j & 1;
         const unsigned char* blob = base + buf * STAGE_BYTES;
         const uint32_t sblob = stage0 + buf * STAGE_BYTES;
-        const int s = unit_slab(L, k), rb = unit_rb(L, k);
-        const int cols = unit_cols(L, s);
+        const int cols = min(L.C, L.G - s * L.C);
         float* ys = T.ys[buf];
 
         if (s != cur_slab) {            // activations of a new slab: x, tables, X sums
@@ -251,10 +339,10 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
             }
             __syncthreads();
             for (int pj = tid; pj < cols * 16; pj += THREADS) {
-                const int c = pj >> 4, j = pj & 15;
-                const float4 xv = *reinterpret_cast<const float4*>(&T.xs[(c * 4 + (j >> 2)) * XQ + 4 * (j & 3)]);
+                const int c = pj >> 4, jn = pj & 15;
+                const float4 xv = *reinterpret_cast<const float4*>(&T.xs[(c * 4 + (jn >> 2)) * XQ + 4 * (jn & 3)]);
                 const float t3 = xv.x + xv.y, t12 = xv.w + xv.z;
-                float4* dst = reinterpret_cast<float4*>(T.lut + c * LUT_COL_BYTES + j * 64);
+                float4* dst = reinterpret_cast<float4*>(T.lut + c * LUT_COL_BYTES + jn * 64);
                 dst[0] = make_float4(0.f, xv.x, xv.y, t3);
                 dst[1] = make_float4(xv.z, xv.z + xv.x, xv.z + xv.y, xv.z + t3);
                 dst[2] = make_float4(xv.w, xv.w + xv.x, xv.w + xv.y, xv.w + t3);
@@ -265,17 +353,17 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
                 const float* t = reinterpret_cast<const float*>(T.lut + tid * LUT_COL_BYTES);
                 float v[16];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) v[j] = t[j * 16 + 15];
+                for (int jn = 0; jn < 16; ++jn) v[jn] = t[jn * 16 + 15];
                 T.xlut[tid] = tree16(v);
                 // X for the 4-bit zero level, summed as dot4_half accumulates
 #pragma unroll
                 for (int hh = 0; hh < 2; ++hh) {
                     float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
-                    for (int t = 0; t < 4; ++t) {
-                        float2& cc = (t & 1) ? cb : ca;
+                    for (int t4 = 0; t4 < 4; ++t4) {
+                        float2& cc = (t4 & 1) ? cb : ca;
                         for (int e = 0; e < 8; e += 2) {
-                            const int j = 32 * hh + 8 * t + e;
-                            const float* xq = &T.xs[(tid * 4 + (j >> 4)) * XQ + (j & 15)];
+                            const int jj = 32 * hh + 8 * t4 + e;
+                            const float* xq = &T.xs[(tid * 4 + (jj >> 4)) * XQ + (jj & 15)];
                             cc = __ffma2_rn(f2(xq[0], xq[1]), f2(0x1p-100f, 0x1p-100f), cc);
                         }
                     }
@@ -285,34 +373,39 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
             cur_slab = s;
         }
 
-        cp_async_wait_1();              // this thread's copies of unit k have landed
-        __syncthreads();                // ... and everyone's
+        ok = mbar_wait(bar0 + 8 * buf, (j >> 1) & 1);   // unit k's blob has landed (each thread waits)
         const UnitHeader h = *reinterpret_cast<const UnitHeader*>(blob);
-        const int n[4] = {h.n[0], h.n[1], h.n[2], h.n[3]};
+        const int n0 = h.n[0], n1 = h.n[1], n2 = h.n[2], n3 = h.n[3];
+        const uint32_t cb1 = (n0 + 15) & ~15, cb2 = cb1 + ((n1 + 15) & ~15), cb3 = cb2 + ((n2 + 15) & ~15);
+        if (ok && tid < 4 * cols) {     // one thread per (width, column) run
+            const uint16_t* cend = reinterpret_cast<const uint16_t*>(blob + h.cc16 * 16);
+            const int w = tid / cols, c = tid - w * cols;
+            const int a = c == 0 ? 0 : cend[w * L.C + c - 1], e = cend[w * L.C + c];
+            const uint32_t cb = cola + (w == 0 ? 0u : w == 1 ? cb1 : w == 2 ? cb2 : cb3);
+            fill_run(cb, a, e, c);
+        }
+        if (!__syncthreads_and(ok)) break;
 
-        // warp tasks: 64 one-bit groups (two per lane), 32 two-bit groups, 16
-        // four-bit groups (two lanes each), 8 eight-bit groups (four lanes each)
-        const int t1 = (n[0] + 63) >> 6, t2 = (n[1] + 31) >> 5, t4 = (n[2] + 15) >> 4, t8 = (n[3] + 7) >> 3;
-        const int ntask = t1 + t2 + t4 + t8;
-        const uint16_t* cend = reinterpret_cast<const uint16_t*>(blob + h.cc16 * 16);
+        // warp tasks: 16 four-bit groups (two lanes each), 8 eight-bit groups
+        // (four lanes each), 32 two-bit groups, 64 one-bit groups (two per lane)
+        const int t4 = (n2 + 15) >> 4, t8 = (n3 + 7) >> 3, t2 = (n1 + 31) >> 5, t1 = (n0 + 63) >> 6;
+        const int ntask = t4 + t8 + t2 + t1;
         for (int t = warp; t < ntask; t += WARPS) {
             if (t < t4) {                                   // 4-bit: two lanes per group, one half each
                 // lanes l and l+16 share group l%16; the half is swizzled so that a
                 // quarter-warp reads 8 distinct 16-byte bank groups
                 const int e = lane & 15, hh = ((e >> 2) + (lane >> 4)) & 1;
-                const int i0 = t * 16, i = i0 + e;
-                const uint16_t* ce = cend + 2 * L.C;
-                const int c0 = task_first_column(ce, cols, i0, lane);
+                const int i = t * 16 + e;
                 float part = 0.f;
-                if (i < n[2]) {
+                if (i < n2) {
                     const uint4 v = lds_u32x4(sblob + h.pay16[2] * 16 + i * 32 + hh * 16);
-                    const int c = column_of(ce, cols, c0, i);
+                    const int c = lds_u8(cola + cb2 + i);
                     const float2 acc = dot4_half(v, x4s0 + (c * 2 + hh) * XH * 4);
                     const float2 z = lds_f32x2(x4z0 + (c * 2 + hh) * 8);
                     part = (acc.x - 8.f * z.x) + (acc.y - 8.f * z.y);
                 }
                 part += __shfl_xor_sync(0xffffffffu, part, 16);
-                if (i < n[2] && lane < 16) {
+                if (i < n2 && lane < 16) {
                     const int r = lds_u8(sblob + h.row16[2] * 16 + i);
                     atomicAdd(&ys[r], (half_bits(lds_u16(sblob + h.sc16[2] * 16 + 2 * i)) * 0x1p100f) * part);
                 }
@@ -320,28 +413,24 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
                 // lane 8k + e takes quarter ((e >> 1) + k) % 4 of group e: a quarter-warp
                 // reads 8 distinct 16-byte bank groups
                 const int e = lane & 7, q = ((e >> 1) + (lane >> 3)) & 3;
-                const int i0 = (t - t4) * 8, i = i0 + e;
-                const uint16_t* ce = cend + 3 * L.C;
-                const int c0 = task_first_column(ce, cols, i0, lane);
+                const int i = (t - t4) * 8 + e;
                 float part = 0.f;
-                if (i < n[3]) {
+                if (i < n3) {
                     const uint4 v = lds_u32x4(sblob + h.pay16[3] * 16 + i * 64 + q * 16);
-                    const int c = column_of(ce, cols, c0, i);
+                    const int c = lds_u8(cola + cb3 + i);
                     part = dot8_quarter(v, xs0 + (c * 4 + q) * XQ * 4);
                 }
                 part += __shfl_xor_sync(0xffffffffu, part, 8);
                 part += __shfl_xor_sync(0xffffffffu, part, 16);
-                if (i < n[3] && lane < 8) {
+                if (i < n3 && lane < 8) {
                     const int r = lds_u8(sblob + h.row16[3] * 16 + i);
                     atomicAdd(&ys[r], half_bits(lds_u16(sblob + h.sc16[3] * 16 + 2 * i)) * part);
                 }
             } else if (t < t4 + t8 + t2) {                  // 2-bit: one group per lane
-                const int i0 = (t - t4 - t8) * 32, i = i0 + lane;
-                const uint16_t* ce = cend + L.C;
-                const int c0 = task_first_column(ce, cols, i0, lane);
-                if (i < n[1]) {
+                const int i = (t - t4 - t8) * 32 + lane;
+                if (i < n1) {
                     const uint4 pl = lds_u32x4(sblob + h.pay16[1] * 16 + i * 16);
-                    const int c = column_of(ce, cols, c0, i);
+                    const int c = lds_u8(cola + cb1 + i);
                     const uint32_t tb = lut0 + c * LUT_COL_BYTES;
                     const float s0 = plane_sum(tb, pl.x, pl.y);
                     const float s1 = plane_sum(tb, pl.z, pl.w);
@@ -350,16 +439,16 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
                                           (s0 + 2.f * (s1 - lds_f32r(xlut0 + 4 * c))));
                 }
             } else {                                        // 1-bit: two groups per lane
-                const int i0 = (t - t4 - t8 - t2) * 64, i = i0 + 2 * lane;
-                const int c0 = task_first_column(cend, cols, i0, lane);
-                if (i < n[0]) {
+                const int i = (t - t4 - t8 - t2) * 64 + 2 * lane;
+                if (i < n0) {
                     const uint4 v = lds_u32x4(sblob + h.pay16[0] * 16 + i * 8);
                     const uint32_t rows2 = lds_u16(sblob + h.row16[0] * 16 + i);
-                    const uint32_t sc2 = *reinterpret_cast<const uint32_t*>(blob + h.sc16[0] * 16 + 2 * i);
-                    const int ca = column_of(cend, cols, c0, i);
+                    const uint32_t sc2 = lds_u32(sblob + h.sc16[0] * 16 + 2 * i);
+                    const uint32_t cols2 = lds_u16(cola + i);
+                    const int ca = cols2 & 0xff;
                     const float suma = plane_sum(lut0 + ca * LUT_COL_BYTES, v.x, v.y);
-                    if (i + 1 < n[0]) {
-                        const int cb = column_of(cend, cols, ca, i + 1);
+                    if (i + 1 < n0) {
+                        const int cb = cols2 >> 8;
                         const float sumb = plane_sum(lut0 + cb * LUT_COL_BYTES, v.z, v.w);
                         atomicAdd(&ys[rows2 >> 8], half_bits(sc2 >> 16) * (2.f * sumb - lds_f32r(xlut0 + 4 * cb)));
                     }
@@ -367,11 +456,31 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
                 }
             }
         }
-        __syncthreads();                // unit k done: its stage and ys[buf] are complete
-        if (k + 2 < u_end) issue_unit(L, k + 2, stage0 + buf * STAGE_BYTES);
-        cp_async_commit();
-        const int rows = unit_rows(L, rb);
+        __syncthreads();                // unit k done: its stage, colarr and ys[buf] are free
+        if (tid == 0 && k + 2 < u_end) issue_unit(L, k + 2, sblob, bar0 + 8 * buf);
+        const int rows = min(RB, (int)(L.N - (int64_t)rb * RB));
         float* dst = y + (int64_t)rb * RB;
+        if (L.S > 1 && j == 0) {
+            // Before its first additions into y, the block checks that every row
+            // block it will add a slab s > 0 into has been zeroed in this call
+            // (slab-0 owners zero theirs when they start, so this rarely waits).
+            if (tid == 0) {
+                bool seen = true;
+                const unsigned long long t0 = global_ns();
+                int s2 = s, rb2 = rb;
+                for (int u = k; u < u_end && seen; ++u) {
+                    if (s2 > 0) {
+                        while (!(seen = ld_volatile(L.ctl + 2 + rb2) == T.epoch))
+                            if (global_ns() - t0 > WAIT_LIMIT_NS) break;
+                    }
+                    if (++rb2 == L.nrb) { rb2 = 0; ++s2; }
+                }
+                asm volatile("fence.acq_rel.gpu;" ::: "memory");
+                T.flag_ok = seen;
+            }
+            __syncthreads();
+            if (!T.flag_ok) { ok = false; break; }
+        }
         for (int r = tid; r < RB; r += THREADS) {
             const float v = ys[r];
             ys[r] = 0.f;                // ready for unit k + 2 (the barrier at its start orders this)
@@ -379,6 +488,24 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
                 if (L.S == 1) dst[r] = v;
                 else atomicAdd(dst + r, v);
             }
+        }
+        if (++rb == L.nrb) { rb = 0; ++s; }
+    }
+    if (!ok) {
+        // a copy or a flag never arrived: record it, give the outstanding copies a
+        // bounded time to land, and stop
+        if (tid == 0) {
+            atomicOr(&g_device_status, VBQ_DEVICE_TIMEOUT);
+            mbar_wait(bar0, 0);
+            mbar_wait(bar0 + 8, 0);
+        }
+    }
+    if (L.S > 1 && tid == 0) {
+        // the last block of the call advances the epoch for the next call
+        __threadfence();
+        if (atomicAdd(L.ctl + 1, 1u) == gridDim.x - 1) {
+            st_volatile(L.ctl + 1, 0u);
+            st_volatile(L.ctl, T.epoch);
         }
     }
 }
@@ -484,7 +611,18 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
         attr_set = true;
     }
     const int grid = L.units < 3 * g_sms ? L.units : 3 * g_sms;
-    gemv1_kernel<<<grid, THREADS, GEMV1_SMEM, s>>>(L, x, y);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = GEMV1_SMEM;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, gemv1_kernel, L, x, y);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -194,6 +194,48 @@ def test_pack_rejects_bad_widths_and_codes():
     assert e.value.name == "VBQ_ERR_ALIGN"
 
 
+@pytest.mark.parametrize("shape", [(4096, 4096), (300, 64 * 70), (1000, 768)], ids=lambda s: f"{s[0]}x{s[1]}")
+def test_gemv_repeated_calls(shape):
+    """Repeated batch-1 calls on one layout all stay within the bound (the
+    split-K workspace and its counters are reset by every call) and agree
+    with each other up to summation-order rounding."""
+    n, k = shape
+    m = Matrix(n, k, seed_path=(90, n, k))
+    layout = _pack(m)
+    ys = [_gemv(layout, m) for _ in range(4)]
+    for y in ys:
+        _assert_bound(y, m)
+    for y in ys[1:]:
+        assert np.allclose(y, ys[0], rtol=1e-5, atol=1e-5)
+
+
+def test_gemv_graph_replays():
+    """A captured CUDA graph of several GEMVs replayed repeatedly: each replay
+    overwrites y (filled with NaN in between) with a result within the bound."""
+    mats = [Matrix(n, k, seed_path=(89, n, k)) for n, k in [(4096, 4096), (1024, 64 * 200), (513, 768)]]
+    lays = [_pack(m) for m in mats]
+    xs = [bits_to_i16(m.x_bits[:1]).to(DEV) for m in mats]
+    ys = [torch.empty(m.n, dtype=torch.float32, device=DEV) for m in mats]
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        for lay, x, y in zip(lays, xs, ys):
+            vbq.vbq_gemv(lay, x[0], y, stream=st)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=st):
+        for lay, x, y in zip(lays, xs, ys):
+            vbq.vbq_gemv(lay, x[0], y, stream=st)
+    for _ in range(3):
+        for y in ys:
+            y.fill_(float("nan"))
+        torch.cuda.synchronize()
+        with torch.cuda.stream(st):
+            g.replay()
+        torch.cuda.synchronize()
+        for m, y in zip(mats, ys):
+            _assert_bound(y.cpu().numpy()[None, :], m)
+
+
 def test_empty_output_dequant_is_noop():
     m = Matrix(64, 128, seed_path=(91, 0, 0))
     layout = _pack(m)
