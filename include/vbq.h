@@ -135,6 +135,34 @@ vbq_status_t vbq_gemv(const vbq_layout* layout, const uint16_t* x, float* y,
 vbq_status_t vbq_gemm_small(const vbq_layout* layout, const uint16_t* X, float* Y,
                             int B, void* stream);
 
+/*
+ * vbq_gemv_static — vbq_gemv for callers that must not allocate device memory.
+ * (The paper has no counterpart; this is an operational variant.)
+ *
+ * Some callers cannot call cudaMalloc where they run products: a serving loop
+ * with a fixed memory budget, code inside a stream capture that forbids
+ * allocation calls, or a host framework whose allocator must own every
+ * device byte. This entry point allocates nothing, on the device or the host.
+ * It runs the same batch-1 kernel as vbq_gemv, but keeps the kernel's split-K
+ * control words (a call epoch, a finished-block count and one flag per row
+ * block) in a fixed array inside this library instead of in the layout.
+ *
+ *   layout  a layout with at most 8192 row blocks of 128 rows (N <= 1048576);
+ *           larger layouts give VBQ_ERR_UNSUPPORTED.
+ *   x, y    as in vbq_gemv (device, 16-byte aligned; y is overwritten).
+ *
+ * The array (32 KB) is a static device variable: every GPU that loads the
+ * library holds it until the process exits. The first call on a device looks
+ * up the array's address with that device current, so make the first call
+ * on each device before any stream capture. Every call on a device shares the
+ * array and leaves its contents for the next call: the finished-block count
+ * is cleared on `stream` before each launch, and the epoch only grows, so
+ * flags left behind never match a later call. Calls that overlap on the GPU
+ * race on the array: order them on one stream.
+ */
+vbq_status_t vbq_gemv_static(const vbq_layout* layout, const uint16_t* x, float* y,
+                             void* stream);
+
 /* vbq_free — release a layout and its device memory (NULL is accepted). */
 vbq_status_t vbq_free(vbq_layout* layout);
 

@@ -288,6 +288,20 @@ vbq_status_t vbq_gemm_small(const vbq_layout* L, const uint16_t* X, float* Y, in
     return run_product(L, X, Y, B, stream);
 }
 
+vbq_status_t vbq_gemv_static(const vbq_layout* L, const uint16_t* x, float* y, void* stream) {
+    g_err[0] = 0;
+    vbq_status_t st = check_layout(L);
+    if (st) return st;
+    if (!x || !y) return fail(VBQ_ERR_ARG, "x and y must be non-NULL");
+    if (!aligned16(x) || !aligned16(y)) return fail(VBQ_ERR_ALIGN, "x and y must be 16-byte aligned");
+    if (L->view.nrb > vbq::STATIC_CTL_WORDS - 2)
+        return fail(VBQ_ERR_UNSUPPORTED, "vbq_gemv_static supports at most %d row blocks of 128 rows (N <= %d); "
+                    "this layout has %d", vbq::STATIC_CTL_WORDS - 2, (vbq::STATIC_CTL_WORDS - 2) * vbq::RB,
+                    L->view.nrb);
+    VBQ_CUDA(vbq::launch_gemv1_static(L->view, x, y, static_cast<cudaStream_t>(stream)));
+    return VBQ_OK;
+}
+
 vbq_status_t vbq_free(vbq_layout* L) {
     if (!L) return VBQ_OK;
     cudaError_t e = L->base ? cudaFree(L->base) : cudaSuccess;

@@ -27,6 +27,7 @@
 // Batch 2..16 (gemm_kernel<NB>): one block per unit, one thread per group,
 // plain fp32 FMAs per code and per activation row.
 #include <cstddef>
+#include <mutex>
 
 #include "vbq_kernels.h"
 
@@ -627,6 +628,42 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
 }
 
 }  // namespace
+
+// ---------------------------------------------------------------------------
+// Batch 1 with the split-K control words in a fixed device array instead of
+// the layout's own allocation (for callers that cannot allocate device
+// memory; see vbq_gemv_static in vbq.h). Every call on a device shares the
+// array: word 0 is the call epoch, word 1 the count of finished blocks
+// (cleared on the stream before every launch), words 2.. the per-row-block
+// zeroed flags. Epochs only grow, so flags left by earlier calls never match
+// the current one. Calls that overlap on the GPU race on the array.
+// ---------------------------------------------------------------------------
+
+static __device__ __align__(256) uint32_t g_static_ctl[STATIC_CTL_WORDS];
+
+cudaError_t launch_gemv1_static(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s) {
+    constexpr int MAX_DEVICES = 64;
+    static std::mutex mu;
+    static uint32_t* addr[MAX_DEVICES] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= MAX_DEVICES) return cudaErrorInvalidDevice;
+    uint32_t* ctl;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (!addr[dev]) {       // once per device, with that device current
+            void* p = nullptr;
+            if ((e = cudaGetSymbolAddress(&p, g_static_ctl)) != cudaSuccess) return e;
+            addr[dev] = static_cast<uint32_t*>(p);
+        }
+        ctl = addr[dev];
+    }
+    if ((e = cudaMemsetAsync(ctl + 1, 0, sizeof(uint32_t), s)) != cudaSuccess) return e;
+    LayoutView Ls = L;
+    Ls.ctl = ctl;
+    return launch_gemv1(Ls, x, y, s);
+}
 
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
     if (B <= 1) return launch_gemv1(L, X, Y, s);

@@ -22,4 +22,10 @@ cudaError_t launch_dequant(const LayoutView& L, uint8_t* codes_out, uint8_t* wid
 // per row, units add into Y, which the caller must have zeroed.
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s);
 
+// Batch 1 with the split-K control words in a fixed device array (no
+// allocation anywhere); usable for layouts with at most STATIC_CTL_WORDS - 2
+// row blocks.
+constexpr int STATIC_CTL_WORDS = 2 + 8192;
+cudaError_t launch_gemv1_static(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s);
+
 }  // namespace vbq

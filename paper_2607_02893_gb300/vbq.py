@@ -34,6 +34,7 @@ SIGNATURES = {
     "vbq_dequant": (_I, [_P, _P, _P, _P, _P, _P]),
     "vbq_gemv": (_I, [_P, _P, _P, _P]),
     "vbq_gemm_small": (_I, [_P, _P, _P, _I, _P]),
+    "vbq_gemv_static": (_I, [_P, _P, _P, _P]),
     "vbq_free": (_I, [_P]),
     "vbq_status_string": (ctypes.c_char_p, [_I]),
     "vbq_last_error": (ctypes.c_char_p, []),
@@ -153,6 +154,12 @@ def vbq_dequant(layout: Layout, codes_out=None, bitwidths_out=None, scales_out=N
 
 def vbq_gemv(layout: Layout, x, y, stream=None) -> None:
     _check(load().vbq_gemv(layout, _ptr(x), _ptr(y), _stream(stream, x, y)))
+
+
+def vbq_gemv_static(layout: Layout, x, y, stream=None) -> None:
+    """vbq_gemv that allocates nothing: its split-K control words live in a
+    fixed array inside the library (see include/vbq.h)."""
+    _check(load().vbq_gemv_static(layout, _ptr(x), _ptr(y), _stream(stream, x, y)))
 
 
 def vbq_gemm_small(layout: Layout, X, Y, B: Optional[int] = None, stream=None) -> None:
