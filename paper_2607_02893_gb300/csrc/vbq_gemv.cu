@@ -39,6 +39,7 @@ constexpr int WARPS = THREADS / 32;
 constexpr int XQ = 20;                   // floats per 16-code quarter of x (16 + 4 pad: quarters use other banks)
 constexpr int XH = 36;                   // floats per 32-code half of the pre-scaled x (32 + 4 pad)
 constexpr int LUT_COL_BYTES = 1088;      // 16 tables x 64 bytes + 64: neighbouring columns use other banks
+constexpr int COLARR_BYTES = MAX_UNIT_ITEMS + 64;
 constexpr int STAGE_BYTES = MAX_BLOB_BYTES;   // holds the largest unit blob (the packer guarantees it)
 
 struct __align__(16) Tables {
@@ -49,13 +50,14 @@ struct __align__(16) Tables {
     float xlut[MAX_C];                   // per column: sum of the all-ones entries, in lookup order
     float ys[2][RB];                     // row partials of the current and the previous unit
     unsigned long long bar[2];           // one mbarrier per stage
-    alignas(16) uint8_t colarr[MAX_UNIT_ITEMS + 64];   // column of every item of the current unit (16-byte stores)
+    alignas(16) uint8_t colarr[2][COLARR_BYTES];       // column of every item of the last two units (16-byte stores)
     uint32_t epoch;                      // this call's epoch (split-K y zeroing)
     int flag_ok;
 };
 static_assert(offsetof(Tables, colarr) % 16 == 0, "colarr takes 16-byte stores");
 static_assert(offsetof(Tables, bar) % 8 == 0, "mbarriers are 8-byte aligned");
 static_assert(offsetof(Tables, lut) == 0, "tables start at the aligned base");
+static_assert(RB <= THREADS, "one thread per row writes a unit's rows");
 
 constexpr size_t GEMV1_SMEM = 128 /* alignment slack */ + 2 * STAGE_BYTES + sizeof(Tables);
 // three blocks per SM: 3 x (GEMV1_SMEM + 1 KB reserved per block) must fit in 228 KB
@@ -266,6 +268,39 @@ __device__ __forceinline__ void fill_run(uint32_t cb, int a, int e, int c) {
     for (int i = e16; i < e; ++i) asm volatile("st.shared.u8 [%0], %1;" :: "r"(cb + i), "r"(c) : "memory");
 }
 
+// Split-K: true once every row block this block adds a slab s > 0 into has
+// been zeroed in this call (flag == epoch), within the wait limit. Thread 0
+// only; ends with an acquire fence.
+__device__ __forceinline__ bool split_k_flags_ready(const LayoutView& L, uint32_t epoch, int u_begin, int u_end,
+                                                    int s0, int rb0) {
+    bool seen = true;
+    const unsigned long long t0 = global_ns();
+    int s2 = s0, rb2 = rb0;
+    for (int u = u_begin; u < u_end && seen; ++u) {
+        if (s2 > 0) {
+            while (!(seen = ld_volatile(L.ctl + 2 + rb2) == epoch))
+                if (global_ns() - t0 > WAIT_LIMIT_NS) break;
+        }
+        if (++rb2 == L.nrb) { rb2 = 0; ++s2; }
+    }
+    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+    return seen;
+}
+
+// A finished unit's row partials ys (row block rbw) go to y: stored when the
+// row has one slab, added otherwise; ys is zeroed for reuse.
+__device__ __forceinline__ void write_rows(const LayoutView& L, float* y, float* ys, int rbw, int tid) {
+    if (tid >= RB) return;
+    const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
+    const float v = ys[tid];
+    ys[tid] = 0.f;
+    if (tid < rows) {
+        float* dst = y + (int64_t)rbw * RB + tid;
+        if (L.S == 1) *dst = v;
+        else atomicAdd(dst, v);
+    }
+}
+
 __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
                                                            float* __restrict__ y) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -313,16 +348,19 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
     for (int i = tid; i < 2 * RB; i += THREADS) (&T.ys[0][0])[i] = 0.f;
 
     const uint32_t lut0 = smem_u32(T.lut), xs0 = smem_u32(T.xs), x4s0 = smem_u32(T.x4s);
-    const uint32_t x4z0 = smem_u32(T.x4z), xlut0 = smem_u32(T.xlut), cola = smem_u32(T.colarr);
-    int s = u_begin / L.nrb, rb = u_begin - s * L.nrb;
+    const uint32_t x4z0 = smem_u32(T.x4z), xlut0 = smem_u32(T.xlut), cola0 = smem_u32(&T.colarr[0][0]);
+    const int s0 = u_begin / L.nrb, rb0 = u_begin - s0 * L.nrb;
+    int s = s0, rb = rb0, prev_rb = rb0;
     int cur_slab = -1;
     bool ok = true;
+    bool checked = L.S == 1;            // split-K zeroing flags verified (or not needed)
     for (int k = u_begin; k < u_end; ++k) {
         const int j = k - u_begin, buf = j & 1;
         const unsigned char* blob = base + buf * STAGE_BYTES;
         const uint32_t sblob = stage0 + buf * STAGE_BYTES;
         const int cols = min(L.C, L.G - s * L.C);
         float* ys = T.ys[buf];
+        const uint32_t cola = cola0 + buf * COLARR_BYTES;
 
         if (s != cur_slab) {            // activations of a new slab: x, tables, X sums
             const int64_t k0 = (int64_t)s * L.C * GROUP;
@@ -385,7 +423,18 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
             const uint32_t cb = cola + (w == 0 ? 0u : w == 1 ? cb1 : w == 2 ? cb2 : cb3);
             fill_run(cb, a, e, c);
         }
+        if (!checked && j == 1 && tid == 0) T.flag_ok = split_k_flags_ready(L, T.epoch, u_begin, u_end, s0, rb0);
+        // one barrier per unit: unit k's column array is complete and every warp
+        // has finished unit k-1, whose stage, rows and partials are now free
         if (!__syncthreads_and(ok)) break;
+        if (j >= 1) {
+            if (!checked) {
+                checked = true;
+                if (!T.flag_ok) { ok = false; break; }
+            }
+            if (tid == 0 && k + 1 < u_end) issue_unit(L, k + 1, stage0 + (buf ^ 1) * STAGE_BYTES, bar0 + 8 * (buf ^ 1));
+            write_rows(L, y, T.ys[buf ^ 1], prev_rb, tid);
+        }
 
         // warp tasks: 16 four-bit groups (two lanes each), 8 eight-bit groups
         // (four lanes each), 32 two-bit groups, 64 one-bit groups (two per lane)
@@ -457,40 +506,14 @@ __global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const u
                 }
             }
         }
-        __syncthreads();                // unit k done: its stage, colarr and ys[buf] are free
-        if (tid == 0 && k + 2 < u_end) issue_unit(L, k + 2, sblob, bar0 + 8 * buf);
-        const int rows = min(RB, (int)(L.N - (int64_t)rb * RB));
-        float* dst = y + (int64_t)rb * RB;
-        if (L.S > 1 && j == 0) {
-            // Before its first additions into y, the block checks that every row
-            // block it will add a slab s > 0 into has been zeroed in this call
-            // (slab-0 owners zero theirs when they start, so this rarely waits).
-            if (tid == 0) {
-                bool seen = true;
-                const unsigned long long t0 = global_ns();
-                int s2 = s, rb2 = rb;
-                for (int u = k; u < u_end && seen; ++u) {
-                    if (s2 > 0) {
-                        while (!(seen = ld_volatile(L.ctl + 2 + rb2) == T.epoch))
-                            if (global_ns() - t0 > WAIT_LIMIT_NS) break;
-                    }
-                    if (++rb2 == L.nrb) { rb2 = 0; ++s2; }
-                }
-                asm volatile("fence.acq_rel.gpu;" ::: "memory");
-                T.flag_ok = seen;
-            }
-            __syncthreads();
-            if (!T.flag_ok) { ok = false; break; }
-        }
-        for (int r = tid; r < RB; r += THREADS) {
-            const float v = ys[r];
-            ys[r] = 0.f;                // ready for unit k + 2 (the barrier at its start orders this)
-            if (r < rows) {
-                if (L.S == 1) dst[r] = v;
-                else atomicAdd(dst + r, v);
-            }
-        }
+        prev_rb = rb;
         if (++rb == L.nrb) { rb = 0; ++s; }
+    }
+    if (ok) {                           // the last unit's rows
+        if (!checked && tid == 0) T.flag_ok = split_k_flags_ready(L, T.epoch, u_begin, u_end, s0, rb0);
+        __syncthreads();
+        if (!checked && !T.flag_ok) ok = false;
+        else write_rows(L, y, T.ys[(u_end - 1 - u_begin) & 1], prev_rb, tid);
     }
     if (!ok) {
         // a copy or a flag never arrived: record it, give the outstanding copies a

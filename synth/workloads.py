@@ -85,6 +85,7 @@ def workload(name: str, batch: int = 1) -> Workload:
     stack1b     d_model 2048, 22 layers, Q/O 2048, K/V 256, MLP 5632, head 32000 (155 GEMVs).
     stack9b     d_model 4096, 32 layers, Q/O 4096, K/V 1024, MLP 14336, head 128256 (225 GEMVs).
     sweep:<n>:<dist>  one n x n GEMV, dist in all1/all2/all4/all8/mixed.
+    matrix:<n>:<k>:<dist>  one n x k GEMV (for profiling single shapes).
     """
     if name == "single768":
         return Workload(name, 0, batch, [MatrixSpec("w", 768, 768, DIST_MAIN, (0, 0, 0))])
@@ -94,6 +95,14 @@ def workload(name: str, batch: int = 1) -> Workload:
         return Workload(name, 2, batch, _stack(2, 2048, 22, 2048, 256, 5632, 32000))
     if name == "stack9b":
         return Workload(name, 3, batch, _stack(3, 4096, 32, 4096, 1024, 14336, 128256))
+    if name.startswith("matrix:"):
+        # matrix:N:K:dist, dist in main / mlp0 / head / all1 / all2 / all4 / all8
+        _, n, k, dist = name.split(":")
+        dists = {"main": DIST_MAIN, "mlp0": DIST_MLP0, "head": DIST_HEAD, **{
+            d: SWEEP_DISTS[d] for d in ("all1", "all2", "all4", "all8")}}
+        n, k = int(n), int(k)
+        return Workload(name, 5, batch, [MatrixSpec(f"m{n}x{k}.{dist}", n, k, dists[dist],
+                                                    (5, n, k, list(dists).index(dist)))])
     if name.startswith("sweep:"):
         _, n, dist = name.split(":")
         n = int(n)
