@@ -3,16 +3,28 @@
 // the group's scale, accumulate the matrix-vector product; the wide weights
 // never reach memory).
 //
-// Batch 1 (gemv1_kernel): a persistent grid of three blocks per SM. Block p
-// owns a contiguous range of units in slab-major order, so consecutive units
-// share their activations. Unit blobs stream into two shared-memory stages
-// with cp.async (the next unit loads while the current one is computed).
-// Per slab the block stages x as fp32 and builds, for every 4 consecutive
-// weights of a group column, the 16 subset sums of their activations (a
-// lookup table indexed by 4 code bits). Per unit, the four widths are split
-// into warp tasks:
+// Batch 1 (gemv1_kernel): one persistent block per SM, warp-specialised.
+//   warp 0 (copier)    streams unit blobs into NSTAGE shared-memory stages with
+//                      TMA bulk copies and, once a unit is consumed, writes its
+//                      row partials to y and starts the copy of a later unit
+//                      into the freed stage;
+//   warps 1.. (NCW)    consumers, in 1, 2 or 4 teams (more units per block,
+//                      more teams): unit j goes to team j % teams, whose warps
+//                      split its items into warp
+//                      tasks and accumulate the group dot products into the
+//                      stage's row partials; an item's column comes from the
+//                      blob's column ends (a ballot per task, see col_uniform).
+// The roles hand stages to one another through two mbarriers per stage
+// (full: blob landed; empty: the unit's team is done), so no block-wide
+// barrier sits in the steady state and up to NSTAGE units are in flight per SM. Block p owns a contiguous range of units in
+// slab-major order, so consecutive units share their activations; on a slab
+// change the consumer warps rebuild, under a named barrier of their own, the
+// per-slab activation tables: x as fp32 and, for every 4 consecutive weights of
+// a group column, the 16 subset sums of their activations (a lookup table
+// indexed by 4 code bits). Per width:
 //   b = 1  one table lookup per 4 weights: S = sum of x over set bits, and
 //          the group's dot product is 2S - X (L_1(u) = 2u - 1, X = sum of x);
+//          two groups per lane, their sums added as f32x2 pairs;
 //   b = 2  the two bit planes use the same tables: S0 + 2 S1 - 2X;
 //   b = 4  codes are masked in place and read as exact denormal floats
 //          against activations pre-scaled per code slot (packed f32x2 FMAs);
@@ -22,7 +34,7 @@
 // whose codes are all at the zero level contributes exactly 0. Each group's
 // fp32 dot product is scaled once by its FP16 scale and added to its row's
 // shared-memory partial; a unit's rows then go to y directly (one slab per
-// row) or through the layout's split-K workspace (several slabs).
+// row) or through atomics (several slabs).
 //
 // Batch 2..16 (gemm_kernel<NB>): one block per unit, one thread per group,
 // plain fp32 FMAs per code and per activation row.
@@ -34,34 +46,38 @@
 namespace vbq {
 namespace {
 
-constexpr int THREADS = 256;
-constexpr int WARPS = THREADS / 32;
+constexpr int THREADS = 256;             // batch 2..16 kernel
+constexpr int NCW = 16;                  // consumer warps of the batch-1 kernel
+constexpr int NCT = 32 * NCW;            // consumer threads
+constexpr int MAX_TEAMS = 4;             // consumer teams (1, 2 or 4 by units per block); unit j goes to team j % teams
+static_assert(NCW == 16 && MAX_TEAMS == 4, "teams of 16, 8 or 4 warps (powers of two)");
+constexpr int G1_THREADS = 32 * (NCW + 1);
+constexpr int NSTAGE = 8;                // blob stages in flight per SM
+static_assert((NSTAGE & (NSTAGE - 1)) == 0, "power-of-two stage count");
 constexpr int XQ = 20;                   // floats per 16-code quarter of x (16 + 4 pad: quarters use other banks)
 constexpr int XH = 36;                   // floats per 32-code half of the pre-scaled x (32 + 4 pad)
-constexpr int LUT_COL_BYTES = 1088;      // 16 tables x 64 bytes + 64: neighbouring columns use other banks
-constexpr int COLARR_BYTES = MAX_UNIT_ITEMS + 64;
+constexpr int LUT_COL_BYTES = 1024;      // 16 tables x 64 bytes per column, columns on 256-byte boundaries
 constexpr int STAGE_BYTES = MAX_BLOB_BYTES;   // holds the largest unit blob (the packer guarantees it)
+static_assert(STAGE_BYTES % 256 == 0, "stages keep the tables 256-byte aligned");
 
 struct __align__(16) Tables {
-    uint8_t lut[MAX_C * LUT_COL_BYTES];  // column c, nibble j, entry m at c*1088 + j*64 + m*4
+    uint8_t lut[MAX_C * LUT_COL_BYTES];  // column c, nibble j, entry m at c*1024 + j*64 + m*4
     float xs[MAX_C * 4 * XQ];            // x as fp32; quarter (c, q) at (c*4 + q) * XQ
     float x4s[MAX_C * 2 * XH];           // x pre-scaled per 4-bit nibble slot (see dot4_half); half (c, h) at (c*2 + h) * XH
     float2 x4z[MAX_C][2];                // per column and half: sums of x * 2^-100, even / odd codes
     float xlut[MAX_C];                   // per column: sum of the all-ones entries, in lookup order
-    float ys[2][RB];                     // row partials of the current and the previous unit
-    unsigned long long bar[2];           // one mbarrier per stage
-    alignas(16) uint8_t colarr[2][COLARR_BYTES];       // column of every item of the last two units (16-byte stores)
-    uint32_t epoch;                      // this call's epoch (split-K y zeroing)
-    int flag_ok;
+    float ys[NSTAGE][RB];                // row partials of the unit in each stage
+    unsigned long long full[NSTAGE];     // blob landed (TMA transaction count)
+    unsigned long long empty[NSTAGE];    // the unit's team is done (one arrival per team warp)
+    int abort;                           // set by any role whose wait ran out
 };
-static_assert(offsetof(Tables, colarr) % 16 == 0, "colarr takes 16-byte stores");
-static_assert(offsetof(Tables, bar) % 8 == 0, "mbarriers are 8-byte aligned");
+static_assert(offsetof(Tables, full) % 8 == 0, "mbarriers are 8-byte aligned");
 static_assert(offsetof(Tables, lut) == 0, "tables start at the aligned base");
-static_assert(RB <= THREADS, "one thread per row writes a unit's rows");
+static_assert(RB % 32 == 0, "the copier flushes rows a warp at a time");
+static_assert(MAX_C <= 32, "a warp holds a unit's column ends one per lane");
 
-constexpr size_t GEMV1_SMEM = 128 /* alignment slack */ + 2 * STAGE_BYTES + sizeof(Tables);
-// three blocks per SM: 3 x (GEMV1_SMEM + 1 KB reserved per block) must fit in 228 KB
-static_assert(3 * (GEMV1_SMEM + 1024) <= 228 * 1024, "three blocks per SM");
+constexpr size_t GEMV1_SMEM = 256 /* alignment slack */ + (size_t)NSTAGE * STAGE_BYTES + sizeof(Tables);
+static_assert(GEMV1_SMEM <= 227 * 1024, "one block per SM");
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -117,41 +133,56 @@ __device__ __forceinline__ uint32_t lds_u32(uint32_t addr) {
 
 __device__ __forceinline__ float2 f2(float a, float b) { return make_float2(a, b); }
 
-// Byte offset of nibble I (0..7) of w, scaled by 4 (a table entry is 4 bytes).
-template <int I>
-__device__ __forceinline__ uint32_t nib4(uint32_t w) {
-    return (I == 0 ? (w << 2) : (w >> (4 * I - 2))) & 0x3Cu;
+// y += v on a shared-memory float (32-bit shared address) / a global float.
+__device__ __forceinline__ void red_shared(uint32_t addr, float v) {
+    asm volatile("red.shared.add.f32 [%0], %1;" :: "r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void red_global(float* p, float v) {
+    asm volatile("red.global.add.f32 [%0], %1;" :: "l"(p), "f"(v) : "memory");
 }
 
-// Sum over the 16 nibbles of a 64-bit bit plane (words lo, hi) of the table
-// entries they select; tb = shared address of the column's tables. The 16
-// lookups are added as a balanced tree (pairs, then pairs of pairs), the same
-// tree that builds xlut.
+// The 16 table entries that a 64-bit bit plane (words lo, hi) selects from a
+// column's tables at tb (256-byte aligned): nibble p of the plane picks entry
+// m at tb + 64 p + 4 m. Even and odd nibbles are masked into the bytes of two
+// words as 4 m; a byte permute then merges one such byte with the upper bytes
+// of tb, so every lookup address costs one instruction.
+__device__ __forceinline__ void plane_entries(uint32_t tb, uint32_t lo, uint32_t hi, float (&v)[16]) {
+    const uint32_t M = 0x3C3C3C3Cu;
+    const uint32_t le = (lo << 2) & M, lo_ = (lo >> 2) & M, he = (hi << 2) & M, ho = (hi >> 2) & M;
+    v[0] = lds_f32<0>(__byte_perm(le, tb, 0x7650));
+    v[1] = lds_f32<64>(__byte_perm(lo_, tb, 0x7650));
+    v[2] = lds_f32<128>(__byte_perm(le, tb, 0x7651));
+    v[3] = lds_f32<192>(__byte_perm(lo_, tb, 0x7651));
+    v[4] = lds_f32<256>(__byte_perm(le, tb, 0x7652));
+    v[5] = lds_f32<320>(__byte_perm(lo_, tb, 0x7652));
+    v[6] = lds_f32<384>(__byte_perm(le, tb, 0x7653));
+    v[7] = lds_f32<448>(__byte_perm(lo_, tb, 0x7653));
+    v[8] = lds_f32<512>(__byte_perm(he, tb, 0x7650));
+    v[9] = lds_f32<576>(__byte_perm(ho, tb, 0x7650));
+    v[10] = lds_f32<640>(__byte_perm(he, tb, 0x7651));
+    v[11] = lds_f32<704>(__byte_perm(ho, tb, 0x7651));
+    v[12] = lds_f32<768>(__byte_perm(he, tb, 0x7652));
+    v[13] = lds_f32<832>(__byte_perm(ho, tb, 0x7652));
+    v[14] = lds_f32<896>(__byte_perm(he, tb, 0x7653));
+    v[15] = lds_f32<960>(__byte_perm(ho, tb, 0x7653));
+}
+
+// Sum of 16 values as a balanced tree (pairs, then pairs of pairs): the order
+// every lookup sum and xlut use.
 __device__ __forceinline__ float tree16(const float* v) {
     const float a0 = v[0] + v[1], a1 = v[2] + v[3], a2 = v[4] + v[5], a3 = v[6] + v[7];
     const float a4 = v[8] + v[9], a5 = v[10] + v[11], a6 = v[12] + v[13], a7 = v[14] + v[15];
     return ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
 }
 
-__device__ __forceinline__ float plane_sum(uint32_t tb, uint32_t lo, uint32_t hi) {
-    float v[16];
-    v[0] = lds_f32<0>(nib4<0>(lo) | tb);
-    v[1] = lds_f32<64>(nib4<1>(lo) | tb);
-    v[2] = lds_f32<128>(nib4<2>(lo) | tb);
-    v[3] = lds_f32<192>(nib4<3>(lo) | tb);
-    v[4] = lds_f32<256>(nib4<4>(lo) | tb);
-    v[5] = lds_f32<320>(nib4<5>(lo) | tb);
-    v[6] = lds_f32<384>(nib4<6>(lo) | tb);
-    v[7] = lds_f32<448>(nib4<7>(lo) | tb);
-    v[8] = lds_f32<512>(nib4<0>(hi) | tb);
-    v[9] = lds_f32<576>(nib4<1>(hi) | tb);
-    v[10] = lds_f32<640>(nib4<2>(hi) | tb);
-    v[11] = lds_f32<704>(nib4<3>(hi) | tb);
-    v[12] = lds_f32<768>(nib4<4>(hi) | tb);
-    v[13] = lds_f32<832>(nib4<5>(hi) | tb);
-    v[14] = lds_f32<896>(nib4<6>(hi) | tb);
-    v[15] = lds_f32<960>(nib4<7>(hi) | tb);
-    return tree16(v);
+// tree16 of a (in .x) and of b (in .y) at once, with f32x2 adds.
+__device__ __forceinline__ float2 tree16x2(const float (&a)[16], const float (&b)[16]) {
+    float2 p[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) p[i] = __fadd2_rn(f2(a[2 * i], b[2 * i]), f2(a[2 * i + 1], b[2 * i + 1]));
+    const float2 q0 = __fadd2_rn(p[0], p[1]), q1 = __fadd2_rn(p[2], p[3]);
+    const float2 q2 = __fadd2_rn(p[4], p[5]), q3 = __fadd2_rn(p[6], p[7]);
+    return __fadd2_rn(__fadd2_rn(q0, q1), __fadd2_rn(q2, q3));
 }
 
 // 4-bit, half a group per lane (32 codes: four words of LSB-first nibbles).
@@ -210,9 +241,11 @@ __device__ __forceinline__ void st_volatile(uint32_t* p, uint32_t v) {
 __device__ __forceinline__ float half_bits(uint32_t bits) { return __half2float(__ushort_as_half((uint16_t)bits)); }
 
 // ---------------------------------------------------------------------------
-// Unit blobs arrive by TMA bulk copy, completion tracked by one mbarrier per
-// stage. Every wait is bounded: after about a second the block records
-// VBQ_DEVICE_TIMEOUT in g_device_status and stops.
+// Unit blobs arrive by TMA bulk copy; roles hand stages over through
+// mbarriers. Every wait is bounded: after about a second (or as soon as another
+// role has given up) the waiting role records VBQ_DEVICE_TIMEOUT in
+// g_device_status, raises the block's abort flag and skips the rest of its
+// work; the copier lets every copy it started land before the block exits.
 // ---------------------------------------------------------------------------
 
 __device__ uint32_t g_device_status;
@@ -236,14 +269,52 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
                  : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
     return ok != 0;
 }
-// Wait until the barrier's phase with this parity completes; false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+// try_wait that lets the hardware suspend the thread for up to `hint` ns while
+// the phase is incomplete (it resumes as soon as the phase completes), so a
+// waiting warp issues a handful of instructions per wait instead of spinning.
+constexpr uint32_t SUSPEND_HINT_NS = 20000;
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(ok) : "r"(bar), "r"(parity), "n"(SUSPEND_HINT_NS) : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ int lds_volatile(uint32_t addr) {
+    int v;
+    asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(bar) : "memory");
+}
+// Wait until the barrier's phase with this parity completes. False when the
+// wait ran out or the block's abort flag (shared address abort_addr) is up.
+// A role off the critical path passes nap_ns > 0 to sleep between polls.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t abort_addr, uint32_t nap_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = global_ns();
-    while (!mbar_try_wait(bar, parity)) {
+    while (!mbar_try_wait_sleep(bar, parity)) {
+        if (nap_ns) __nanosleep(nap_ns);
+        if (lds_volatile(abort_addr) || global_ns() - t0 > WAIT_LIMIT_NS) return false;
+    }
+    return true;
+}
+// mbar_wait by a whole warp, with one verdict for all lanes (the roles' code
+// after a wait uses full-warp shuffles and must not diverge on it).
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint32_t abort_addr, uint32_t nap_ns = 0) {
+    return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_addr, nap_ns));
+}
+// Plain bounded wait (no abort flag), for the copier's final drain.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait_sleep(bar, parity)) {
         if (global_ns() - t0 > WAIT_LIMIT_NS) return false;
     }
     return true;
+}
+__device__ __forceinline__ void raise_abort(int* abort_flag) {
+    atomicOr(&g_device_status, VBQ_DEVICE_TIMEOUT);
+    *reinterpret_cast<volatile int*>(abort_flag) = 1;
 }
 // One thread: expect `bytes` on the barrier and start the bulk copy.
 __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
@@ -257,20 +328,28 @@ __device__ __forceinline__ void issue_unit(const LayoutView& L, int u, uint32_t 
     bulk_load(dst, L.blobs + (int64_t)o0 * 16, (o1 - o0) * 16, bar);
 }
 
-// Fill colarr[cb + a .. cb + e) with column c: bytes up to a 16-byte boundary,
-// 16-byte stores in between, bytes after.
-__device__ __forceinline__ void fill_run(uint32_t cb, int a, int e, int c) {
-    const uint32_t b4 = 0x01010101u * (uint32_t)c;
-    const int a16 = min((a + 15) & ~15, e), e16 = max(e & ~15, a16);
-    for (int i = a; i < a16; ++i) asm volatile("st.shared.u8 [%0], %1;" :: "r"(cb + i), "r"(c) : "memory");
-    for (int i = a16; i < e16; i += 16)
-        asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" :: "r"(cb + i), "r"(b4) : "memory");
-    for (int i = e16; i < e; ++i) asm volatile("st.shared.u8 [%0], %1;" :: "r"(cb + i), "r"(c) : "memory");
+// Consumer warps only (named barrier 1).
+__device__ __forceinline__ void consumer_sync() {
+    asm volatile("bar.sync 1, %0;" :: "n"(NCT) : "memory");
+}
+
+// Columns of a unit's items without a per-item array: lane t holds cend[t]
+// of one width (0xFFFF past the unit's last column), and item i of that width
+// lies in column #{t : cend[t] <= i}. A warp finds the columns of a task's
+// first and last items by one ballot each; only a task across column ends
+// (cf < cl) walks the few ends in between.
+__device__ __forceinline__ int col_uniform(uint32_t ce, int i) {   // i the same on every lane
+    return __popc(__ballot_sync(0xffffffffu, ce <= (uint32_t)i));
+}
+__device__ __forceinline__ int col_within(uint32_t ce, int cf, int cl, int i) {   // cf, cl the same on every lane
+    int c = cf;
+    for (int t = cf; t < cl; ++t) c += __shfl_sync(0xffffffffu, ce, t) <= (uint32_t)i;
+    return c;
 }
 
 // Split-K: true once every row block this block adds a slab s > 0 into has
-// been zeroed in this call (flag == epoch), within the wait limit. Thread 0
-// only; ends with an acquire fence.
+// been zeroed in this call (flag == epoch), within the wait limit. One thread;
+// ends with an acquire fence.
 __device__ __forceinline__ bool split_k_flags_ready(const LayoutView& L, uint32_t epoch, int u_begin, int u_end,
                                                     int s0, int rb0) {
     bool seen = true;
@@ -287,250 +366,304 @@ __device__ __forceinline__ bool split_k_flags_ready(const LayoutView& L, uint32_
     return seen;
 }
 
-// A finished unit's row partials ys (row block rbw) go to y: stored when the
-// row has one slab, added otherwise; ys is zeroed for reuse.
-__device__ __forceinline__ void write_rows(const LayoutView& L, float* y, float* ys, int rbw, int tid) {
-    if (tid >= RB) return;
-    const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
-    const float v = ys[tid];
-    ys[tid] = 0.f;
-    if (tid < rows) {
-        float* dst = y + (int64_t)rbw * RB + tid;
-        if (L.S == 1) *dst = v;
-        else atomicAdd(dst, v);
+// Activations of slab s: x as fp32, the pre-scaled x of the 4-bit slots, the
+// nibble lookup tables, and the per-column sums in lookup order. Consumer
+// threads only (ct = 0 .. NCT-1); starts and ends with a consumer barrier.
+__device__ void build_tables(Tables& T, const LayoutView& L, const uint16_t* __restrict__ x, int s, int ct) {
+    const int cols = min(L.C, L.G - s * L.C);
+    const int64_t k0 = (int64_t)s * L.C * GROUP;
+    consumer_sync();                // nobody still reads the old tables
+    for (int i = ct; i < cols * 32; i += NCT) {
+        const uint32_t two = __ldg(reinterpret_cast<const uint32_t*>(x + k0) + i);
+        const float xa = __uint_as_float(two << 16), xb = __uint_as_float(two & 0xFFFF0000u);
+        const int kk = 2 * i, c = kk >> 6, jj = kk & 63;
+        *reinterpret_cast<float2*>(&T.xs[(c * 4 + (jj >> 4)) * XQ + (jj & 15)]) = f2(xa, xb);
+        // 4-bit slot shifts: nibble slots 0..5 of a word keep their place, 6 and 7 come down by 24
+        const int slot = jj & 7, e = slot < 6 ? 4 * slot : 4 * (slot - 6);
+        *reinterpret_cast<float2*>(&T.x4s[(c * 2 + (jj >> 5)) * XH + (jj & 31)]) =
+            f2(xa * __uint_as_float((uint32_t)(127 + 49 - e) << 23),
+               xb * __uint_as_float((uint32_t)(127 + 49 - e - 4) << 23));
+    }
+    consumer_sync();
+    for (int pj = ct; pj < cols * 16; pj += NCT) {
+        const int c = pj >> 4, jn = pj & 15;
+        const float4 xv = *reinterpret_cast<const float4*>(&T.xs[(c * 4 + (jn >> 2)) * XQ + 4 * (jn & 3)]);
+        const float t3 = xv.x + xv.y, t12 = xv.w + xv.z;
+        float4* dst = reinterpret_cast<float4*>(T.lut + c * LUT_COL_BYTES + jn * 64);
+        dst[0] = make_float4(0.f, xv.x, xv.y, t3);
+        dst[1] = make_float4(xv.z, xv.z + xv.x, xv.z + xv.y, xv.z + t3);
+        dst[2] = make_float4(xv.w, xv.w + xv.x, xv.w + xv.y, xv.w + t3);
+        dst[3] = make_float4(t12, t12 + xv.x, t12 + xv.y, t12 + t3);
+    }
+    consumer_sync();
+    if (ct < cols) {
+        const float* t = reinterpret_cast<const float*>(T.lut + ct * LUT_COL_BYTES);
+        float v[16];
+#pragma unroll
+        for (int jn = 0; jn < 16; ++jn) v[jn] = t[jn * 16 + 15];
+        T.xlut[ct] = tree16(v);
+        // X for the 4-bit zero level, summed as dot4_half accumulates
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
+#pragma unroll
+            for (int t4 = 0; t4 < 4; ++t4) {
+                float2& cc = (t4 & 1) ? cb : ca;
+#pragma unroll
+                for (int e = 0; e < 8; e += 2) {
+                    const int jj = 32 * hh + 8 * t4 + e;
+                    const float* xq = &T.xs[(ct * 4 + (jj >> 4)) * XQ + (jj & 15)];
+                    cc = __ffma2_rn(f2(xq[0], xq[1]), f2(0x1p-100f, 0x1p-100f), cc);
+                }
+            }
+            T.x4z[ct][hh] = __fadd2_rn(ca, cb);
+        }
+    }
+    consumer_sync();
+}
+
+// One consumer warp's share of a unit (blob at shared address sblob, cols
+// group columns): tasks t = t0, t0 + tstep, ... of 16 four-bit groups (two
+// lanes each), 8 eight-bit groups (four lanes each), 32 two-bit groups, 64
+// one-bit groups (two per lane). Partials go to the row partials at shared
+// address ys by shared-memory reductions.
+__device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, int C, int cols, uint32_t ys,
+                                             int t0, int tstep, int lane) {
+    const uint32_t lut0 = smem_u32(T.lut), xs0 = smem_u32(T.xs), x4s0 = smem_u32(T.x4s);
+    const uint32_t x4z0 = smem_u32(T.x4z), xlut0 = smem_u32(T.xlut);
+    // UnitHeader fields, read as three 16-byte words
+    const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
+    const int n0 = h0.x & 0xFFFF, n1 = h0.x >> 16, n2 = h0.y & 0xFFFF, n3 = h0.y >> 16;
+    const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
+    uint32_t ce[4];                                     // this lane's column end of each width
+#pragma unroll
+    for (int w = 0; w < 4; ++w) ce[w] = lane < cols ? lds_u16(cc + 2 * (w * C + lane)) : 0xFFFFu;
+    const int t4 = (n2 + 15) >> 4, t48 = t4 + ((n3 + 7) >> 3), t482 = t48 + ((n1 + 31) >> 5);
+    const int ntask = t482 + ((n0 + 63) >> 6);
+    for (int t = t0; t < ntask; t += tstep) {
+        if (t < t4) {                                   // 4-bit: two lanes per group, one half each
+            const uint32_t pay = sblob + (h0.w & 0xFFFF) * 16, sc = sblob + (h1.y & 0xFFFF) * 16;
+            const uint32_t row = sblob + (h1.w & 0xFFFF) * 16;
+            // lanes l and l+16 share group l%16; the half is swizzled so that a
+            // quarter-warp reads 8 distinct 16-byte bank groups
+            const int e = lane & 15, hh = ((e >> 2) + (lane >> 4)) & 1;
+            const int i0 = t * 16, i = i0 + e;
+            const int cf = col_uniform(ce[2], i0), cl = col_uniform(ce[2], min(i0 + 15, n2 - 1));
+            const int c = col_within(ce[2], cf, cl, i);
+            float part = 0.f;
+            if (i < n2) {
+                const uint4 v = lds_u32x4(pay + i * 32 + hh * 16);
+                const float2 acc = dot4_half(v, x4s0 + (c * 2 + hh) * XH * 4);
+                const float2 z = lds_f32x2(x4z0 + (c * 2 + hh) * 8);
+                part = (acc.x - 8.f * z.x) + (acc.y - 8.f * z.y);
+            }
+            part += __shfl_xor_sync(0xffffffffu, part, 16);
+            if (i < n2 && lane < 16)
+                red_shared(ys + 4 * lds_u8(row + i), (half_bits(lds_u16(sc + 2 * i)) * 0x1p100f) * part);
+        } else if (t < t48) {                           // 8-bit: four lanes per group, one quarter each
+            const uint32_t pay = sblob + (h0.w >> 16) * 16, sc = sblob + (h1.y >> 16) * 16;
+            const uint32_t row = sblob + (h1.w >> 16) * 16;
+            // lane 8k + e takes quarter ((e >> 1) + k) % 4 of group e: a quarter-warp
+            // reads 8 distinct 16-byte bank groups
+            const int e = lane & 7, q = ((e >> 1) + (lane >> 3)) & 3;
+            const int i0 = (t - t4) * 8, i = i0 + e;
+            const int cf = col_uniform(ce[3], i0), cl = col_uniform(ce[3], min(i0 + 7, n3 - 1));
+            const int c = col_within(ce[3], cf, cl, i);
+            float part = 0.f;
+            if (i < n3) {
+                const uint4 v = lds_u32x4(pay + i * 64 + q * 16);
+                part = dot8_quarter(v, xs0 + (c * 4 + q) * XQ * 4);
+            }
+            part += __shfl_xor_sync(0xffffffffu, part, 8);
+            part += __shfl_xor_sync(0xffffffffu, part, 16);
+            if (i < n3 && lane < 8)
+                red_shared(ys + 4 * lds_u8(row + i), half_bits(lds_u16(sc + 2 * i)) * part);
+        } else if (t < t482) {                          // 2-bit: one group per lane, both planes at once
+            const uint32_t pay = sblob + (h0.z >> 16) * 16, sc = sblob + (h1.x >> 16) * 16;
+            const uint32_t row = sblob + (h1.z >> 16) * 16;
+            const int i0 = (t - t48) * 32, i = i0 + lane;
+            const int cf = col_uniform(ce[1], i0), cl = col_uniform(ce[1], min(i0 + 31, n1 - 1));
+            const int c = col_within(ce[1], cf, cl, i);
+            if (i < n1) {
+                const uint4 pl = lds_u32x4(pay + i * 16);
+                const uint32_t tb = lut0 + c * LUT_COL_BYTES;
+                float va[16], vb[16];
+                plane_entries(tb, pl.x, pl.y, va);
+                plane_entries(tb, pl.z, pl.w, vb);
+                const float2 sp = tree16x2(va, vb);
+                red_shared(ys + 4 * lds_u8(row + i),
+                           half_bits(lds_u16(sc + 2 * i)) * (sp.x + 2.f * (sp.y - lds_f32r(xlut0 + 4 * c))));
+            }
+        } else {                                        // 1-bit: two groups per lane, summed as a pair
+            const uint32_t pay = sblob + (h0.z & 0xFFFF) * 16, sc = sblob + (h1.x & 0xFFFF) * 16;
+            const uint32_t row = sblob + (h1.z & 0xFFFF) * 16;
+            const int i0 = (t - t482) * 64, i = i0 + 2 * lane;
+            const int cf = col_uniform(ce[0], i0), cl = col_uniform(ce[0], min(i0 + 63, n0 - 1));
+            int ca = cf, cb = cf;
+            if (cf != cl) {
+                ca = col_within(ce[0], cf, cl, i);
+                cb = col_within(ce[0], cf, cl, min(i + 1, n0 - 1));
+            }
+            if (i < n0) {
+                const bool two = i + 1 < n0;
+                const uint4 v = lds_u32x4(pay + i * 8);
+                const uint32_t rows2 = lds_u16(row + i);
+                const uint32_t sc2 = lds_u32(sc + 2 * i);
+                float va[16], vb[16];
+                plane_entries(lut0 + ca * LUT_COL_BYTES, v.x, v.y, va);
+                plane_entries(lut0 + cb * LUT_COL_BYTES, v.z, v.w, vb);
+                const float2 sp = tree16x2(va, vb);
+                if (two)
+                    red_shared(ys + 4 * (rows2 >> 8), half_bits(sc2 >> 16) * (2.f * sp.y - lds_f32r(xlut0 + 4 * cb)));
+                red_shared(ys + 4 * (rows2 & 0xff), half_bits(sc2) * (2.f * sp.x - lds_f32r(xlut0 + 4 * ca)));
+            }
+        }
     }
 }
 
-__global__ void __launch_bounds__(THREADS, 3) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
-                                                           float* __restrict__ y) {
+__global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
+                                                              float* __restrict__ y) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    // stages and tables on a 128-byte boundary: lookups OR a nibble offset into table addresses
-    unsigned char* base = smem_raw + ((128u - (smem_u32(smem_raw) & 127u)) & 127u);
-    Tables& T = *reinterpret_cast<Tables*>(base + 2 * STAGE_BYTES);
+    // stages and tables on a 256-byte boundary: lookups merge a byte into table addresses
+    unsigned char* base = smem_raw + ((256u - (smem_u32(smem_raw) & 255u)) & 255u);
+    Tables& T = *reinterpret_cast<Tables*>(base + (size_t)NSTAGE * STAGE_BYTES);
     const uint32_t stage0 = smem_u32(base);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int P = gridDim.x, p = blockIdx.x;
-    const int u_begin = (int)((int64_t)L.units * p / P), u_end = (int)((int64_t)L.units * (p + 1) / P);
-    if (u_begin >= u_end) return;
+    // balanced contiguous split of the units over the blocks
+    const int per = L.units / P, extra = L.units - per * P;
+    const int u_begin = p * per + min(p, extra), u_end = u_begin + per + (p < extra ? 1 : 0);
+    const int n_units = u_end - u_begin;
+    if (n_units <= 0) return;
+    const int s0 = u_begin / L.nrb, rb0 = u_begin - s0 * L.nrb;
+    // more units per block -> more teams: each warp then covers more groups per
+    // unit (less per-unit overhead); few units -> whole-block teams (less latency)
+    const int lg_teams = n_units >= 4 * MAX_TEAMS ? 2 : n_units >= 8 ? 1 : 0;
+    const int teams = 1 << lg_teams, tw = NCW >> lg_teams;
 
-    const uint32_t bar0 = smem_u32(&T.bar[0]);
+    const uint32_t full0 = smem_u32(&T.full[0]), empty0 = smem_u32(&T.empty[0]);
+    const uint32_t abort_addr = smem_u32(&T.abort);
     if (tid == 0) {
-        mbar_init(bar0, 1);
-        mbar_init(bar0 + 8, 1);
+        for (int i = 0; i < NSTAGE; ++i) {
+            mbar_init(full0 + 8 * i, 1);
+            mbar_init(empty0 + 8 * i, tw);
+        }
+        T.abort = 0;
         fence_barrier_init();
     }
+    for (int i = tid; i < NSTAGE * RB; i += G1_THREADS) (&T.ys[0][0])[i] = 0.f;
     __syncthreads();
     if (tid == 0) {
-        issue_unit(L, u_begin, stage0, bar0);
-        if (u_begin + 1 < u_end) issue_unit(L, u_begin + 1, stage0 + STAGE_BYTES, bar0 + 8);
+        const int first = n_units < NSTAGE ? n_units : NSTAGE;
+        for (int j = 0; j < first; ++j) issue_unit(L, u_begin + j, stage0 + j * STAGE_BYTES, full0 + 8 * j);
     }
-    // Weights never depend on earlier work in the stream, so their first copies
+    // Weights never depend on earlier work in the stream, so the first copies
     // are in flight before this grid waits for its predecessor (programmatic
-    // dependent launch); x, y and the workspace are touched only after the wait.
+    // dependent launch); x, y and the control words are touched only after.
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    if (L.S > 1) {
-        // split-K: this call's epoch; zero y for the row blocks whose slab 0 this
-        // block owns (units u < nrb) and publish them
-        if (tid == 0) T.epoch = ld_volatile(L.ctl) + 1u;
-        const int z_end = min(u_end, L.nrb);
-        for (int u = u_begin; u < z_end; ++u) {
-            float* dst = y + (int64_t)u * RB;
-            const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
-            for (int r = tid; r < rows; r += THREADS) dst[r] = 0.f;
-        }
-        __syncthreads();
-        if (tid == 0 && u_begin < z_end) {
-            __threadfence();
-            for (int u = u_begin; u < z_end; ++u) st_volatile(L.ctl + 2 + u, T.epoch);
-        }
-    }
-    for (int i = tid; i < 2 * RB; i += THREADS) (&T.ys[0][0])[i] = 0.f;
 
-    const uint32_t lut0 = smem_u32(T.lut), xs0 = smem_u32(T.xs), x4s0 = smem_u32(T.x4s);
-    const uint32_t x4z0 = smem_u32(T.x4z), xlut0 = smem_u32(T.xlut), cola0 = smem_u32(&T.colarr[0][0]);
-    const int s0 = u_begin / L.nrb, rb0 = u_begin - s0 * L.nrb;
-    int s = s0, rb = rb0, prev_rb = rb0;
-    int cur_slab = -1;
-    bool ok = true;
-    bool checked = L.S == 1;            // split-K zeroing flags verified (or not needed)
-    for (int k = u_begin; k < u_end; ++k) {
-        const int j = k - u_begin, buf = j & 1;
-        const unsigned char* blob = base + buf * STAGE_BYTES;
-        const uint32_t sblob = stage0 + buf * STAGE_BYTES;
-        const int cols = min(L.C, L.G - s * L.C);
-        float* ys = T.ys[buf];
-        const uint32_t cola = cola0 + buf * COLARR_BYTES;
-
-        if (s != cur_slab) {            // activations of a new slab: x, tables, X sums
-            const int64_t k0 = (int64_t)s * L.C * GROUP;
-            __syncthreads();            // nobody still reads the old tables
-            for (int i = tid; i < cols * 32; i += THREADS) {
-                const uint32_t two = __ldg(reinterpret_cast<const uint32_t*>(x + k0) + i);
-                const float xa = __uint_as_float(two << 16), xb = __uint_as_float(two & 0xFFFF0000u);
-                const int kk = 2 * i, c = kk >> 6, jj = kk & 63;
-                *reinterpret_cast<float2*>(&T.xs[(c * 4 + (jj >> 4)) * XQ + (jj & 15)]) = f2(xa, xb);
-                // 4-bit slot shifts: nibble slots 0..5 of a word keep their place, 6 and 7 come down by 24
-                const int slot = jj & 7, e = slot < 6 ? 4 * slot : 4 * (slot - 6);
-                *reinterpret_cast<float2*>(&T.x4s[(c * 2 + (jj >> 5)) * XH + (jj & 31)]) =
-                    f2(xa * __uint_as_float((uint32_t)(127 + 49 - e) << 23),
-                       xb * __uint_as_float((uint32_t)(127 + 49 - e - 4) << 23));
+    if (warp == 0) {
+        // ---- copier: split-K zeroing, then per unit: rows out, next copy in ----
+        uint32_t epoch = 0;
+        if (L.S > 1) {
+            // this call's epoch; zero y for the row blocks whose slab 0 this block
+            // owns (units u < nrb) and publish them
+            epoch = ld_volatile(L.ctl) + 1u;
+            const int z_end = min(u_end, L.nrb);
+            for (int u = u_begin; u < z_end; ++u) {
+                float* dst = y + (int64_t)u * RB;
+                const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
+                for (int r = lane; r < rows; r += 32) dst[r] = 0.f;
             }
-            __syncthreads();
-            for (int pj = tid; pj < cols * 16; pj += THREADS) {
-                const int c = pj >> 4, jn = pj & 15;
-                const float4 xv = *reinterpret_cast<const float4*>(&T.xs[(c * 4 + (jn >> 2)) * XQ + 4 * (jn & 3)]);
-                const float t3 = xv.x + xv.y, t12 = xv.w + xv.z;
-                float4* dst = reinterpret_cast<float4*>(T.lut + c * LUT_COL_BYTES + jn * 64);
-                dst[0] = make_float4(0.f, xv.x, xv.y, t3);
-                dst[1] = make_float4(xv.z, xv.z + xv.x, xv.z + xv.y, xv.z + t3);
-                dst[2] = make_float4(xv.w, xv.w + xv.x, xv.w + xv.y, xv.w + t3);
-                dst[3] = make_float4(t12, t12 + xv.x, t12 + xv.y, t12 + t3);
+            __syncwarp();
+            if (lane == 0 && u_begin < z_end) {
+                __threadfence();
+                for (int u = u_begin; u < z_end; ++u) st_volatile(L.ctl + 2 + u, epoch);
             }
-            __syncthreads();
-            if (tid < cols) {
-                const float* t = reinterpret_cast<const float*>(T.lut + tid * LUT_COL_BYTES);
-                float v[16];
-#pragma unroll
-                for (int jn = 0; jn < 16; ++jn) v[jn] = t[jn * 16 + 15];
-                T.xlut[tid] = tree16(v);
-                // X for the 4-bit zero level, summed as dot4_half accumulates
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
-                    for (int t4 = 0; t4 < 4; ++t4) {
-                        float2& cc = (t4 & 1) ? cb : ca;
-                        for (int e = 0; e < 8; e += 2) {
-                            const int jj = 32 * hh + 8 * t4 + e;
-                            const float* xq = &T.xs[(tid * 4 + (jj >> 4)) * XQ + (jj & 15)];
-                            cc = __ffma2_rn(f2(xq[0], xq[1]), f2(0x1p-100f, 0x1p-100f), cc);
-                        }
-                    }
-                    T.x4z[tid][hh] = __fadd2_rn(ca, cb);
-                }
-            }
-            cur_slab = s;
         }
-
-        ok = mbar_wait(bar0 + 8 * buf, (j >> 1) & 1);   // unit k's blob has landed (each thread waits)
-        const UnitHeader h = *reinterpret_cast<const UnitHeader*>(blob);
-        const int n0 = h.n[0], n1 = h.n[1], n2 = h.n[2], n3 = h.n[3];
-        const uint32_t cb1 = (n0 + 15) & ~15, cb2 = cb1 + ((n1 + 15) & ~15), cb3 = cb2 + ((n2 + 15) & ~15);
-        if (ok && tid < 4 * cols) {     // one thread per (width, column) run
-            const uint16_t* cend = reinterpret_cast<const uint16_t*>(blob + h.cc16 * 16);
-            const int w = tid / cols, c = tid - w * cols;
-            const int a = c == 0 ? 0 : cend[w * L.C + c - 1], e = cend[w * L.C + c];
-            const uint32_t cb = cola + (w == 0 ? 0u : w == 1 ? cb1 : w == 2 ? cb2 : cb3);
-            fill_run(cb, a, e, c);
-        }
-        if (!checked && j == 1 && tid == 0) T.flag_ok = split_k_flags_ready(L, T.epoch, u_begin, u_end, s0, rb0);
-        // one barrier per unit: unit k's column array is complete and every warp
-        // has finished unit k-1, whose stage, rows and partials are now free
-        if (!__syncthreads_and(ok)) break;
-        if (j >= 1) {
-            if (!checked) {
+        bool dead = false, checked = L.S == 1;
+        int st = 0, rbw = rb0, issued = n_units < NSTAGE ? n_units : NSTAGE;
+        uint32_t par = 0;
+        for (int j = 0; j < n_units; ++j) {
+            if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 256)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
+            if (!dead && !checked) {
+                // before the first add into y: every row block this block adds a
+                // slab s > 0 into has been zeroed in this call
+                int ok = 1;
+                if (lane == 0) ok = split_k_flags_ready(L, epoch, u_begin, u_end, s0, rb0);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
                 checked = true;
-                if (!T.flag_ok) { ok = false; break; }
+                if (!ok) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             }
-            if (tid == 0 && k + 1 < u_end) issue_unit(L, k + 1, stage0 + (buf ^ 1) * STAGE_BYTES, bar0 + 8 * (buf ^ 1));
-            write_rows(L, y, T.ys[buf ^ 1], prev_rb, tid);
-        }
-
-        // warp tasks: 16 four-bit groups (two lanes each), 8 eight-bit groups
-        // (four lanes each), 32 two-bit groups, 64 one-bit groups (two per lane)
-        const int t4 = (n2 + 15) >> 4, t8 = (n3 + 7) >> 3, t2 = (n1 + 31) >> 5, t1 = (n0 + 63) >> 6;
-        const int ntask = t4 + t8 + t2 + t1;
-        for (int t = warp; t < ntask; t += WARPS) {
-            if (t < t4) {                                   // 4-bit: two lanes per group, one half each
-                // lanes l and l+16 share group l%16; the half is swizzled so that a
-                // quarter-warp reads 8 distinct 16-byte bank groups
-                const int e = lane & 15, hh = ((e >> 2) + (lane >> 4)) & 1;
-                const int i = t * 16 + e;
-                float part = 0.f;
-                if (i < n2) {
-                    const uint4 v = lds_u32x4(sblob + h.pay16[2] * 16 + i * 32 + hh * 16);
-                    const int c = lds_u8(cola + cb2 + i);
-                    const float2 acc = dot4_half(v, x4s0 + (c * 2 + hh) * XH * 4);
-                    const float2 z = lds_f32x2(x4z0 + (c * 2 + hh) * 8);
-                    part = (acc.x - 8.f * z.x) + (acc.y - 8.f * z.y);
-                }
-                part += __shfl_xor_sync(0xffffffffu, part, 16);
-                if (i < n2 && lane < 16) {
-                    const int r = lds_u8(sblob + h.row16[2] * 16 + i);
-                    atomicAdd(&ys[r], (half_bits(lds_u16(sblob + h.sc16[2] * 16 + 2 * i)) * 0x1p100f) * part);
-                }
-            } else if (t < t4 + t8) {                       // 8-bit: four lanes per group, one quarter each
-                // lane 8k + e takes quarter ((e >> 1) + k) % 4 of group e: a quarter-warp
-                // reads 8 distinct 16-byte bank groups
-                const int e = lane & 7, q = ((e >> 1) + (lane >> 3)) & 3;
-                const int i = (t - t4) * 8 + e;
-                float part = 0.f;
-                if (i < n3) {
-                    const uint4 v = lds_u32x4(sblob + h.pay16[3] * 16 + i * 64 + q * 16);
-                    const int c = lds_u8(cola + cb3 + i);
-                    part = dot8_quarter(v, xs0 + (c * 4 + q) * XQ * 4);
-                }
-                part += __shfl_xor_sync(0xffffffffu, part, 8);
-                part += __shfl_xor_sync(0xffffffffu, part, 16);
-                if (i < n3 && lane < 8) {
-                    const int r = lds_u8(sblob + h.row16[3] * 16 + i);
-                    atomicAdd(&ys[r], half_bits(lds_u16(sblob + h.sc16[3] * 16 + 2 * i)) * part);
-                }
-            } else if (t < t4 + t8 + t2) {                  // 2-bit: one group per lane
-                const int i = (t - t4 - t8) * 32 + lane;
-                if (i < n1) {
-                    const uint4 pl = lds_u32x4(sblob + h.pay16[1] * 16 + i * 16);
-                    const int c = lds_u8(cola + cb1 + i);
-                    const uint32_t tb = lut0 + c * LUT_COL_BYTES;
-                    const float s0 = plane_sum(tb, pl.x, pl.y);
-                    const float s1 = plane_sum(tb, pl.z, pl.w);
-                    const int r = lds_u8(sblob + h.row16[1] * 16 + i);
-                    atomicAdd(&ys[r], half_bits(lds_u16(sblob + h.sc16[1] * 16 + 2 * i)) *
-                                          (s0 + 2.f * (s1 - lds_f32r(xlut0 + 4 * c))));
-                }
-            } else {                                        // 1-bit: two groups per lane
-                const int i = (t - t4 - t8 - t2) * 64 + 2 * lane;
-                if (i < n0) {
-                    const uint4 v = lds_u32x4(sblob + h.pay16[0] * 16 + i * 8);
-                    const uint32_t rows2 = lds_u16(sblob + h.row16[0] * 16 + i);
-                    const uint32_t sc2 = lds_u32(sblob + h.sc16[0] * 16 + 2 * i);
-                    const uint32_t cols2 = lds_u16(cola + i);
-                    const int ca = cols2 & 0xff;
-                    const float suma = plane_sum(lut0 + ca * LUT_COL_BYTES, v.x, v.y);
-                    if (i + 1 < n0) {
-                        const int cb = cols2 >> 8;
-                        const float sumb = plane_sum(lut0 + cb * LUT_COL_BYTES, v.z, v.w);
-                        atomicAdd(&ys[rows2 >> 8], half_bits(sc2 >> 16) * (2.f * sumb - lds_f32r(xlut0 + 4 * cb)));
+            if (!dead) {
+                float* ys = T.ys[st];
+                const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
+                float* yr = y + (int64_t)rbw * RB;
+#pragma unroll
+                for (int q = 0; q < RB / 32; ++q) {
+                    const int r = lane + 32 * q;
+                    const float v = ys[r];
+                    ys[r] = 0.f;
+                    if (r < rows) {
+                        if (L.S == 1) yr[r] = v;
+                        else red_global(yr + r, v);
                     }
-                    atomicAdd(&ys[rows2 & 0xff], half_bits(sc2) * (2.f * suma - lds_f32r(xlut0 + 4 * ca)));
+                }
+                __syncwarp();
+                if (j + NSTAGE < n_units) {
+                    if (lane == 0) issue_unit(L, u_begin + j + NSTAGE, stage0 + st * STAGE_BYTES, full0 + 8 * st);
+                    ++issued;
                 }
             }
+            if (++st == NSTAGE) { st = 0; par ^= 1; }
+            if (++rbw == L.nrb) rbw = 0;
         }
-        prev_rb = rb;
-        if (++rb == L.nrb) { rb = 0; ++s; }
-    }
-    if (ok) {                           // the last unit's rows
-        if (!checked && tid == 0) T.flag_ok = split_k_flags_ready(L, T.epoch, u_begin, u_end, s0, rb0);
-        __syncthreads();
-        if (!checked && !T.flag_ok) ok = false;
-        else write_rows(L, y, T.ys[(u_end - 1 - u_begin) & 1], prev_rb, tid);
-    }
-    if (!ok) {
-        // a copy or a flag never arrived: record it, give the outstanding copies a
-        // bounded time to land, and stop
-        if (tid == 0) {
-            atomicOr(&g_device_status, VBQ_DEVICE_TIMEOUT);
-            mbar_wait(bar0, 0);
-            mbar_wait(bar0 + 8, 0);
+        if (dead && lane == 0) {
+            // let every copy this block started land before the block exits: the
+            // last unit issued into each stage, with that unit's parity (a phase
+            // that already completed returns at once)
+            for (int i = 0; i < NSTAGE && i < issued; ++i) {
+                const int jl = i + ((issued - 1 - i) / NSTAGE) * NSTAGE;   // last unit issued into stage i
+                mbar_wait_bounded(full0 + 8 * i, (uint32_t)((jl / NSTAGE) & 1));
+            }
         }
-    }
-    if (L.S > 1 && tid == 0) {
-        // the last block of the call advances the epoch for the next call
-        __threadfence();
-        if (atomicAdd(L.ctl + 1, 1u) == gridDim.x - 1) {
-            st_volatile(L.ctl + 1, 0u);
-            st_volatile(L.ctl, T.epoch);
+        if (L.S > 1 && lane == 0) {
+            // the last block of the call advances the epoch for the next call
+            __threadfence();
+            if (atomicAdd(L.ctl + 1, 1u) == gridDim.x - 1) {
+                st_volatile(L.ctl + 1, 0u);
+                st_volatile(L.ctl, epoch);
+            }
         }
+    } else {
+        // ---- consumers: team `team` takes units j = team, team + teams, ... ----
+        const int cw = warp - 1, ct = tid - 32, team = cw / tw, wt = cw - team * tw;
+        const int s_last = (u_end - 1) / L.nrb;
+        bool dead = false;
+        int cur = s0;
+        int rbj = rb0 + team, sj = s0;                  // row block and slab of unit j
+        while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
+        build_tables(T, L, x, s0, ct);
+        for (int j = team; j < n_units; j += teams) {
+            // every consumer warp rebuilds the tables at every slab boundary of the
+            // block's range, in order (the rebuild's named barrier waits for all)
+            while (cur < sj) build_tables(T, L, x, ++cur, ct);
+            const int st = j & (NSTAGE - 1);
+            const uint32_t par = (uint32_t)(j / NSTAGE) & 1u;
+            if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
+            if (!dead) {
+                // tasks rotate over the team's warps from unit to unit, so no warp always draws the costly ones
+                const int t0 = (wt - (j >> lg_teams)) & (tw - 1);
+                consume_unit(T, stage0 + st * STAGE_BYTES, L.C, min(L.C, L.G - sj * L.C), smem_u32(T.ys[st]), t0,
+                             tw, lane);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty0 + 8 * st);
+            }
+            rbj += teams;
+            while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
+        }
+        while (cur < s_last) build_tables(T, L, x, ++cur, ct);   // boundaries past this team's last unit
     }
 }
 
@@ -634,10 +767,10 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
         if ((e = cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
         attr_set = true;
     }
-    const int grid = L.units < 3 * g_sms ? L.units : 3 * g_sms;
+    const int grid = L.units < g_sms ? L.units : g_sms;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(THREADS);
+    cfg.blockDim = dim3(G1_THREADS);
     cfg.dynamicSmemBytes = GEMV1_SMEM;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
