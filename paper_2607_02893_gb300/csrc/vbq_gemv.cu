@@ -52,7 +52,7 @@ constexpr int NCT = 32 * NCW;            // consumer threads
 constexpr int MAX_TEAMS = 4;             // consumer teams (1, 2 or 4 by units per block); unit j goes to team j % teams
 static_assert(NCW == 16 && MAX_TEAMS == 4, "teams of 16, 8 or 4 warps (powers of two)");
 constexpr int G1_THREADS = 32 * (NCW + 1);
-constexpr int NSTAGE = 8;                // blob stages in flight per SM
+constexpr int NSTAGE = 4;                // blob stages in flight per SM
 static_assert((NSTAGE & (NSTAGE - 1)) == 0, "power-of-two stage count");
 constexpr int XQ = 20;                   // floats per 16-code quarter of x (16 + 4 pad: quarters use other banks)
 constexpr int XH = 36;                   // floats per 32-code half of the pre-scaled x (32 + 4 pad)
