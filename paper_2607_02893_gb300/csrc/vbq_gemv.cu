@@ -56,12 +56,13 @@ constexpr int NSTAGE = 4;                // blob stages in flight per SM
 static_assert((NSTAGE & (NSTAGE - 1)) == 0, "power-of-two stage count");
 constexpr int XQ = 20;                   // floats per 16-code quarter of x (16 + 4 pad: quarters use other banks)
 constexpr int XH = 36;                   // floats per 32-code half of the pre-scaled x (32 + 4 pad)
-constexpr int LUT_COL_BYTES = 1024;      // 16 tables x 64 bytes per column, columns on 256-byte boundaries
+constexpr int LUT_COL_BYTES = 1280;      // 16 tables x 64 bytes (+64 for odd columns), columns on 256-byte boundaries
 constexpr int STAGE_BYTES = MAX_BLOB_BYTES;   // holds the largest unit blob (the packer guarantees it)
 static_assert(STAGE_BYTES % 256 == 0, "stages keep the tables 256-byte aligned");
+static_assert(LUT_COL_BYTES % 256 == 0 && 64 + 16 * 64 <= LUT_COL_BYTES, "column tables: 256-byte aligned, room for the odd shift");
 
 struct __align__(16) Tables {
-    uint8_t lut[MAX_C * LUT_COL_BYTES];  // column c, nibble j, entry m at c*1024 + j*64 + m*4
+    uint8_t lut[MAX_C * LUT_COL_BYTES];  // column c, nibble j, entry m at c*1280 + (c&1)*64 + j*64 + m*4
     float xs[MAX_C * 4 * XQ];            // x as fp32; quarter (c, q) at (c*4 + q) * XQ
     float x4s[MAX_C * 2 * XH];           // x pre-scaled per 4-bit nibble slot (see dot4_half); half (c, h) at (c*2 + h) * XH
     float2 x4z[MAX_C][2];                // per column and half: sums of x * 2^-100, even / odd codes
@@ -143,12 +144,17 @@ __device__ __forceinline__ void red_global(float* p, float v) {
 
 // The 16 table entries that a 64-bit bit plane (words lo, hi) selects from a
 // column's tables at tb (256-byte aligned): nibble p of the plane picks entry
-// m at tb + 64 p + 4 m. Even and odd nibbles are masked into the bytes of two
-// words as 4 m; a byte permute then merges one such byte with the upper bytes
-// of tb, so every lookup address costs one instruction.
-__device__ __forceinline__ void plane_entries(uint32_t tb, uint32_t lo, uint32_t hi, float (&v)[16]) {
+// m at tb + sh + 64 p + 4 m, where sh is 64 for odd columns and 0 for even
+// ones (odd columns sit in the other half of the banks, so a warp whose lanes
+// straddle two columns reads without bank conflicts). Even and odd nibbles are
+// masked into the bytes of two words as 4 m + sh (sh4 = sh in every byte); a
+// byte permute then merges one such byte with the upper bytes of tb, so every
+// lookup address costs one instruction.
+__device__ __forceinline__ uint32_t col_shift4(int c) { return (uint32_t)(c & 1) * 0x40404040u; }
+__device__ __forceinline__ void plane_entries(uint32_t tb, uint32_t sh4, uint32_t lo, uint32_t hi, float (&v)[16]) {
     const uint32_t M = 0x3C3C3C3Cu;
-    const uint32_t le = (lo << 2) & M, lo_ = (lo >> 2) & M, he = (hi << 2) & M, ho = (hi >> 2) & M;
+    const uint32_t le = ((lo << 2) & M) | sh4, lo_ = ((lo >> 2) & M) | sh4;
+    const uint32_t he = ((hi << 2) & M) | sh4, ho = ((hi >> 2) & M) | sh4;
     v[0] = lds_f32<0>(__byte_perm(le, tb, 0x7650));
     v[1] = lds_f32<64>(__byte_perm(lo_, tb, 0x7650));
     v[2] = lds_f32<128>(__byte_perm(le, tb, 0x7651));
@@ -389,7 +395,7 @@ __device__ void build_tables(Tables& T, const LayoutView& L, const uint16_t* __r
         const int c = pj >> 4, jn = pj & 15;
         const float4 xv = *reinterpret_cast<const float4*>(&T.xs[(c * 4 + (jn >> 2)) * XQ + 4 * (jn & 3)]);
         const float t3 = xv.x + xv.y, t12 = xv.w + xv.z;
-        float4* dst = reinterpret_cast<float4*>(T.lut + c * LUT_COL_BYTES + jn * 64);
+        float4* dst = reinterpret_cast<float4*>(T.lut + c * LUT_COL_BYTES + (c & 1) * 64 + jn * 64);
         dst[0] = make_float4(0.f, xv.x, xv.y, t3);
         dst[1] = make_float4(xv.z, xv.z + xv.x, xv.z + xv.y, xv.z + t3);
         dst[2] = make_float4(xv.w, xv.w + xv.x, xv.w + xv.y, xv.w + t3);
@@ -397,7 +403,7 @@ __device__ void build_tables(Tables& T, const LayoutView& L, const uint16_t* __r
     }
     consumer_sync();
     if (ct < cols) {
-        const float* t = reinterpret_cast<const float*>(T.lut + ct * LUT_COL_BYTES);
+        const float* t = reinterpret_cast<const float*>(T.lut + ct * LUT_COL_BYTES + (ct & 1) * 64);
         float v[16];
 #pragma unroll
         for (int jn = 0; jn < 16; ++jn) v[jn] = t[jn * 16 + 15];
@@ -488,8 +494,8 @@ __device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, in
                 const uint4 pl = lds_u32x4(pay + i * 16);
                 const uint32_t tb = lut0 + c * LUT_COL_BYTES;
                 float va[16], vb[16];
-                plane_entries(tb, pl.x, pl.y, va);
-                plane_entries(tb, pl.z, pl.w, vb);
+                plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
+                plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
                 const float2 sp = tree16x2(va, vb);
                 red_shared(ys + 4 * lds_u8(row + i),
                            half_bits(lds_u16(sc + 2 * i)) * (sp.x + 2.f * (sp.y - lds_f32r(xlut0 + 4 * c))));
@@ -510,8 +516,8 @@ __device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, in
                 const uint32_t rows2 = lds_u16(row + i);
                 const uint32_t sc2 = lds_u32(sc + 2 * i);
                 float va[16], vb[16];
-                plane_entries(lut0 + ca * LUT_COL_BYTES, v.x, v.y, va);
-                plane_entries(lut0 + cb * LUT_COL_BYTES, v.z, v.w, vb);
+                plane_entries(lut0 + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
+                plane_entries(lut0 + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
                 const float2 sp = tree16x2(va, vb);
                 if (two)
                     red_shared(ys + 4 * (rows2 >> 8), half_bits(sc2 >> 16) * (2.f * sp.y - lds_f32r(xlut0 + 4 * cb)));
