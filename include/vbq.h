@@ -163,6 +163,34 @@ vbq_status_t vbq_gemm_small(const vbq_layout* layout, const uint16_t* X, float* 
 vbq_status_t vbq_gemv_static(const vbq_layout* layout, const uint16_t* x, float* y,
                              void* stream);
 
+/*
+ * vbq_device_status — report (and clear) a bounded wait that gave up.
+ * (The paper has no counterpart; this is the library's failure report.)
+ *
+ * Every wait inside the product kernels (a copy landing in shared memory, a
+ * hand-over between warps, another block's split-K flag) is bounded to about
+ * one second. A wait that runs out records VBQ_ERR_TIMEOUT in a device word,
+ * lets its block finish without further writes to y and without leaving
+ * copies in flight, so the CUDA context stays usable; the affected y is
+ * undefined. This call synchronises `stream`, then reads and clears the word.
+ *
+ *   Returns VBQ_OK, VBQ_ERR_TIMEOUT (some product since the last call gave
+ *   up), or VBQ_ERR_CUDA.
+ */
+vbq_status_t vbq_device_status(void* stream);
+
+/*
+ * vbq_selftest_timeout — exercise the bounded-wait path on the device.
+ * (The paper has no counterpart; this is a test of vbq_device_status.)
+ *
+ * Launches one block whose thread 0 waits on a shared-memory barrier that
+ * nothing completes, with the wait bounded to limit_us microseconds
+ * (1..1000000, else VBQ_ERR_ARG). Afterwards vbq_device_status reports
+ * VBQ_ERR_TIMEOUT. Nothing faults and nothing hangs: the block returns when
+ * its limit runs out.
+ */
+vbq_status_t vbq_selftest_timeout(int limit_us, void* stream);
+
 /* vbq_free — release a layout and its device memory (NULL is accepted). */
 vbq_status_t vbq_free(vbq_layout* layout);
 

@@ -302,6 +302,21 @@ vbq_status_t vbq_gemv_static(const vbq_layout* L, const uint16_t* x, float* y, v
     return VBQ_OK;
 }
 
+vbq_status_t vbq_device_status(void* stream) {
+    g_err[0] = 0;
+    uint32_t word = 0;
+    VBQ_CUDA(vbq::read_device_status(&word, static_cast<cudaStream_t>(stream)));
+    if (word) return fail(VBQ_ERR_TIMEOUT, "a bounded device wait gave up (status word 0x%x)", word);
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_selftest_timeout(int limit_us, void* stream) {
+    g_err[0] = 0;
+    if (limit_us < 1 || limit_us > 1000000) return fail(VBQ_ERR_ARG, "limit_us must be in 1..1000000, got %d", limit_us);
+    VBQ_CUDA(vbq::launch_selftest_timeout(1000ull * (unsigned long long)limit_us, static_cast<cudaStream_t>(stream)));
+    return VBQ_OK;
+}
+
 vbq_status_t vbq_free(vbq_layout* L) {
     if (!L) return VBQ_OK;
     cudaError_t e = L->base ? cudaFree(L->base) : cudaSuccess;

@@ -827,6 +827,44 @@ cudaError_t launch_gemv1_static(const LayoutView& L, const uint16_t* x, float* y
     return launch_gemv1(Ls, x, y, s);
 }
 
+// ---------------------------------------------------------------------------
+// Failure report of the bounded waits, and its self-test.
+// ---------------------------------------------------------------------------
+
+namespace {
+
+// One block: thread 0 waits on a barrier that nothing completes, bounded to
+// limit_ns, and records the timeout the way the product kernels do.
+__global__ void selftest_timeout_kernel(unsigned long long limit_ns) {
+    __shared__ __align__(8) unsigned long long bar;
+    const uint32_t b = smem_u32(&bar);
+    if (threadIdx.x == 0) {
+        mbar_init(b, 1);
+        fence_barrier_init();
+        const unsigned long long t0 = global_ns();
+        bool done = false;
+        while (!(done = mbar_try_wait_sleep(b, 0))) {
+            if (global_ns() - t0 > limit_ns) break;
+        }
+        if (!done) atomicOr(&g_device_status, VBQ_DEVICE_TIMEOUT);
+    }
+}
+
+}  // namespace
+
+cudaError_t read_device_status(uint32_t* status, cudaStream_t s) {
+    cudaError_t e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return e;
+    if ((e = cudaMemcpyFromSymbol(status, g_device_status, sizeof(uint32_t))) != cudaSuccess) return e;
+    const uint32_t zero = 0;
+    return cudaMemcpyToSymbol(g_device_status, &zero, sizeof(uint32_t));
+}
+
+cudaError_t launch_selftest_timeout(unsigned long long limit_ns, cudaStream_t s) {
+    selftest_timeout_kernel<<<1, 32, 0, s>>>(limit_ns);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
     if (B <= 1) return launch_gemv1(L, X, Y, s);
     if (B <= 2) return launch_nb<2>(L, X, Y, B, s);

@@ -35,6 +35,8 @@ SIGNATURES = {
     "vbq_gemv": (_I, [_P, _P, _P, _P]),
     "vbq_gemm_small": (_I, [_P, _P, _P, _I, _P]),
     "vbq_gemv_static": (_I, [_P, _P, _P, _P]),
+    "vbq_device_status": (_I, [_P]),
+    "vbq_selftest_timeout": (_I, [_I, _P]),
     "vbq_free": (_I, [_P]),
     "vbq_status_string": (ctypes.c_char_p, [_I]),
     "vbq_last_error": (ctypes.c_char_p, []),
@@ -166,6 +168,17 @@ def vbq_gemm_small(layout: Layout, X, Y, B: Optional[int] = None, stream=None) -
     if B is None:
         B = int(X.shape[0])
     _check(load().vbq_gemm_small(layout, _ptr(X), _ptr(Y), int(B), _stream(stream, X, Y)))
+
+
+def vbq_device_status(stream=None) -> None:
+    """Synchronise the stream; raise VbqError(VBQ_ERR_TIMEOUT) if a bounded
+    device wait gave up since the last call (the record is cleared)."""
+    _check(load().vbq_device_status(_stream(stream)))
+
+
+def vbq_selftest_timeout(limit_us: int, stream=None) -> None:
+    """Launch the one-block kernel whose wait runs out after limit_us."""
+    _check(load().vbq_selftest_timeout(int(limit_us), _stream(stream)))
 
 
 def vbq_free(layout: Layout) -> None:

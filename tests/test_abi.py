@@ -85,3 +85,12 @@ def test_binding_raises_typed_errors(lib):
 def test_missing_library_fails_loudly(tmp_path):
     with pytest.raises(RuntimeError, match="not built"):
         binding.load(str(tmp_path / "libvbq.so"))
+
+
+def test_selftest_timeout_rejects_bad_limits():
+    import paper_2607_02893_gb300 as vbq
+    vbq.load()
+    for bad in (0, -5, 1000001):
+        with pytest.raises(vbq.VbqError) as e:
+            vbq.vbq_selftest_timeout(bad, stream=0)
+        assert e.value.name == "VBQ_ERR_ARG"
