@@ -273,10 +273,7 @@ static vbq_status_t run_product(const vbq_layout* L, const uint16_t* X, float* Y
     if (!X || !Y) return fail(VBQ_ERR_ARG, "x and y must be non-NULL");
     if (B < 1 || B > vbq::MAX_BATCH) return fail(VBQ_ERR_UNSUPPORTED, "batch %d outside 1..16", B);
     if (!aligned16(X) || !aligned16(Y)) return fail(VBQ_ERR_ALIGN, "x and y must be 16-byte aligned");
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (B > 1 && L->view.S > 1)       // the batched kernel adds slab partials into a zeroed Y
-        VBQ_CUDA(cudaMemsetAsync(Y, 0, (size_t)B * (size_t)L->view.N * sizeof(float), s));
-    VBQ_CUDA(vbq::launch_gemv(L->view, X, Y, B, s));
+    VBQ_CUDA(vbq::launch_gemv(L->view, X, Y, B, static_cast<cudaStream_t>(stream)));
     return VBQ_OK;
 }
 

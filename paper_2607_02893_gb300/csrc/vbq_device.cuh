@@ -1,0 +1,215 @@
+// vbq_device.cuh — device helpers shared by the product kernels of this
+// library: shared-memory access by 32-bit shared address, reductions, the
+// bounded mbarrier waits and TMA bulk copies of unit blobs, the split-K flag
+// wait, and the column lookup of a unit's items.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda_fp16.h>
+
+#include "vbq_common.cuh"
+
+namespace vbq {
+namespace {
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+template <int OFF>
+__device__ __forceinline__ float lds_f32(uint32_t addr) {
+    float v;
+    asm("ld.shared.f32 %0, [%1+%2];" : "=f"(v) : "r"(addr), "n"(OFF));
+    return v;
+}
+
+__device__ __forceinline__ float4 lds_f32x4(uint32_t addr) {
+    float4 v;
+    asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint32_t lds_u8(uint32_t addr) {
+    uint32_t v;
+    asm("ld.shared.u8 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ uint32_t lds_u16(uint32_t addr) {
+    uint32_t v;
+    asm("ld.shared.u16 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ float lds_f32r(uint32_t addr) {
+    float v;
+    asm("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ float2 lds_f32x2(uint32_t addr) {
+    float2 v;
+    asm("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint4 lds_u32x4(uint32_t addr) {
+    uint4 v;
+    asm("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint2 lds_u32x2(uint32_t addr) {
+    uint2 v;
+    asm("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint32_t lds_u32(uint32_t addr) {
+    uint32_t v;
+    asm("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ float2 f2(float a, float b) { return make_float2(a, b); }
+
+// y += v on a shared-memory float (32-bit shared address) / a global float.
+__device__ __forceinline__ void red_shared(uint32_t addr, float v) {
+    asm volatile("red.shared.add.f32 [%0], %1;" :: "r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void red_global(float* p, float v) {
+    asm volatile("red.global.add.f32 [%0], %1;" :: "l"(p), "f"(v) : "memory");
+}
+
+__device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) {
+    return *reinterpret_cast<const volatile uint32_t*>(p);
+}
+__device__ __forceinline__ void st_volatile(uint32_t* p, uint32_t v) {
+    *reinterpret_cast<volatile uint32_t*>(p) = v;
+}
+
+__device__ __forceinline__ float half_bits(uint32_t bits) { return __half2float(__ushort_as_half((uint16_t)bits)); }
+
+// ---------------------------------------------------------------------------
+// Unit blobs arrive by TMA bulk copy; roles hand stages over through
+// mbarriers. Every wait is bounded: after about a second (or as soon as another
+// role has given up) the waiting role records VBQ_DEVICE_TIMEOUT in
+// g_device_status, raises the block's abort flag and skips the rest of its
+// work; the copier lets every copy it started land before the block exits.
+// ---------------------------------------------------------------------------
+
+__device__ uint32_t g_device_status;     // one word per translation unit (internal linkage)
+constexpr uint32_t VBQ_DEVICE_TIMEOUT = 1u;
+constexpr unsigned long long WAIT_LIMIT_NS = 1000000000ull;
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_barrier_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+    return ok != 0;
+}
+// try_wait that lets the hardware suspend the thread for up to `hint` ns while
+// the phase is incomplete (it resumes as soon as the phase completes), so a
+// waiting warp issues a handful of instructions per wait instead of spinning.
+constexpr uint32_t SUSPEND_HINT_NS = 20000;
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(ok) : "r"(bar), "r"(parity), "n"(SUSPEND_HINT_NS) : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ int lds_volatile(uint32_t addr) {
+    int v;
+    asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(bar) : "memory");
+}
+// Wait until the barrier's phase with this parity completes. False when the
+// wait ran out or the block's abort flag (shared address abort_addr) is up.
+// A role off the critical path passes nap_ns > 0 to sleep between polls.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t abort_addr, uint32_t nap_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait_sleep(bar, parity)) {
+        if (nap_ns) __nanosleep(nap_ns);
+        if (lds_volatile(abort_addr) || global_ns() - t0 > WAIT_LIMIT_NS) return false;
+    }
+    return true;
+}
+// mbar_wait by a whole warp, with one verdict for all lanes (the roles' code
+// after a wait uses full-warp shuffles and must not diverge on it).
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint32_t abort_addr, uint32_t nap_ns = 0) {
+    return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_addr, nap_ns));
+}
+// Plain bounded wait (no abort flag), for the copier's final drain.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait_sleep(bar, parity)) {
+        if (global_ns() - t0 > WAIT_LIMIT_NS) return false;
+    }
+    return true;
+}
+__device__ __forceinline__ void raise_abort(int* abort_flag) {
+    atomicOr(&g_device_status, VBQ_DEVICE_TIMEOUT);
+    *reinterpret_cast<volatile int*>(abort_flag) = 1;
+}
+// One thread: expect `bytes` on the barrier and start the bulk copy.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(bar), "r"(bytes) : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void issue_unit(const LayoutView& L, int u, uint32_t dst, uint32_t bar) {
+    const uint32_t o0 = L.blob_off[u], o1 = L.blob_off[u + 1];
+    bulk_load(dst, L.blobs + (int64_t)o0 * 16, (o1 - o0) * 16, bar);
+}
+
+// Columns of a unit's items without a per-item array: lane t holds cend[t]
+// of one width (0xFFFF past the unit's last column), and item i of that width
+// lies in column #{t : cend[t] <= i}. A warp finds the columns of a task's
+// first and last items by one ballot each; only a task across column ends
+// (cf < cl) walks the few ends in between.
+__device__ __forceinline__ int col_uniform(uint32_t ce, int i) {   // i the same on every lane
+    return __popc(__ballot_sync(0xffffffffu, ce <= (uint32_t)i));
+}
+__device__ __forceinline__ int col_within(uint32_t ce, int cf, int cl, int i) {   // cf, cl the same on every lane
+    int c = cf;
+    for (int t = cf; t < cl; ++t) c += __shfl_sync(0xffffffffu, ce, t) <= (uint32_t)i;
+    return c;
+}
+
+// Split-K: true once every row block this block adds a slab s > 0 into has
+// been zeroed in this call (flag == epoch), within the wait limit. One thread;
+// ends with an acquire fence.
+__device__ __forceinline__ bool split_k_flags_ready(const LayoutView& L, uint32_t epoch, int u_begin, int u_end,
+                                                    int s0, int rb0) {
+    bool seen = true;
+    const unsigned long long t0 = global_ns();
+    int s2 = s0, rb2 = rb0;
+    for (int u = u_begin; u < u_end && seen; ++u) {
+        if (s2 > 0) {
+            while (!(seen = ld_volatile(L.ctl + 2 + rb2) == epoch))
+                if (global_ns() - t0 > WAIT_LIMIT_NS) break;
+        }
+        if (++rb2 == L.nrb) { rb2 = 0; ++s2; }
+    }
+    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+    return seen;
+}
+
+}  // namespace
+}  // namespace vbq

@@ -1,0 +1,465 @@
+// vbq_gemm.cu — batched product Y = X W^T for 2..16 activation rows (§6's
+// fused dequantise-and-multiply, several tokens at once) on the tensor cores.
+//
+// With B activation rows every decoded weight is used B times, so the product
+// is a dense contraction over dequantised tiles: here mma.sync m16n8k16 with
+// fp16 operands and fp32 accumulators. The operands are arranged so that the
+// packed bits go into B fragments with masks and byte permutes only:
+//
+//   A (16 x 16 per k-step) = activations: row b = batch row b (rows >= B are
+//       zero), pre-scaled per (batch row, group column) by 2^(24 - E), E set
+//       from the largest |x| of that column so every value stays in fp16
+//       range; built once per slab into shared memory, one fragment set per
+//       column and lane.
+//   B (16 x 8) = eight items (groups) of one width and one column: lane (g, t)
+//       holds item g's weights 16t + rho (low half) and 16t + 8 + rho (high
+//       half) of register rho. Any fixed assignment of the 64 weights of a
+//       group to the MMA's k positions gives the same sum, as long as A uses
+//       the same one; this one lets every width expand with one or two
+//       instructions per register into exact fp16 denormals u * 2^-24.
+//       One more packed fp16 subtraction (a fused 2u - 1 for one bit) turns
+//       u * 2^-24 into L(u) * 2^-24, exactly (every value is an integer times
+//       the smallest fp16 denormal, and fp16 arithmetic keeps denormals).
+//   D (16 x 8) = batch row x item: sum over the group of L(u) * x * 2^-E.
+//       Every product is exact, so a group whose codes all sit at the zero
+//       level gives exactly 0.
+//
+// The epilogue scales D by the item's FP16 scale and 2^E and adds it to the
+// stage's row partials of that batch row. The kernel around it is the batch-1
+// pipeline: one persistent block per SM, a copier warp streaming unit blobs by
+// TMA bulk copies into shared-memory stages and writing row partials to Y,
+// consumer warps in teams, two mbarriers per stage, split-K y zeroing by
+// epoch-tagged flags (see vbq_gemv.cu).
+#include <cstddef>
+
+#include "vbq_kernels.h"
+#include "vbq_device.cuh"
+
+namespace vbq {
+namespace {
+
+constexpr int NCWB = 16;                 // consumer warps
+constexpr int NCTB = 32 * NCWB;
+constexpr int GB_THREADS = 32 * (NCWB + 1);
+constexpr int NSTAGE_B = 3;              // blob stages in flight per SM
+constexpr int STAGE_BYTES_B = MAX_BLOB_BYTES;
+static_assert(STAGE_BYTES_B % 256 == 0, "stage alignment");
+
+// Shared-memory tables of the batched kernel; NB = 8 or 16 A rows.
+template <int NB>
+struct __align__(16) TablesB {
+    uint32_t afr[MAX_C][32][NB];         // A fragments (fp16x2) per column and lane: NB/4 per k-step
+    float e2[MAX_C][16];                 // per column and batch row: 2^E (0 for absent rows)
+    float ys[NSTAGE_B][NB][RB];          // row partials of each stage, per batch row
+    unsigned long long full[NSTAGE_B];   // blob landed
+    unsigned long long empty[NSTAGE_B];  // the unit's team is done
+    int abort;
+};
+
+template <int NB>
+constexpr size_t gemmb_smem() { return 256 + (size_t)NSTAGE_B * STAGE_BYTES_B + sizeof(TablesB<NB>); }
+static_assert(gemmb_smem<16>() <= 227 * 1024, "one block per SM");
+
+__device__ __forceinline__ void consumer_sync_b() {
+    asm volatile("bar.sync 1, %0;" :: "n"(NCTB) : "memory");
+}
+
+__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ float bf16_bits(uint32_t b) { return __uint_as_float(b << 16); }
+
+// Per slab: E and the A fragments of every column.
+// Consumer threads only (ct = 0 .. NCTB-1); starts and ends with a consumer barrier.
+template <int NB>
+__device__ void build_tables_b(TablesB<NB>& T, const LayoutView& L, const uint16_t* __restrict__ X, int B, int s,
+                               int ct) {
+    const int cols = min(L.C, L.G - s * L.C);
+    const int64_t k0 = (int64_t)s * L.C * GROUP;
+    const int lane = ct & 31, cwarp = ct >> 5;
+    consumer_sync_b();                   // nobody still reads the old fragments
+    // one warp per (batch row, column): max |x| over the column's 64 values
+    for (int p = cwarp; p < 16 * cols; p += NCWB) {
+        const int b = p / cols, c = p - b * cols;
+        float m = 0.f;
+        if (b < B) {
+            const uint32_t two = __ldg(reinterpret_cast<const uint32_t*>(X + (int64_t)b * L.K + k0 + c * GROUP) + lane);
+            m = fmaxf(fabsf(__uint_as_float(two << 16)), fabsf(__uint_as_float(two & 0xFFFF0000u)));
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        if (lane == 0) {
+            // |x| < 2^(ex+1) with ex the exponent of m: x * 2^(24 - E) < 2^14 for E = ex + 11
+            const int ex = m > 0.f ? (int)((__float_as_uint(m) >> 23) & 0xFF) - 127 : -11;
+            const int E = ex + 11;
+            T.e2[c][b] = b < B ? ldexpf(1.f, E) : 0.f;
+        }
+    }
+    consumer_sync_b();
+    // A fragments: register r of lane (g, t) for column c. NB = 16: k-step
+    // s = r / 4, q = r % 4 -> (row g + 8 (q & 1), half h = q >> 1); NB = 8:
+    // s = r / 2, h = r % 2, row g. Register pair (rho = 2s + h): weights
+    // 16t + rho (low) and 16t + 8 + rho (high) of the column.
+    for (int p = ct; p < cols * 32 * NB; p += NCTB) {
+        const int r = p % NB, l = (p / NB) & 31, c = p / (NB * 32);
+        const int g = l >> 2, t = l & 3;
+        int s2, h, row;
+        if (NB == 16) { s2 = r >> 2; h = (r >> 1) & 1; row = g + 8 * (r & 1); }
+        else { s2 = r >> 1; h = r & 1; row = g; }
+        const int rho = 2 * s2 + h;
+        uint32_t v = 0;
+        if (row < B) {
+            const float f = ldexpf(1.f, 24) / T.e2[c][row];
+            const uint16_t* xr = X + (int64_t)row * L.K + k0 + c * GROUP;
+            const float lo = bf16_bits(__ldg(xr + 16 * t + rho)) * f;
+            const float hi = bf16_bits(__ldg(xr + 16 * t + 8 + rho)) * f;
+            const __half2 hv = __floats2half2_rn(lo, hi);
+            v = *reinterpret_cast<const uint32_t*>(&hv);
+        }
+        T.afr[c][l][r] = v;
+    }
+    consumer_sync_b();
+}
+
+// B fragments (8 registers, u * 2^-24 per half) of lane t's 16 weights of one item.
+__device__ __forceinline__ void bfrag_1(uint2 w, int t, uint32_t (&b)[8]) {
+    const uint32_t word = t < 2 ? w.x : w.y;
+    const uint32_t lo = 2u * (t & 1), sel = lo | (lo << 4) | ((lo + 1) << 8) | ((lo + 1) << 12);
+    const uint32_t W = __byte_perm(word, word, sel);          // field bits 0-7 at 0-7, 8-15 at 16-23
+#pragma unroll
+    for (int r = 0; r < 8; ++r) b[r] = (W >> r) & 0x00010001u;
+}
+__device__ __forceinline__ void bfrag_2(uint4 w, int t, uint32_t (&b)[8]) {
+    const uint32_t lo = 2u * (t & 1), sel = lo | (lo << 4) | ((lo + 1) << 8) | ((lo + 1) << 12);
+    const uint32_t W0 = __byte_perm(t < 2 ? w.x : w.y, t < 2 ? w.x : w.y, sel);   // bit plane 0
+    const uint32_t W1 = __byte_perm(t < 2 ? w.z : w.w, t < 2 ? w.z : w.w, sel);   // bit plane 1
+    b[0] = (W0 & 0x00010001u) | ((W1 << 1) & 0x00020002u);
+#pragma unroll
+    for (int r = 1; r < 8; ++r) b[r] = ((W0 >> r) & 0x00010001u) | ((W1 >> (r - 1)) & 0x00020002u);
+}
+__device__ __forceinline__ void bfrag_4(uint2 w, uint32_t (&b)[8]) {   // w = words 2t, 2t+1 of the item
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const uint32_t V = __byte_perm(w.x, w.y, q | (q << 4) | ((4 + q) << 8) | ((4 + q) << 12));
+        b[2 * q] = V & 0x000F000Fu;
+        b[2 * q + 1] = (V >> 4) & 0x000F000Fu;
+    }
+}
+__device__ __forceinline__ void bfrag_8(uint4 w, uint32_t (&b)[8]) {   // w = words 4t .. 4t+3 of the item
+    const uint32_t words[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+        const uint32_t q = r & 3;
+        b[r] = __byte_perm(words[r >> 2], words[2 + (r >> 2)], q | (q << 4) | ((4 + q) << 8) | ((4 + q) << 12)) &
+               0x00FF00FFu;
+    }
+}
+
+__device__ __forceinline__ int pick4(const int (&v)[4], int w) {   // v[w] for a warp-uniform w
+    return w == 0 ? v[0] : w == 1 ? v[1] : w == 2 ? v[2] : v[3];
+}
+
+// u * 2^-24 -> L(u) * 2^-24 in both halves: 2u - 1 (z = 0: one bit) or u - z.
+__device__ __forceinline__ void to_levels(uint32_t (&b)[8], int w) {
+    if (w == 0) {
+        const __half2 two = __floats2half2_rn(2.f, 2.f), m1 = __halves2half2(__ushort_as_half(0x8001u), __ushort_as_half(0x8001u));
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+            const __half2 v = __hfma2(*reinterpret_cast<const __half2*>(&b[r]), two, m1);
+            b[r] = *reinterpret_cast<const uint32_t*>(&v);
+        }
+    } else {
+        const unsigned short zb = w == 1 ? 2 : w == 2 ? 8 : 128;   // z * 2^-24 as fp16 bits (a denormal)
+        const __half2 z = __halves2half2(__ushort_as_half(zb), __ushort_as_half(zb));
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+            const __half2 v = __hsub2(*reinterpret_cast<const __half2*>(&b[r]), z);
+            b[r] = *reinterpret_cast<const uint32_t*>(&v);
+        }
+    }
+}
+
+// One consumer warp's share of a unit: tiles of 8 items of one (column, width)
+// bucket, in (column, width) order; warp wt of a team of tw warps takes a
+// contiguous run of them, so its A fragments change only with the column.
+template <int NB>
+__device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sblob, int C, int cols, uint32_t ys,
+                                               int B, int wt, int tw, int lane) {
+    const int g = lane >> 2, t = lane & 3;
+    const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
+    const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
+    // lane c (< cols) holds, per width, its bucket's first item, end and tile count
+    int start[4], end[4], ntile[4], nt_col = 0;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        const int e = lane < cols ? (int)lds_u16(cc + 2 * (w * C + lane)) : 0;
+        int a = __shfl_up_sync(0xffffffffu, e, 1);
+        if (lane == 0) a = 0;
+        start[w] = a;
+        end[w] = e;
+        ntile[w] = lane < cols ? (e - a + 7) >> 3 : 0;
+        nt_col += ntile[w];
+    }
+    int incl = nt_col;                   // tiles of columns 0..lane
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+    }
+    const int total = __shfl_sync(0xffffffffu, incl, 31);
+    const int ta = (total * wt) / tw, tb = (total * (wt + 1)) / tw;
+    if (ta >= tb) return;
+    // locate tile ta: its column c, width w and tile k within the bucket
+    int c = __popc(__ballot_sync(0xffffffffu, incl <= ta));
+    int k = ta - (__shfl_sync(0xffffffffu, incl, c) - __shfl_sync(0xffffffffu, nt_col, c));
+    int w = 0, ntw = __shfl_sync(0xffffffffu, ntile[0], c);
+    while (k >= ntw) { k -= ntw; ++w; ntw = __shfl_sync(0xffffffffu, pick4(ntile, w), c); }
+    int bs = __shfl_sync(0xffffffffu, pick4(start, w), c), be = __shfl_sync(0xffffffffu, pick4(end, w), c);
+
+    int cur_c = -1;
+    uint32_t a[NB];
+    float e2g = 0.f, e2g8 = 0.f;
+    for (int tile = ta; tile < tb; ++tile) {
+        if (c != cur_c) {                // A fragments, zero-level sums and 2^E of the new column
+            const uint32_t* src = &T.afr[c][lane][0];
+#pragma unroll
+            for (int r = 0; r < NB; r += 4) {
+                const uint4 v = *reinterpret_cast<const uint4*>(src + r);
+                a[r] = v.x; a[r + 1] = v.y; a[r + 2] = v.z; a[r + 3] = v.w;
+            }
+            e2g = T.e2[c][g]; e2g8 = T.e2[c][g + 8];
+            cur_c = c;
+        }
+        const int i0 = bs + 8 * k, nv = min(8, be - i0);           // this tile's items: i0 .. i0 + nv - 1
+        const int ig = i0 + min(g, nv - 1);                        // lane's item (a valid one past the end)
+        uint32_t b[8];
+        uint32_t sc_base, row_base;
+        if (w == 0) {
+            bfrag_1(lds_u32x2(sblob + (h0.z & 0xFFFF) * 16 + ig * 8), t, b);
+            sc_base = sblob + (h1.x & 0xFFFF) * 16; row_base = sblob + (h1.z & 0xFFFF) * 16;
+        } else if (w == 1) {
+            bfrag_2(lds_u32x4(sblob + (h0.z >> 16) * 16 + ig * 16), t, b);
+            sc_base = sblob + (h1.x >> 16) * 16; row_base = sblob + (h1.z >> 16) * 16;
+        } else if (w == 2) {
+            bfrag_4(lds_u32x2(sblob + (h0.w & 0xFFFF) * 16 + ig * 32 + 8 * t), b);
+            sc_base = sblob + (h1.y & 0xFFFF) * 16; row_base = sblob + (h1.w & 0xFFFF) * 16;
+        } else {
+            bfrag_8(lds_u32x4(sblob + (h0.w >> 16) * 16 + ig * 64 + 16 * t), b);
+            sc_base = sblob + (h1.y >> 16) * 16; row_base = sblob + (h1.w >> 16) * 16;
+        }
+        to_levels(b, w);
+        float d[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int s2 = 0; s2 < 4; ++s2) {
+            uint32_t af[4];
+            if (NB == 16) { af[0] = a[4 * s2]; af[1] = a[4 * s2 + 1]; af[2] = a[4 * s2 + 2]; af[3] = a[4 * s2 + 3]; }
+            else { af[0] = a[2 * s2]; af[1] = 0u; af[2] = a[(2 * s2 + 1) % NB]; af[3] = 0u; }
+            mma16816(d, af, b[2 * s2], b[2 * s2 + 1]);
+        }
+        // items 2t and 2t+1 of the tile: scale, add to the row partials of batch rows g and g + 8
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int n = 2 * t + e;
+            if (n < nv) {
+                const int i = i0 + n;
+                const float sc = half_bits(lds_u16(sc_base + 2 * i));
+                const int r = lds_u8(row_base + i);
+                if (g < B) red_shared(ys + 4 * (g * RB + r), d[e] * (sc * e2g));
+                if (NB == 16 && g + 8 < B) red_shared(ys + 4 * ((g + 8) * RB + r), d[2 + e] * (sc * e2g8));
+            }
+        }
+        // next tile: the next one of this bucket, else the next non-empty bucket in (column, width) order
+        if (++k == ntw && tile + 1 < tb) {
+            k = 0;
+            do {
+                if (++w == 4) { w = 0; ++c; }
+                ntw = __shfl_sync(0xffffffffu, pick4(ntile, w), c);
+            } while (ntw == 0);
+            bs = __shfl_sync(0xffffffffu, pick4(start, w), c);
+            be = __shfl_sync(0xffffffffu, pick4(end, w), c);
+        }
+    }
+}
+
+template <int NB>
+__global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, const uint16_t* __restrict__ X,
+                                                              float* __restrict__ Y, int B) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    unsigned char* base = smem_raw + ((256u - (smem_u32(smem_raw) & 255u)) & 255u);
+    TablesB<NB>& T = *reinterpret_cast<TablesB<NB>*>(base + (size_t)NSTAGE_B * STAGE_BYTES_B);
+    const uint32_t stage0 = smem_u32(base);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int P = gridDim.x, p = blockIdx.x;
+    const int per = L.units / P, extra = L.units - per * P;
+    const int u_begin = p * per + min(p, extra), u_end = u_begin + per + (p < extra ? 1 : 0);
+    const int n_units = u_end - u_begin;
+    if (n_units <= 0) return;
+    const int s0 = u_begin / L.nrb, rb0 = u_begin - s0 * L.nrb;
+    // One team: every consumer warp takes every unit, so each waits every phase
+    // of every stage in order. (Several teams over NSTAGE_B = 3 stages would let a
+    // team skip phases of a stage that other teams' units use; a parity wait can
+    // then match an older completed phase. The batch-1 kernel avoids that by
+    // giving each team stages of its own.)
+    const int teams = 1, tw = NCWB;
+
+    const uint32_t full0 = smem_u32(&T.full[0]), empty0 = smem_u32(&T.empty[0]);
+    const uint32_t abort_addr = smem_u32(&T.abort);
+    if (tid == 0) {
+        for (int i = 0; i < NSTAGE_B; ++i) {
+            mbar_init(full0 + 8 * i, 1);
+            mbar_init(empty0 + 8 * i, tw);
+        }
+        T.abort = 0;
+        fence_barrier_init();
+    }
+    for (int i = tid; i < NSTAGE_B * NB * RB; i += GB_THREADS) (&T.ys[0][0][0])[i] = 0.f;
+    __syncthreads();
+    if (tid == 0) {
+        const int first = n_units < NSTAGE_B ? n_units : NSTAGE_B;
+        for (int j = 0; j < first; ++j) issue_unit(L, u_begin + j, stage0 + j * STAGE_BYTES_B, full0 + 8 * j);
+    }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+
+    if (warp == 0) {
+        // ---- copier: split-K zeroing, then per unit: rows out, next copy in ----
+        uint32_t epoch = 0;
+        if (L.S > 1) {
+            epoch = ld_volatile(L.ctl) + 1u;
+            const int z_end = min(u_end, L.nrb);
+            for (int u = u_begin; u < z_end; ++u) {
+                const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
+                for (int q = lane; q < B * rows; q += 32) {
+                    const int b = q / rows, r = q - b * rows;
+                    Y[(int64_t)b * L.N + (int64_t)u * RB + r] = 0.f;
+                }
+            }
+            __syncwarp();
+            if (lane == 0 && u_begin < z_end) {
+                __threadfence();
+                for (int u = u_begin; u < z_end; ++u) st_volatile(L.ctl + 2 + u, epoch);
+            }
+        }
+        bool dead = false, checked = L.S == 1;
+        int st = 0, rbw = rb0, issued = n_units < NSTAGE_B ? n_units : NSTAGE_B;
+        uint32_t par = 0;
+        for (int j = 0; j < n_units; ++j) {
+            if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 256)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
+            if (!dead && !checked) {
+                int ok = 1;
+                if (lane == 0) ok = split_k_flags_ready(L, epoch, u_begin, u_end, s0, rb0);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                checked = true;
+                if (!ok) { dead = true; if (lane == 0) raise_abort(&T.abort); }
+            }
+            if (!dead) {
+                const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
+                for (int b = 0; b < B; ++b) {
+                    float* ys = T.ys[st][b];
+                    float* yr = Y + (int64_t)b * L.N + (int64_t)rbw * RB;
+#pragma unroll
+                    for (int q = 0; q < RB / 32; ++q) {
+                        const int r = lane + 32 * q;
+                        const float v = ys[r];
+                        ys[r] = 0.f;
+                        if (r < rows) {
+                            if (L.S == 1) yr[r] = v;
+                            else red_global(yr + r, v);
+                        }
+                    }
+                }
+                __syncwarp();
+                if (j + NSTAGE_B < n_units) {
+                    if (lane == 0) issue_unit(L, u_begin + j + NSTAGE_B, stage0 + st * STAGE_BYTES_B, full0 + 8 * st);
+                    ++issued;
+                }
+            }
+            if (++st == NSTAGE_B) { st = 0; par ^= 1; }
+            if (++rbw == L.nrb) rbw = 0;
+        }
+        if (dead && lane == 0) {
+            for (int i = 0; i < NSTAGE_B && i < issued; ++i) {
+                const int jl = i + ((issued - 1 - i) / NSTAGE_B) * NSTAGE_B;
+                mbar_wait_bounded(full0 + 8 * i, (uint32_t)((jl / NSTAGE_B) & 1));
+            }
+        }
+        if (L.S > 1 && lane == 0) {
+            __threadfence();
+            if (atomicAdd(L.ctl + 1, 1u) == gridDim.x - 1) {
+                st_volatile(L.ctl + 1, 0u);
+                st_volatile(L.ctl, epoch);
+            }
+        }
+    } else {
+        // ---- consumers: team `team` takes units j = team, team + teams, ... ----
+        const int cw = warp - 1, ct = tid - 32, team = cw / tw, wt = cw - team * tw;
+        const int s_last = (u_end - 1) / L.nrb;
+        bool dead = false;
+        int cur = s0, rbj = rb0 + team, sj = s0;
+        while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
+        build_tables_b(T, L, X, B, s0, ct);
+        for (int j = team; j < n_units; j += teams) {
+            while (cur < sj) build_tables_b(T, L, X, B, ++cur, ct);
+            const int st = j % NSTAGE_B;
+            const uint32_t par = (uint32_t)(j / NSTAGE_B) & 1u;
+            if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
+            if (!dead) {
+                consume_unit_b<NB>(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
+                                   smem_u32(&T.ys[st][0][0]), B, wt, tw, lane);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty0 + 8 * st);
+            }
+            rbj += teams;
+            while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
+        }
+        while (cur < s_last) build_tables_b(T, L, X, B, ++cur, ct);
+    }
+}
+
+int g_sms_b = 0;
+
+template <int NB>
+cudaError_t launch_gemmb(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(gemmb_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)gemmb_smem<NB>());
+        if (e != cudaSuccess) return e;
+        int dev = 0;
+        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+        if ((e = cudaDeviceGetAttribute(&g_sms_b, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int grid = L.units < g_sms_b ? L.units : g_sms_b;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(GB_THREADS);
+    cfg.dynamicSmemBytes = gemmb_smem<NB>();
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, gemmb_kernel<NB>, L, X, Y, B);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_small(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
+    return B <= 8 ? launch_gemmb<8>(L, X, Y, B, s) : launch_gemmb<16>(L, X, Y, B, s);
+}
+
+cudaError_t read_device_status_gemm(uint32_t* status) {
+    cudaError_t e = cudaMemcpyFromSymbol(status, g_device_status, sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    const uint32_t zero = 0;
+    return cudaMemcpyToSymbol(g_device_status, &zero, sizeof(uint32_t));
+}
+
+}  // namespace vbq

@@ -36,24 +36,27 @@
 // shared-memory partial; a unit's rows then go to y directly (one slab per
 // row) or through atomics (several slabs).
 //
-// Batch 2..16 (gemm_kernel<NB>): one block per unit, one thread per group,
-// plain fp32 FMAs per code and per activation row.
+// Batch 2..16 runs on the tensor cores in vbq_gemm.cu.
 #include <cstddef>
 #include <mutex>
 
 #include "vbq_kernels.h"
+#include "vbq_device.cuh"
 
 namespace vbq {
 namespace {
 
-constexpr int THREADS = 256;             // batch 2..16 kernel
 constexpr int NCW = 16;                  // consumer warps of the batch-1 kernel
 constexpr int NCT = 32 * NCW;            // consumer threads
 constexpr int MAX_TEAMS = 4;             // consumer teams (1, 2 or 4 by units per block); unit j goes to team j % teams
 static_assert(NCW == 16 && MAX_TEAMS == 4, "teams of 16, 8 or 4 warps (powers of two)");
+// Unit j uses stage j % NSTAGE and goes to team j % teams; with NSTAGE a
+// multiple of every team count, each stage serves one team only, and that team
+// waits the stage's phases in order (a parity wait never skips a phase).
 constexpr int G1_THREADS = 32 * (NCW + 1);
 constexpr int NSTAGE = 4;                // blob stages in flight per SM
 static_assert((NSTAGE & (NSTAGE - 1)) == 0, "power-of-two stage count");
+static_assert(NSTAGE % 4 == 0, "every team count (1, 2, 4) divides the stage count");
 constexpr int XQ = 20;                   // floats per 16-code quarter of x (16 + 4 pad: quarters use other banks)
 constexpr int XH = 36;                   // floats per 32-code half of the pre-scaled x (32 + 4 pad)
 constexpr int LUT_COL_BYTES = 1280;      // 16 tables x 64 bytes (+64 for odd columns), columns on 256-byte boundaries
@@ -79,68 +82,6 @@ static_assert(MAX_C <= 32, "a warp holds a unit's column ends one per lane");
 
 constexpr size_t GEMV1_SMEM = 256 /* alignment slack */ + (size_t)NSTAGE * STAGE_BYTES + sizeof(Tables);
 static_assert(GEMV1_SMEM <= 227 * 1024, "one block per SM");
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-template <int OFF>
-__device__ __forceinline__ float lds_f32(uint32_t addr) {
-    float v;
-    asm("ld.shared.f32 %0, [%1+%2];" : "=f"(v) : "r"(addr), "n"(OFF));
-    return v;
-}
-
-__device__ __forceinline__ float4 lds_f32x4(uint32_t addr) {
-    float4 v;
-    asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
-                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
-    return v;
-}
-
-__device__ __forceinline__ uint32_t lds_u8(uint32_t addr) {
-    uint32_t v;
-    asm("ld.shared.u8 %0, [%1];" : "=r"(v) : "r"(addr));
-    return v;
-}
-__device__ __forceinline__ uint32_t lds_u16(uint32_t addr) {
-    uint32_t v;
-    asm("ld.shared.u16 %0, [%1];" : "=r"(v) : "r"(addr));
-    return v;
-}
-__device__ __forceinline__ float lds_f32r(uint32_t addr) {
-    float v;
-    asm("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
-    return v;
-}
-__device__ __forceinline__ float2 lds_f32x2(uint32_t addr) {
-    float2 v;
-    asm("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));
-    return v;
-}
-
-__device__ __forceinline__ uint4 lds_u32x4(uint32_t addr) {
-    uint4 v;
-    asm("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
-    return v;
-}
-
-__device__ __forceinline__ uint32_t lds_u32(uint32_t addr) {
-    uint32_t v;
-    asm("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
-    return v;
-}
-
-__device__ __forceinline__ float2 f2(float a, float b) { return make_float2(a, b); }
-
-// y += v on a shared-memory float (32-bit shared address) / a global float.
-__device__ __forceinline__ void red_shared(uint32_t addr, float v) {
-    asm volatile("red.shared.add.f32 [%0], %1;" :: "r"(addr), "f"(v) : "memory");
-}
-__device__ __forceinline__ void red_global(float* p, float v) {
-    asm volatile("red.global.add.f32 [%0], %1;" :: "l"(p), "f"(v) : "memory");
-}
 
 // The 16 table entries that a 64-bit bit plane (words lo, hi) selects from a
 // column's tables at tb (256-byte aligned): nibble p of the plane picks entry
@@ -237,139 +178,9 @@ __device__ __forceinline__ float dot8_quarter(uint4 v, uint32_t xa) {
     return (ca.x + ca.y) + (cb.x + cb.y);
 }
 
-__device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) {
-    return *reinterpret_cast<const volatile uint32_t*>(p);
-}
-__device__ __forceinline__ void st_volatile(uint32_t* p, uint32_t v) {
-    *reinterpret_cast<volatile uint32_t*>(p) = v;
-}
-
-__device__ __forceinline__ float half_bits(uint32_t bits) { return __half2float(__ushort_as_half((uint16_t)bits)); }
-
-// ---------------------------------------------------------------------------
-// Unit blobs arrive by TMA bulk copy; roles hand stages over through
-// mbarriers. Every wait is bounded: after about a second (or as soon as another
-// role has given up) the waiting role records VBQ_DEVICE_TIMEOUT in
-// g_device_status, raises the block's abort flag and skips the rest of its
-// work; the copier lets every copy it started land before the block exits.
-// ---------------------------------------------------------------------------
-
-__device__ uint32_t g_device_status;
-constexpr uint32_t VBQ_DEVICE_TIMEOUT = 1u;
-constexpr unsigned long long WAIT_LIMIT_NS = 1000000000ull;
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void fence_barrier_init() {
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-__device__ __forceinline__ unsigned long long global_ns() {
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
-                 : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
-    return ok != 0;
-}
-// try_wait that lets the hardware suspend the thread for up to `hint` ns while
-// the phase is incomplete (it resumes as soon as the phase completes), so a
-// waiting warp issues a handful of instructions per wait instead of spinning.
-constexpr uint32_t SUSPEND_HINT_NS = 20000;
-__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\tselp.u32 %0, 1, 0, p;\n\t}"
-                 : "=r"(ok) : "r"(bar), "r"(parity), "n"(SUSPEND_HINT_NS) : "memory");
-    return ok != 0;
-}
-__device__ __forceinline__ int lds_volatile(uint32_t addr) {
-    int v;
-    asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
-    return v;
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(bar) : "memory");
-}
-// Wait until the barrier's phase with this parity completes. False when the
-// wait ran out or the block's abort flag (shared address abort_addr) is up.
-// A role off the critical path passes nap_ns > 0 to sleep between polls.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t abort_addr, uint32_t nap_ns) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const unsigned long long t0 = global_ns();
-    while (!mbar_try_wait_sleep(bar, parity)) {
-        if (nap_ns) __nanosleep(nap_ns);
-        if (lds_volatile(abort_addr) || global_ns() - t0 > WAIT_LIMIT_NS) return false;
-    }
-    return true;
-}
-// mbar_wait by a whole warp, with one verdict for all lanes (the roles' code
-// after a wait uses full-warp shuffles and must not diverge on it).
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint32_t abort_addr, uint32_t nap_ns = 0) {
-    return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_addr, nap_ns));
-}
-// Plain bounded wait (no abort flag), for the copier's final drain.
-__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
-    const unsigned long long t0 = global_ns();
-    while (!mbar_try_wait_sleep(bar, parity)) {
-        if (global_ns() - t0 > WAIT_LIMIT_NS) return false;
-    }
-    return true;
-}
-__device__ __forceinline__ void raise_abort(int* abort_flag) {
-    atomicOr(&g_device_status, VBQ_DEVICE_TIMEOUT);
-    *reinterpret_cast<volatile int*>(abort_flag) = 1;
-}
-// One thread: expect `bytes` on the barrier and start the bulk copy.
-__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(bar), "r"(bytes) : "memory");
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-                 :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
-}
-
-__device__ __forceinline__ void issue_unit(const LayoutView& L, int u, uint32_t dst, uint32_t bar) {
-    const uint32_t o0 = L.blob_off[u], o1 = L.blob_off[u + 1];
-    bulk_load(dst, L.blobs + (int64_t)o0 * 16, (o1 - o0) * 16, bar);
-}
-
 // Consumer warps only (named barrier 1).
 __device__ __forceinline__ void consumer_sync() {
     asm volatile("bar.sync 1, %0;" :: "n"(NCT) : "memory");
-}
-
-// Columns of a unit's items without a per-item array: lane t holds cend[t]
-// of one width (0xFFFF past the unit's last column), and item i of that width
-// lies in column #{t : cend[t] <= i}. A warp finds the columns of a task's
-// first and last items by one ballot each; only a task across column ends
-// (cf < cl) walks the few ends in between.
-__device__ __forceinline__ int col_uniform(uint32_t ce, int i) {   // i the same on every lane
-    return __popc(__ballot_sync(0xffffffffu, ce <= (uint32_t)i));
-}
-__device__ __forceinline__ int col_within(uint32_t ce, int cf, int cl, int i) {   // cf, cl the same on every lane
-    int c = cf;
-    for (int t = cf; t < cl; ++t) c += __shfl_sync(0xffffffffu, ce, t) <= (uint32_t)i;
-    return c;
-}
-
-// Split-K: true once every row block this block adds a slab s > 0 into has
-// been zeroed in this call (flag == epoch), within the wait limit. One thread;
-// ends with an acquire fence.
-__device__ __forceinline__ bool split_k_flags_ready(const LayoutView& L, uint32_t epoch, int u_begin, int u_end,
-                                                    int s0, int rb0) {
-    bool seen = true;
-    const unsigned long long t0 = global_ns();
-    int s2 = s0, rb2 = rb0;
-    for (int u = u_begin; u < u_end && seen; ++u) {
-        if (s2 > 0) {
-            while (!(seen = ld_volatile(L.ctl + 2 + rb2) == epoch))
-                if (global_ns() - t0 > WAIT_LIMIT_NS) break;
-        }
-        if (++rb2 == L.nrb) { rb2 = 0; ++s2; }
-    }
-    asm volatile("fence.acq_rel.gpu;" ::: "memory");
-    return seen;
 }
 
 // Activations of slab s: x as fp32, the pre-scaled x of the 4-bit slots, the
@@ -673,93 +484,6 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     }
 }
 
-// ---------------------------------------------------------------------------
-// Batch 2..16: one block per unit, one thread per group.
-// ---------------------------------------------------------------------------
-
-template <int B, int NB>
-__device__ __forceinline__ void dot_item(const uint8_t* __restrict__ src, const float* __restrict__ xs,
-                                         int xstride, int nb, float* acc) {
-    uint32_t w[2 * B];
-    load_item<B>(src, w);
-#pragma unroll
-    for (int j = 0; j < GROUP; ++j) {
-        const float lv = (float)level_of<B>(item_code<B>(w, j));
-#pragma unroll
-        for (int q = 0; q < NB; ++q)
-            if (q < nb) acc[q] = fmaf(lv, xs[q * xstride + j], acc[q]);
-    }
-}
-
-template <int NB>
-__global__ void __launch_bounds__(THREADS) gemm_kernel(LayoutView L, const uint16_t* __restrict__ X,
-                                                       float* __restrict__ Y, int nb) {
-    extern __shared__ float4 smem_f4[];
-    float* xs = reinterpret_cast<float*>(smem_f4);                 // [NB][C*64]
-    __shared__ UnitHeader h;
-    __shared__ float ys[NB][RB];
-
-    const int u = blockIdx.x, rb = unit_rb(L, u), s = unit_slab(L, u);
-    const int rows = unit_rows(L, rb), cols = unit_cols(L, s);
-    const int xstride = L.C * GROUP;
-    const int64_t k0 = (int64_t)s * L.C * GROUP;
-    const uint8_t* blob = L.blobs + (int64_t)L.blob_off[u] * 16;
-
-    if (threadIdx.x == 0) h = *reinterpret_cast<const UnitHeader*>(blob);
-    for (int i = threadIdx.x; i < nb * cols * GROUP; i += blockDim.x) {
-        const int q = i / (cols * GROUP), k = i - q * cols * GROUP;
-        const uint32_t bits = X[(int64_t)q * L.K + k0 + k];
-        xs[q * xstride + k] = __uint_as_float(bits << 16);
-    }
-    for (int i = threadIdx.x; i < NB * RB; i += blockDim.x) (&ys[0][0])[i] = 0.f;
-    __syncthreads();
-    const uint16_t* cend = reinterpret_cast<const uint16_t*>(blob + h.cc16 * 16);
-    const int total = h.n[0] + h.n[1] + h.n[2] + h.n[3];
-    for (int i = threadIdx.x; i < total; i += blockDim.x) {
-        int w = 0, j = i;
-        while (w < 3 && j >= h.n[w]) { j -= h.n[w]; ++w; }
-        const int c = column_of(cend + w * L.C, cols, 0, j);
-        const int r = blob[h.row16[w] * 16 + j];
-        const float sf = __half2float(__ushort_as_half(reinterpret_cast<const uint16_t*>(blob + h.sc16[w] * 16)[j]));
-        const uint8_t* pay = blob + h.pay16[w] * 16;
-        float acc[NB];
-#pragma unroll
-        for (int q = 0; q < NB; ++q) acc[q] = 0.f;
-        const float* xc = xs + c * GROUP;
-        switch (w) {
-            case 0: dot_item<1, NB>(pay + j * 8, xc, xstride, nb, acc); break;
-            case 1: dot_item<2, NB>(pay + j * 16, xc, xstride, nb, acc); break;
-            case 2: dot_item<4, NB>(pay + j * 32, xc, xstride, nb, acc); break;
-            default: dot_item<8, NB>(pay + j * 64, xc, xstride, nb, acc); break;
-        }
-#pragma unroll
-        for (int q = 0; q < NB; ++q)
-            if (q < nb) atomicAdd(&ys[q][r], sf * acc[q]);
-    }
-    __syncthreads();
-    const bool direct = (L.S == 1);
-    for (int i = threadIdx.x; i < nb * rows; i += blockDim.x) {
-        const int q = i / rows, r = i - q * rows;
-        float* dst = Y + (int64_t)q * L.N + (int64_t)rb * RB + r;
-        if (direct) *dst = ys[q][r];
-        else atomicAdd(dst, ys[q][r]);
-    }
-}
-
-template <int NB>
-cudaError_t launch_nb(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
-    const size_t dyn = (size_t)NB * L.C * GROUP * sizeof(float);
-    static bool attr_set = false;           // the attribute is per function; set once per process
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)(NB * MAX_C * GROUP * sizeof(float)));
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
-    gemm_kernel<NB><<<L.units, THREADS, dyn, s>>>(L, X, Y, B);
-    return cudaGetLastError();
-}
-
 int g_sms = 0;
 
 cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s) {
@@ -855,9 +579,13 @@ __global__ void selftest_timeout_kernel(unsigned long long limit_ns) {
 cudaError_t read_device_status(uint32_t* status, cudaStream_t s) {
     cudaError_t e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return e;
-    if ((e = cudaMemcpyFromSymbol(status, g_device_status, sizeof(uint32_t))) != cudaSuccess) return e;
+    uint32_t mine = 0, gemm = 0;
+    if ((e = cudaMemcpyFromSymbol(&mine, g_device_status, sizeof(uint32_t))) != cudaSuccess) return e;
     const uint32_t zero = 0;
-    return cudaMemcpyToSymbol(g_device_status, &zero, sizeof(uint32_t));
+    if ((e = cudaMemcpyToSymbol(g_device_status, &zero, sizeof(uint32_t))) != cudaSuccess) return e;
+    if ((e = read_device_status_gemm(&gemm)) != cudaSuccess) return e;
+    *status = mine | gemm;
+    return cudaSuccess;
 }
 
 cudaError_t launch_selftest_timeout(unsigned long long limit_ns, cudaStream_t s) {
@@ -866,11 +594,7 @@ cudaError_t launch_selftest_timeout(unsigned long long limit_ns, cudaStream_t s)
 }
 
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
-    if (B <= 1) return launch_gemv1(L, X, Y, s);
-    if (B <= 2) return launch_nb<2>(L, X, Y, B, s);
-    if (B <= 4) return launch_nb<4>(L, X, Y, B, s);
-    if (B <= 8) return launch_nb<8>(L, X, Y, B, s);
-    return launch_nb<16>(L, X, Y, B, s);
+    return B <= 1 ? launch_gemv1(L, X, Y, s) : launch_gemm_small(L, X, Y, B, s);
 }
 
 }  // namespace vbq

@@ -28,10 +28,14 @@ cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B,
 constexpr int STATIC_CTL_WORDS = 2 + 8192;
 cudaError_t launch_gemv1_static(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s);
 
-// Bounded-wait report: synchronise s, read and clear the device status word
-// (nonzero when some wait gave up); and the self-test that makes one wait run
-// out after limit_ns.
+// Batch 2..16 on the tensor cores (vbq_gemm.cu); Y is B x N, overwritten.
+cudaError_t launch_gemm_small(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s);
+
+// Bounded-wait report: synchronise s, read and clear the device status words
+// of both product files (nonzero when some wait gave up); and the self-test
+// that makes one wait run out after limit_ns.
 cudaError_t read_device_status(uint32_t* status, cudaStream_t s);
+cudaError_t read_device_status_gemm(uint32_t* status);
 cudaError_t launch_selftest_timeout(unsigned long long limit_ns, cudaStream_t s);
 
 }  // namespace vbq

@@ -139,6 +139,41 @@ def test_all_zero_level(b):
     assert float(y.abs().max()) <= 1e-5
 
 
+@pytest.mark.parametrize("b", [1, 2, 4, 8])
+@pytest.mark.parametrize("batch", [3, 16])
+def test_all_zero_level_batched(b, batch):
+    n, k = 256, 2048
+    codes = np.full((n, k), 1 << (b - 1) if b > 1 else 0, np.uint8)
+    widths = np.full((n, k // 64), b, np.uint8)
+    m = Matrix(n, k, seed_path=(95, b, 1), batch=batch)
+    layout = vbq.vbq_pack(torch.from_numpy(codes).to(DEV), torch.from_numpy(widths).to(DEV),
+                          scales_to_i16(m.scales).to(DEV))
+    x = bits_to_i16(m.x_bits).to(DEV)
+    y = torch.empty((batch, n), dtype=torch.float32, device=DEV)
+    vbq.vbq_gemm_small(layout, x, y, batch)
+    if b > 1:                                # every code at the zero level: exactly 0
+        assert float(y.abs().max()) == 0.0
+    else:                                    # one bit has no zero level: y = -s * sum(x) per group
+        y_ref, a_ref = oracle.gemv(codes, widths, m.scales, m.x()[:batch])
+        assert oracle.within_bound(y.cpu().numpy(), y_ref, a_ref).all()
+
+
+def test_one_hot_exact_batched():
+    m = Matrix(640, 1024, seed_path=(94, 1, 0))
+    layout = _pack(m)
+    w_ref = oracle.dequant(m.codes.numpy(), m.widths, m.scales)
+    cols = (0, 1, 63, 64, 511, 1023)
+    xb = np.zeros((len(cols), 1024), np.uint16)
+    for r, j in enumerate(cols):
+        xb[r, j] = 0x3F80                    # bf16 1.0
+    x = bits_to_i16(xb).to(DEV)
+    y = torch.empty((len(cols), 640), dtype=torch.float32, device=DEV)
+    vbq.vbq_gemm_small(layout, x, y, len(cols))
+    torch.cuda.synchronize()
+    for r, j in enumerate(cols):
+        assert np.array_equal(y[r].cpu().numpy().astype(np.float64), w_ref[:, j])
+
+
 def test_one_hot_exact():
     m = Matrix(640, 1024, seed_path=(94, 0, 0))
     layout = _pack(m)
