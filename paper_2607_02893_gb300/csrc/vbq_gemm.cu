@@ -41,8 +41,13 @@ namespace {
 constexpr int NCWB = 16;                 // consumer warps
 constexpr int NCTB = 32 * NCWB;
 constexpr int GB_THREADS = 32 * (NCWB + 1);
-constexpr int NSTAGE_B = 3;              // blob stages in flight per SM
 constexpr int STAGE_BYTES_B = MAX_BLOB_BYTES;
+// Stages and consumer teams: with NB = 8 A rows the tables leave room for four
+// stages, so up to four teams (each team's units then use stages of their
+// own); NB = 16 fits three stages and one team.
+template <int NB> struct Pipe { static constexpr int stages = NB == 8 ? 4 : 3, max_teams = NB == 8 ? 4 : 1; };
+static_assert(Pipe<8>::stages % Pipe<8>::max_teams == 0 && Pipe<16>::stages % Pipe<16>::max_teams == 0,
+              "each team's units use stages no other team uses");
 static_assert(STAGE_BYTES_B % 256 == 0, "stage alignment");
 
 // Shared-memory tables of the batched kernel; NB = 8 or 16 A rows.
@@ -50,15 +55,15 @@ template <int NB>
 struct __align__(16) TablesB {
     uint32_t afr[MAX_C][32][NB];         // A fragments (fp16x2) per column and lane: NB/4 per k-step
     float e2[MAX_C][16];                 // per column and batch row: 2^E (0 for absent rows)
-    float ys[NSTAGE_B][NB][RB];          // row partials of each stage, per batch row
-    unsigned long long full[NSTAGE_B];   // blob landed
-    unsigned long long empty[NSTAGE_B];  // the unit's team is done
+    float ys[Pipe<NB>::stages][NB][RB];            // row partials of each stage, per batch row
+    unsigned long long full[Pipe<NB>::stages];     // blob landed
+    unsigned long long empty[Pipe<NB>::stages];    // the unit's team is done
     int abort;
 };
 
 template <int NB>
-constexpr size_t gemmb_smem() { return 256 + (size_t)NSTAGE_B * STAGE_BYTES_B + sizeof(TablesB<NB>); }
-static_assert(gemmb_smem<16>() <= 227 * 1024, "one block per SM");
+constexpr size_t gemmb_smem() { return 256 + (size_t)Pipe<NB>::stages * STAGE_BYTES_B + sizeof(TablesB<NB>); }
+static_assert(gemmb_smem<16>() <= 227 * 1024 && gemmb_smem<8>() <= 227 * 1024, "one block per SM");
 
 __device__ __forceinline__ void consumer_sync_b() {
     asm volatile("bar.sync 1, %0;" :: "n"(NCTB) : "memory");
@@ -68,6 +73,13 @@ __device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], 
     asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
                  : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
                  : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// The same with a zero accumulator (the first k-step of a tile).
+__device__ __forceinline__ void mma16816_z(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%10,%10};"
+                 : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
 }
 
 __device__ __forceinline__ float bf16_bits(uint32_t b) { return __uint_as_float(b << 16); }
@@ -158,13 +170,10 @@ __device__ __forceinline__ void bfrag_8(uint4 w, uint32_t (&b)[8]) {   // w = wo
     }
 }
 
-__device__ __forceinline__ int pick4(const int (&v)[4], int w) {   // v[w] for a warp-uniform w
-    return w == 0 ? v[0] : w == 1 ? v[1] : w == 2 ? v[2] : v[3];
-}
-
-// u * 2^-24 -> L(u) * 2^-24 in both halves: 2u - 1 (z = 0: one bit) or u - z.
-__device__ __forceinline__ void to_levels(uint32_t (&b)[8], int w) {
-    if (w == 0) {
+// u * 2^-24 -> L(u) * 2^-24 in both halves: 2u - 1 for one bit, u - z otherwise.
+template <int W>
+__device__ __forceinline__ void to_levels(uint32_t (&b)[8]) {
+    if (W == 0) {
         const __half2 two = __floats2half2_rn(2.f, 2.f), m1 = __halves2half2(__ushort_as_half(0x8001u), __ushort_as_half(0x8001u));
 #pragma unroll
         for (int r = 0; r < 8; ++r) {
@@ -172,12 +181,52 @@ __device__ __forceinline__ void to_levels(uint32_t (&b)[8], int w) {
             b[r] = *reinterpret_cast<const uint32_t*>(&v);
         }
     } else {
-        const unsigned short zb = w == 1 ? 2 : w == 2 ? 8 : 128;   // z * 2^-24 as fp16 bits (a denormal)
+        constexpr unsigned short zb = W == 1 ? 2 : W == 2 ? 8 : 128;   // z * 2^-24 as fp16 bits (a denormal)
         const __half2 z = __halves2half2(__ushort_as_half(zb), __ushort_as_half(zb));
 #pragma unroll
         for (int r = 0; r < 8; ++r) {
             const __half2 v = __hsub2(*reinterpret_cast<const __half2*>(&b[r]), z);
             b[r] = *reinterpret_cast<const uint32_t*>(&v);
+        }
+    }
+}
+
+// Tiles k0 .. k1-1 of one (column, width W) bucket: items bs + 8k .. of the
+// bucket [bs, be); pay / scb / rwb: the width's payload, scales and row bytes.
+template <int NB, int W>
+__device__ __forceinline__ void run_tiles(const uint32_t (&a)[NB], float e2g, float e2g8, uint32_t pay, uint32_t scb,
+                                          uint32_t rwb, int bs, int be, int k0, int k1, uint32_t ys, int B, int g,
+                                          int t) {
+    for (int k = k0; k < k1; ++k) {
+        const int i0 = bs + 8 * k, nv = min(8, be - i0);              // this tile's items: i0 .. i0 + nv - 1
+        const int ig = i0 + min(g, nv - 1);                          // lane's item (a valid one past the end)
+        uint32_t b[8];
+        if (W == 0) bfrag_1(lds_u32x2(pay + ig * 8), t, b);
+        else if (W == 1) bfrag_2(lds_u32x4(pay + ig * 16), t, b);
+        else if (W == 2) bfrag_4(lds_u32x2(pay + ig * 32 + 8 * t), b);
+        else bfrag_8(lds_u32x4(pay + ig * 64 + 16 * t), b);
+        // scales and rows of the lane's output items 2t, 2t+1 (loaded early)
+        const int ia = i0 + min(2 * t, nv - 1), ib = i0 + min(2 * t + 1, nv - 1);
+        const float sa = half_bits(lds_u16(scb + 2 * ia)), sb = half_bits(lds_u16(scb + 2 * ib));
+        const int ra = lds_u8(rwb + ia), rb = lds_u8(rwb + ib);
+        to_levels<W>(b);
+        float d[4];
+#pragma unroll
+        for (int s2 = 0; s2 < 4; ++s2) {
+            uint32_t af[4];
+            if (NB == 16) { af[0] = a[4 * s2]; af[1] = a[4 * s2 + 1]; af[2] = a[4 * s2 + 2]; af[3] = a[4 * s2 + 3]; }
+            else { af[0] = a[2 * s2]; af[1] = 0u; af[2] = a[(2 * s2 + 1) % NB]; af[3] = 0u; }
+            if (s2 == 0) mma16816_z(d, af, b[0], b[1]);
+            else mma16816(d, af, b[2 * s2], b[2 * s2 + 1]);
+        }
+        // items 2t and 2t+1: scaled, added to the row partials of batch rows g and g + 8
+        if (g < B) {
+            if (2 * t < nv) red_shared(ys + 4 * (g * RB + ra), d[0] * (sa * e2g));
+            if (2 * t + 1 < nv) red_shared(ys + 4 * (g * RB + rb), d[1] * (sb * e2g));
+        }
+        if (NB == 16 && g + 8 < B) {
+            if (2 * t < nv) red_shared(ys + 4 * ((g + 8) * RB + ra), d[2] * (sa * e2g8));
+            if (2 * t + 1 < nv) red_shared(ys + 4 * ((g + 8) * RB + rb), d[3] * (sb * e2g8));
         }
     }
 }
@@ -191,7 +240,7 @@ __device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sb
     const int g = lane >> 2, t = lane & 3;
     const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
     const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
-    // lane c (< cols) holds, per width, its bucket's first item, end and tile count
+    // lane c (< cols) holds, per width, its bucket's first item and end, and tile counts
     int start[4], end[4], ntile[4], nt_col = 0;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
@@ -212,74 +261,39 @@ __device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sb
     const int total = __shfl_sync(0xffffffffu, incl, 31);
     const int ta = (total * wt) / tw, tb = (total * (wt + 1)) / tw;
     if (ta >= tb) return;
-    // locate tile ta: its column c, width w and tile k within the bucket
-    int c = __popc(__ballot_sync(0xffffffffu, incl <= ta));
-    int k = ta - (__shfl_sync(0xffffffffu, incl, c) - __shfl_sync(0xffffffffu, nt_col, c));
-    int w = 0, ntw = __shfl_sync(0xffffffffu, ntile[0], c);
-    while (k >= ntw) { k -= ntw; ++w; ntw = __shfl_sync(0xffffffffu, pick4(ntile, w), c); }
-    int bs = __shfl_sync(0xffffffffu, pick4(start, w), c), be = __shfl_sync(0xffffffffu, pick4(end, w), c);
-
-    int cur_c = -1;
-    uint32_t a[NB];
-    float e2g = 0.f, e2g8 = 0.f;
-    for (int tile = ta; tile < tb; ++tile) {
-        if (c != cur_c) {                // A fragments, zero-level sums and 2^E of the new column
+    const uint32_t pay[4] = {sblob + (h0.z & 0xFFFF) * 16, sblob + (h0.z >> 16) * 16, sblob + (h0.w & 0xFFFF) * 16,
+                             sblob + (h0.w >> 16) * 16};
+    const uint32_t scb[4] = {sblob + (h1.x & 0xFFFF) * 16, sblob + (h1.x >> 16) * 16, sblob + (h1.y & 0xFFFF) * 16,
+                             sblob + (h1.y >> 16) * 16};
+    const uint32_t rwb[4] = {sblob + (h1.z & 0xFFFF) * 16, sblob + (h1.z >> 16) * 16, sblob + (h1.w & 0xFFFF) * 16,
+                             sblob + (h1.w >> 16) * 16};
+    // walk the columns that hold tiles ta .. tb-1; per column, its four width buckets
+    for (int c = __popc(__ballot_sync(0xffffffffu, incl <= ta)); c < cols; ++c) {
+        const int c_end = __shfl_sync(0xffffffffu, incl, c), c_begin = c_end - __shfl_sync(0xffffffffu, nt_col, c);
+        if (c_begin >= tb) break;
+        uint32_t a[NB];
+        {
             const uint32_t* src = &T.afr[c][lane][0];
 #pragma unroll
             for (int r = 0; r < NB; r += 4) {
                 const uint4 v = *reinterpret_cast<const uint4*>(src + r);
                 a[r] = v.x; a[r + 1] = v.y; a[r + 2] = v.z; a[r + 3] = v.w;
             }
-            e2g = T.e2[c][g]; e2g8 = T.e2[c][g + 8];
-            cur_c = c;
         }
-        const int i0 = bs + 8 * k, nv = min(8, be - i0);           // this tile's items: i0 .. i0 + nv - 1
-        const int ig = i0 + min(g, nv - 1);                        // lane's item (a valid one past the end)
-        uint32_t b[8];
-        uint32_t sc_base, row_base;
-        if (w == 0) {
-            bfrag_1(lds_u32x2(sblob + (h0.z & 0xFFFF) * 16 + ig * 8), t, b);
-            sc_base = sblob + (h1.x & 0xFFFF) * 16; row_base = sblob + (h1.z & 0xFFFF) * 16;
-        } else if (w == 1) {
-            bfrag_2(lds_u32x4(sblob + (h0.z >> 16) * 16 + ig * 16), t, b);
-            sc_base = sblob + (h1.x >> 16) * 16; row_base = sblob + (h1.z >> 16) * 16;
-        } else if (w == 2) {
-            bfrag_4(lds_u32x2(sblob + (h0.w & 0xFFFF) * 16 + ig * 32 + 8 * t), b);
-            sc_base = sblob + (h1.y & 0xFFFF) * 16; row_base = sblob + (h1.w & 0xFFFF) * 16;
-        } else {
-            bfrag_8(lds_u32x4(sblob + (h0.w >> 16) * 16 + ig * 64 + 16 * t), b);
-            sc_base = sblob + (h1.y >> 16) * 16; row_base = sblob + (h1.w >> 16) * 16;
-        }
-        to_levels(b, w);
-        float d[4] = {0.f, 0.f, 0.f, 0.f};
+        const float e2g = T.e2[c][g], e2g8 = T.e2[c][g + 8];
+        int tile0 = c_begin;                            // global index of the bucket's first tile
 #pragma unroll
-        for (int s2 = 0; s2 < 4; ++s2) {
-            uint32_t af[4];
-            if (NB == 16) { af[0] = a[4 * s2]; af[1] = a[4 * s2 + 1]; af[2] = a[4 * s2 + 2]; af[3] = a[4 * s2 + 3]; }
-            else { af[0] = a[2 * s2]; af[1] = 0u; af[2] = a[(2 * s2 + 1) % NB]; af[3] = 0u; }
-            mma16816(d, af, b[2 * s2], b[2 * s2 + 1]);
-        }
-        // items 2t and 2t+1 of the tile: scale, add to the row partials of batch rows g and g + 8
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            const int n = 2 * t + e;
-            if (n < nv) {
-                const int i = i0 + n;
-                const float sc = half_bits(lds_u16(sc_base + 2 * i));
-                const int r = lds_u8(row_base + i);
-                if (g < B) red_shared(ys + 4 * (g * RB + r), d[e] * (sc * e2g));
-                if (NB == 16 && g + 8 < B) red_shared(ys + 4 * ((g + 8) * RB + r), d[2 + e] * (sc * e2g8));
+        for (int w = 0; w < 4; ++w) {
+            const int nt = __shfl_sync(0xffffffffu, ntile[w], c);
+            const int k0 = max(ta - tile0, 0), k1 = min(tb - tile0, nt);
+            if (k0 < k1) {
+                const int bs = __shfl_sync(0xffffffffu, start[w], c), be = __shfl_sync(0xffffffffu, end[w], c);
+                if (w == 0) run_tiles<NB, 0>(a, e2g, e2g8, pay[0], scb[0], rwb[0], bs, be, k0, k1, ys, B, g, t);
+                else if (w == 1) run_tiles<NB, 1>(a, e2g, e2g8, pay[1], scb[1], rwb[1], bs, be, k0, k1, ys, B, g, t);
+                else if (w == 2) run_tiles<NB, 2>(a, e2g, e2g8, pay[2], scb[2], rwb[2], bs, be, k0, k1, ys, B, g, t);
+                else run_tiles<NB, 3>(a, e2g, e2g8, pay[3], scb[3], rwb[3], bs, be, k0, k1, ys, B, g, t);
             }
-        }
-        // next tile: the next one of this bucket, else the next non-empty bucket in (column, width) order
-        if (++k == ntw && tile + 1 < tb) {
-            k = 0;
-            do {
-                if (++w == 4) { w = 0; ++c; }
-                ntw = __shfl_sync(0xffffffffu, pick4(ntile, w), c);
-            } while (ntw == 0);
-            bs = __shfl_sync(0xffffffffu, pick4(start, w), c);
-            be = __shfl_sync(0xffffffffu, pick4(end, w), c);
+            tile0 += nt;
         }
     }
 }
@@ -287,9 +301,10 @@ __device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sb
 template <int NB>
 __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, const uint16_t* __restrict__ X,
                                                               float* __restrict__ Y, int B) {
+    constexpr int NST = Pipe<NB>::stages;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     unsigned char* base = smem_raw + ((256u - (smem_u32(smem_raw) & 255u)) & 255u);
-    TablesB<NB>& T = *reinterpret_cast<TablesB<NB>*>(base + (size_t)NSTAGE_B * STAGE_BYTES_B);
+    TablesB<NB>& T = *reinterpret_cast<TablesB<NB>*>(base + (size_t)NST * STAGE_BYTES_B);
     const uint32_t stage0 = smem_u32(base);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int P = gridDim.x, p = blockIdx.x;
@@ -298,27 +313,27 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
     const int n_units = u_end - u_begin;
     if (n_units <= 0) return;
     const int s0 = u_begin / L.nrb, rb0 = u_begin - s0 * L.nrb;
-    // One team: every consumer warp takes every unit, so each waits every phase
-    // of every stage in order. (Several teams over NSTAGE_B = 3 stages would let a
-    // team skip phases of a stage that other teams' units use; a parity wait can
-    // then match an older completed phase. The batch-1 kernel avoids that by
-    // giving each team stages of its own.)
-    const int teams = 1, tw = NCWB;
+    // Teams as in the batch-1 kernel, at most Pipe<NB>::max_teams: unit j uses
+    // stage j % stages and goes to team j % teams, and teams divides stages, so
+    // each team waits the phases of its own stages in order (a parity wait that
+    // skipped a phase could match an older completed one).
+    const int lg_teams = Pipe<NB>::max_teams == 4 ? (n_units >= 16 ? 2 : n_units >= 8 ? 1 : 0) : 0;
+    const int teams = 1 << lg_teams, tw = NCWB >> lg_teams;
 
     const uint32_t full0 = smem_u32(&T.full[0]), empty0 = smem_u32(&T.empty[0]);
     const uint32_t abort_addr = smem_u32(&T.abort);
     if (tid == 0) {
-        for (int i = 0; i < NSTAGE_B; ++i) {
+        for (int i = 0; i < NST; ++i) {
             mbar_init(full0 + 8 * i, 1);
             mbar_init(empty0 + 8 * i, tw);
         }
         T.abort = 0;
         fence_barrier_init();
     }
-    for (int i = tid; i < NSTAGE_B * NB * RB; i += GB_THREADS) (&T.ys[0][0][0])[i] = 0.f;
+    for (int i = tid; i < NST * NB * RB; i += GB_THREADS) (&T.ys[0][0][0])[i] = 0.f;
     __syncthreads();
     if (tid == 0) {
-        const int first = n_units < NSTAGE_B ? n_units : NSTAGE_B;
+        const int first = n_units < NST ? n_units : NST;
         for (int j = 0; j < first; ++j) issue_unit(L, u_begin + j, stage0 + j * STAGE_BYTES_B, full0 + 8 * j);
     }
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -344,7 +359,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             }
         }
         bool dead = false, checked = L.S == 1;
-        int st = 0, rbw = rb0, issued = n_units < NSTAGE_B ? n_units : NSTAGE_B;
+        int st = 0, rbw = rb0, issued = n_units < NST ? n_units : NST;
         uint32_t par = 0;
         for (int j = 0; j < n_units; ++j) {
             if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 256)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
@@ -372,18 +387,18 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
                     }
                 }
                 __syncwarp();
-                if (j + NSTAGE_B < n_units) {
-                    if (lane == 0) issue_unit(L, u_begin + j + NSTAGE_B, stage0 + st * STAGE_BYTES_B, full0 + 8 * st);
+                if (j + NST < n_units) {
+                    if (lane == 0) issue_unit(L, u_begin + j + NST, stage0 + st * STAGE_BYTES_B, full0 + 8 * st);
                     ++issued;
                 }
             }
-            if (++st == NSTAGE_B) { st = 0; par ^= 1; }
+            if (++st == NST) { st = 0; par ^= 1; }
             if (++rbw == L.nrb) rbw = 0;
         }
         if (dead && lane == 0) {
-            for (int i = 0; i < NSTAGE_B && i < issued; ++i) {
-                const int jl = i + ((issued - 1 - i) / NSTAGE_B) * NSTAGE_B;
-                mbar_wait_bounded(full0 + 8 * i, (uint32_t)((jl / NSTAGE_B) & 1));
+            for (int i = 0; i < NST && i < issued; ++i) {
+                const int jl = i + ((issued - 1 - i) / NST) * NST;
+                mbar_wait_bounded(full0 + 8 * i, (uint32_t)((jl / NST) & 1));
             }
         }
         if (L.S > 1 && lane == 0) {
@@ -403,8 +418,8 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
         build_tables_b(T, L, X, B, s0, ct);
         for (int j = team; j < n_units; j += teams) {
             while (cur < sj) build_tables_b(T, L, X, B, ++cur, ct);
-            const int st = j % NSTAGE_B;
-            const uint32_t par = (uint32_t)(j / NSTAGE_B) & 1u;
+            const int st = j % NST;
+            const uint32_t par = (uint32_t)(j / NST) & 1u;
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
                 consume_unit_b<NB>(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
