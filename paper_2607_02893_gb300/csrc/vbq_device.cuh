@@ -81,6 +81,13 @@ __device__ __forceinline__ void red_global(float* p, float v) {
     asm volatile("red.global.add.f32 [%0], %1;" :: "l"(p), "f"(v) : "memory");
 }
 
+// Bring the 128-byte line holding p into L2 (no value is read: safe before
+// griddepcontrol.wait, since a later write by the previous grid updates the
+// line in L2, where coherence is kept).
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+    asm volatile("prefetch.global.L2 [%0];" :: "l"(p));
+}
+
 __device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) {
     return *reinterpret_cast<const volatile uint32_t*>(p);
 }

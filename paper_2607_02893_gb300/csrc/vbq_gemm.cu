@@ -336,6 +336,12 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
         const int first = n_units < NST ? n_units : NST;
         for (int j = 0; j < first; ++j) issue_unit(L, u_begin + j, stage0 + j * STAGE_BYTES_B, full0 + 8 * j);
     }
+    {   // the first slab's activations into L2 while waiting for the previous grid
+        const int64_t k0 = (int64_t)s0 * L.C * GROUP;
+        const int lines = (min(L.C, L.G - s0 * L.C) * GROUP * 2 + 127) / 128;
+        for (int q = tid - 32; q >= 0 && q < lines * B; q += GB_THREADS - 32)
+            prefetch_l2(X + (int64_t)(q / lines) * L.K + k0 + (int64_t)(q % lines) * 64);
+    }
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");
 

@@ -376,7 +376,13 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     }
     // Weights never depend on earlier work in the stream, so the first copies
     // are in flight before this grid waits for its predecessor (programmatic
-    // dependent launch); x, y and the control words are touched only after.
+    // dependent launch); x, y and the control words are read only after. The
+    // first slab's activations are prefetched into L2 meanwhile.
+    {
+        const int64_t k0 = (int64_t)s0 * L.C * GROUP;
+        const int lines = (min(L.C, L.G - s0 * L.C) * GROUP * 2 + 127) / 128;
+        if (tid >= 32 && tid - 32 < lines) prefetch_l2(x + k0 + (int64_t)(tid - 32) * 64);
+    }
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");
 
