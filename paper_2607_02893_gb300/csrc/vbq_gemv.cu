@@ -114,15 +114,8 @@ __device__ __forceinline__ void plane_entries(uint32_t tb, uint32_t sh4, uint32_
     v[15] = lds_f32<960>(__byte_perm(ho, tb, 0x7653));
 }
 
-// Sum of 16 values as a balanced tree (pairs, then pairs of pairs): the order
-// every lookup sum and xlut use.
-__device__ __forceinline__ float tree16(const float* v) {
-    const float a0 = v[0] + v[1], a1 = v[2] + v[3], a2 = v[4] + v[5], a3 = v[6] + v[7];
-    const float a4 = v[8] + v[9], a5 = v[10] + v[11], a6 = v[12] + v[13], a7 = v[14] + v[15];
-    return ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
-}
-
-// tree16 of a (in .x) and of b (in .y) at once, with f32x2 adds.
+// Sums of a (in .x) and of b (in .y) as balanced trees (pairs, then pairs of
+// pairs: the order the all-ones column sums xlut use), with f32x2 adds.
 __device__ __forceinline__ float2 tree16x2(const float (&a)[16], const float (&b)[16]) {
     float2 p[8];
 #pragma unroll
@@ -185,55 +178,68 @@ __device__ __forceinline__ void consumer_sync() {
 
 // Activations of slab s: x as fp32, the pre-scaled x of the 4-bit slots, the
 // nibble lookup tables, and the per-column sums in lookup order. Consumer
-// threads only (ct = 0 .. NCT-1); starts and ends with a consumer barrier.
+// threads only (ct = 0 .. NCT-1), one thread per (column, 4 weights): each
+// reads its 4 activations from global memory (L2), so the whole build is one
+// phase between two consumer barriers. The column sum of the all-ones entries
+// (xlut) is added over the column's half-warp in the pairs tree16x2 uses.
 __device__ void build_tables(Tables& T, const LayoutView& L, const uint16_t* __restrict__ x, int s, int ct) {
     const int cols = min(L.C, L.G - s * L.C);
-    const int64_t k0 = (int64_t)s * L.C * GROUP;
+    const uint16_t* xg = x + (int64_t)s * L.C * GROUP;
     consumer_sync();                // nobody still reads the old tables
-    for (int i = ct; i < cols * 32; i += NCT) {
-        const uint32_t two = __ldg(reinterpret_cast<const uint32_t*>(x + k0) + i);
-        const float xa = __uint_as_float(two << 16), xb = __uint_as_float(two & 0xFFFF0000u);
-        const int kk = 2 * i, c = kk >> 6, jj = kk & 63;
-        *reinterpret_cast<float2*>(&T.xs[(c * 4 + (jj >> 4)) * XQ + (jj & 15)]) = f2(xa, xb);
+    if (ct < cols * 16) {
+        const int c = ct >> 4, jn = ct & 15, jj = 4 * jn;
+        const uint2 four = __ldg(reinterpret_cast<const uint2*>(xg + c * GROUP + jj));
+        const float x0 = __uint_as_float(four.x << 16), x1 = __uint_as_float(four.x & 0xFFFF0000u);
+        const float x2 = __uint_as_float(four.y << 16), x3 = __uint_as_float(four.y & 0xFFFF0000u);
+        *reinterpret_cast<float4*>(&T.xs[(c * 4 + (jj >> 4)) * XQ + (jj & 15)]) = make_float4(x0, x1, x2, x3);
         // 4-bit slot shifts: nibble slots 0..5 of a word keep their place, 6 and 7 come down by 24
-        const int slot = jj & 7, e = slot < 6 ? 4 * slot : 4 * (slot - 6);
-        *reinterpret_cast<float2*>(&T.x4s[(c * 2 + (jj >> 5)) * XH + (jj & 31)]) =
-            f2(xa * __uint_as_float((uint32_t)(127 + 49 - e) << 23),
-               xb * __uint_as_float((uint32_t)(127 + 49 - e - 4) << 23));
-    }
-    consumer_sync();
-    for (int pj = ct; pj < cols * 16; pj += NCT) {
-        const int c = pj >> 4, jn = pj & 15;
-        const float4 xv = *reinterpret_cast<const float4*>(&T.xs[(c * 4 + (jn >> 2)) * XQ + 4 * (jn & 3)]);
-        const float t3 = xv.x + xv.y, t12 = xv.w + xv.z;
+        float p4[4];
+        const float xv4[4] = {x0, x1, x2, x3};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int slot = (jj + i) & 7, e = slot < 6 ? 4 * slot : 4 * (slot - 6);
+            p4[i] = xv4[i] * __uint_as_float((uint32_t)(127 + 49 - e) << 23);
+        }
+        *reinterpret_cast<float4*>(&T.x4s[(c * 2 + (jj >> 5)) * XH + (jj & 31)]) = make_float4(p4[0], p4[1], p4[2], p4[3]);
+        const float t3 = x0 + x1, t12 = x3 + x2;
         float4* dst = reinterpret_cast<float4*>(T.lut + c * LUT_COL_BYTES + (c & 1) * 64 + jn * 64);
-        dst[0] = make_float4(0.f, xv.x, xv.y, t3);
-        dst[1] = make_float4(xv.z, xv.z + xv.x, xv.z + xv.y, xv.z + t3);
-        dst[2] = make_float4(xv.w, xv.w + xv.x, xv.w + xv.y, xv.w + t3);
-        dst[3] = make_float4(t12, t12 + xv.x, t12 + xv.y, t12 + t3);
-    }
-    consumer_sync();
-    if (ct < cols) {
-        const float* t = reinterpret_cast<const float*>(T.lut + ct * LUT_COL_BYTES + (ct & 1) * 64);
-        float v[16];
+        dst[0] = make_float4(0.f, x0, x1, t3);
+        dst[1] = make_float4(x2, x2 + x0, x2 + x1, x2 + t3);
+        dst[2] = make_float4(x3, x3 + x0, x3 + x1, x3 + t3);
+        dst[3] = make_float4(t12, t12 + x0, t12 + x1, t12 + t3);
+        // xlut: balanced tree over the column's 16 all-ones entries (xor 1, 2, 4, 8
+        // pair them as tree16x2 pairs the lookups)
+        const unsigned half = (ct & 16) ? 0xFFFF0000u : 0x0000FFFFu;
+        float v = t12 + t3;
+        v += __shfl_xor_sync(half, v, 1);
+        v += __shfl_xor_sync(half, v, 2);
+        v += __shfl_xor_sync(half, v, 4);
+        v += __shfl_xor_sync(half, v, 8);
+        if (jn == 0) T.xlut[c] = v;
+        // X for the 4-bit zero level of half hh, summed as dot4_half accumulates
+        if ((jn & 7) == 0) {
+            const int hh = jn >> 3;
+            const uint4* src = reinterpret_cast<const uint4*>(xg + c * GROUP + 32 * hh);
+            float xh[32];
 #pragma unroll
-        for (int jn = 0; jn < 16; ++jn) v[jn] = t[jn * 16 + 15];
-        T.xlut[ct] = tree16(v);
-        // X for the 4-bit zero level, summed as dot4_half accumulates
+            for (int q = 0; q < 4; ++q) {
+                const uint4 w = __ldg(src + q);
+                const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
+                for (int i = 0; i < 4; ++i) {
+                    xh[8 * q + 2 * i] = __uint_as_float(ws[i] << 16);
+                    xh[8 * q + 2 * i + 1] = __uint_as_float(ws[i] & 0xFFFF0000u);
+                }
+            }
             float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
 #pragma unroll
             for (int t4 = 0; t4 < 4; ++t4) {
                 float2& cc = (t4 & 1) ? cb : ca;
 #pragma unroll
-                for (int e = 0; e < 8; e += 2) {
-                    const int jj = 32 * hh + 8 * t4 + e;
-                    const float* xq = &T.xs[(ct * 4 + (jj >> 4)) * XQ + (jj & 15)];
-                    cc = __ffma2_rn(f2(xq[0], xq[1]), f2(0x1p-100f, 0x1p-100f), cc);
-                }
+                for (int e = 0; e < 8; e += 2)
+                    cc = __ffma2_rn(f2(xh[8 * t4 + e], xh[8 * t4 + e + 1]), f2(0x1p-100f, 0x1p-100f), cc);
             }
-            T.x4z[ct][hh] = __fadd2_rn(ca, cb);
+            T.x4z[c][hh] = __fadd2_rn(ca, cb);
         }
     }
     consumer_sync();
