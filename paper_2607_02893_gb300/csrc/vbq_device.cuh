@@ -200,22 +200,22 @@ __device__ __forceinline__ int col_within(uint32_t ce, int cf, int cl, int i) { 
 }
 
 // Split-K: true once every row block this block adds a slab s > 0 into has
-// been zeroed in this call (flag == epoch), within the wait limit. One thread;
-// ends with an acquire fence.
+// been zeroed in this call (flag == epoch), within the wait limit. A whole warp:
+// lane i watches units u_begin + i, + 32, ..., so one round trip covers them
+// all; ends with an acquire fence.
 __device__ __forceinline__ bool split_k_flags_ready(const LayoutView& L, uint32_t epoch, int u_begin, int u_end,
-                                                    int s0, int rb0) {
+                                                    int lane) {
     bool seen = true;
     const unsigned long long t0 = global_ns();
-    int s2 = s0, rb2 = rb0;
-    for (int u = u_begin; u < u_end && seen; ++u) {
-        if (s2 > 0) {
-            while (!(seen = ld_volatile(L.ctl + 2 + rb2) == epoch))
+    for (int u = u_begin + lane; u < u_end && seen; u += 32) {
+        if (u >= L.nrb) {               // slab > 0
+            const uint32_t* f = L.ctl + 2 + (u % L.nrb);
+            while (!(seen = ld_volatile(f) == epoch))
                 if (global_ns() - t0 > WAIT_LIMIT_NS) break;
         }
-        if (++rb2 == L.nrb) { rb2 = 0; ++s2; }
     }
     asm volatile("fence.acq_rel.gpu;" ::: "memory");
-    return seen;
+    return __all_sync(0xffffffffu, seen);
 }
 
 }  // namespace

@@ -364,18 +364,16 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
                 for (int u = u_begin; u < z_end; ++u) st_volatile(L.ctl + 2 + u, epoch);
             }
         }
-        bool dead = false, checked = L.S == 1;
+        bool dead = false;
+        if (L.S > 1 && !split_k_flags_ready(L, epoch, u_begin, u_end, lane)) {
+            // a row block this block adds into was never zeroed in time
+            dead = true;
+            if (lane == 0) raise_abort(&T.abort);
+        }
         int st = 0, rbw = rb0, issued = n_units < NST ? n_units : NST;
         uint32_t par = 0;
         for (int j = 0; j < n_units; ++j) {
             if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 256)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
-            if (!dead && !checked) {
-                int ok = 1;
-                if (lane == 0) ok = split_k_flags_ready(L, epoch, u_begin, u_end, s0, rb0);
-                ok = __shfl_sync(0xffffffffu, ok, 0);
-                checked = true;
-                if (!ok) { dead = true; if (lane == 0) raise_abort(&T.abort); }
-            }
             if (!dead) {
                 const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
                 for (int b = 0; b < B; ++b) {

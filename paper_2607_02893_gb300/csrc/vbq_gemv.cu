@@ -411,20 +411,16 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                 for (int u = u_begin; u < z_end; ++u) st_volatile(L.ctl + 2 + u, epoch);
             }
         }
-        bool dead = false, checked = L.S == 1;
+        bool dead = false;
+        if (L.S > 1 && !split_k_flags_ready(L, epoch, u_begin, u_end, lane)) {
+            // a row block this block adds into was never zeroed in time
+            dead = true;
+            if (lane == 0) raise_abort(&T.abort);
+        }
         int st = 0, rbw = rb0, issued = n_units < NSTAGE ? n_units : NSTAGE;
         uint32_t par = 0;
         for (int j = 0; j < n_units; ++j) {
             if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 256)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
-            if (!dead && !checked) {
-                // before the first add into y: every row block this block adds a
-                // slab s > 0 into has been zeroed in this call
-                int ok = 1;
-                if (lane == 0) ok = split_k_flags_ready(L, epoch, u_begin, u_end, s0, rb0);
-                ok = __shfl_sync(0xffffffffu, ok, 0);
-                checked = true;
-                if (!ok) { dead = true; if (lane == 0) raise_abort(&T.abort); }
-            }
             if (!dead) {
                 float* ys = T.ys[st];
                 const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
