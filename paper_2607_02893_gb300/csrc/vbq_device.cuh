@@ -88,6 +88,19 @@ __device__ __forceinline__ void prefetch_l2(const void* p) {
     asm volatile("prefetch.global.L2 [%0];" :: "l"(p));
 }
 
+// Order this thread's earlier writes (and those it has observed) before its
+// later ones, GPU-wide: the release half of __threadfence, without waiting for
+// sequential consistency.
+__device__ __forceinline__ void fence_release_gpu() {
+    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+}
+// Atomic add with acquire-release ordering at GPU scope; returns the old value.
+__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
 __device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) {
     return *reinterpret_cast<const volatile uint32_t*>(p);
 }

@@ -360,7 +360,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             }
             __syncwarp();
             if (lane == 0 && u_begin < z_end) {
-                __threadfence();
+                fence_release_gpu();        // the zeros before the flags
                 for (int u = u_begin; u < z_end; ++u) st_volatile(L.ctl + 2 + u, epoch);
             }
         }
@@ -406,8 +406,9 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             }
         }
         if (L.S > 1 && lane == 0) {
-            __threadfence();
-            if (atomicAdd(L.ctl + 1, 1u) == gridDim.x - 1) {
+            // (acquire-release: this block's read of the epoch comes before its
+            // count, and the last block's epoch write after every count)
+            if (atom_add_acq_rel(L.ctl + 1, 1u) == gridDim.x - 1) {
                 st_volatile(L.ctl + 1, 0u);
                 st_volatile(L.ctl, epoch);
             }
