@@ -1,10 +1,13 @@
 """Benchmark: batch-1 VBQ decode GEMV over a synthetic decoder linear stack.
 
-One step = one token through every linear layer of the stack (per layer Q, K,
-V, O, gate, up, down, then the LM head), each a packed VBQ GEMV run by
-libvbq.so on one stream, replayed from a CUDA graph. Weights are
-random-but-seeded (synthetic) with the per-projection width distributions of
-the workload; every GEMV has its own resident BF16 activation vector.
+One step = one token through every linear layer of the stack, each a packed
+VBQ GEMV run by libvbq.so on one stream, replayed from a CUDA graph. The
+default workload, stack9b-fused, issues the projections that read the same
+input as one matrix (per layer QKV, O, gate-up, down, then the LM head);
+`--workload stack9b` runs one GEMV per projection (Q, K, V, O, gate, up,
+down). Weights are random-but-seeded (synthetic) with the per-projection width
+distributions of the workload; every GEMV has its own resident BF16 activation
+vector.
 
 Printed JSON line (rank 0):
   value         algorithmic HBM GB/s of the whole step: sum over GEMVs of
@@ -56,7 +59,7 @@ def parse():
     p.add_argument("--steps", type=int, default=300)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--workload", default="stack9b")
+    p.add_argument("--workload", default="stack9b-fused")
     p.add_argument("--batch", type=int, default=1)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--event-ring", type=int, default=4)

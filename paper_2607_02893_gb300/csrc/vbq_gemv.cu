@@ -49,7 +49,7 @@ namespace {
 constexpr int NCW = 16;                  // consumer warps of the batch-1 kernel
 constexpr int NCT = 32 * NCW;            // consumer threads
 constexpr int MAX_TEAMS = 4;             // consumer teams (1, 2 or 4 by units per block); unit j goes to team j % teams
-static_assert(NCW == 16 && MAX_TEAMS == 4, "teams of 16, 8 or 4 warps (powers of two)");
+static_assert(MAX_TEAMS == 4 && NCW % MAX_TEAMS == 0, "every team count splits the consumer warps evenly");
 // Unit j uses stage j % NSTAGE and goes to team j % teams; with NSTAGE a
 // multiple of every team count, each stage serves one team only, and that team
 // waits the stage's phases in order (a parity wait never skips a phase).
@@ -77,6 +77,8 @@ struct __align__(16) Tables {
 };
 static_assert(offsetof(Tables, full) % 8 == 0, "mbarriers are 8-byte aligned");
 static_assert(offsetof(Tables, lut) == 0, "tables start at the aligned base");
+static_assert(offsetof(Tables, x4z) % 16 == 0 && offsetof(Tables, xs) % 16 == 0 && offsetof(Tables, x4s) % 16 == 0,
+              "16-byte table reads");
 static_assert(RB % 32 == 0, "the copier flushes rows a warp at a time");
 static_assert(MAX_C <= 32, "a warp holds a unit's column ends one per lane");
 
@@ -245,102 +247,149 @@ __device__ void build_tables(Tables& T, const LayoutView& L, const uint16_t* __r
     consumer_sync();
 }
 
-// One consumer warp's share of a unit (blob at shared address sblob, cols
-// group columns): tasks t = t0, t0 + tstep, ... of 16 four-bit groups (two
-// lanes each), 8 eight-bit groups (four lanes each), 32 two-bit groups, 64
-// one-bit groups (two per lane). Partials go to the row partials at shared
-// address ys by shared-memory reductions.
-__device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, int C, int cols, uint32_t ys,
-                                             int t0, int tstep, int lane) {
-    const uint32_t lut0 = smem_u32(T.lut), xs0 = smem_u32(T.xs), x4s0 = smem_u32(T.x4s);
-    const uint32_t x4z0 = smem_u32(T.x4z), xlut0 = smem_u32(T.xlut);
-    // UnitHeader fields, read as three 16-byte words
-    const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
-    const int n0 = h0.x & 0xFFFF, n1 = h0.x >> 16, n2 = h0.y & 0xFFFF, n3 = h0.y >> 16;
-    const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
-    uint32_t ce[4];                                     // this lane's column end of each width
+// Shared-memory addresses of one unit's blob and of the slab's tables, for
+// the per-width task loops.
+struct UnitView {
+    uint32_t pay, sc, row;      // this width's payload, FP16 scales, row bytes
+    uint32_t ce;                // this lane's column end for this width (0xFFFF past the slab's columns)
+    int n;                      // items of this width
+};
+
+// Column of item i (tasks hold items i0 .. i0 + span - 1; lanes agree on i0).
+__device__ __forceinline__ int task_column(uint32_t ce, int i0, int span, int n, int i) {
+    const int cf = col_uniform(ce, i0), cl = col_uniform(ce, min(i0 + span - 1, n - 1));
+    return cf == cl ? cf : col_within(ce, cf, cl, i);
+}
+
+// Tasks of one width: items are taken 32 (64 for 1-bit) at a time, task
+// k = first, first + tstep, ... of this width's nt tasks. Every lane holds
+// whole groups, so a task's bookkeeping is shared by 32 groups.
+template <int W>
+__device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, uint32_t ys, int first, int tstep,
+                                          int lane) {
+    constexpr int SPAN = W == 0 ? 64 : 32;
+    const int nt = (U.n + SPAN - 1) / SPAN;
+    for (int k = first; k < nt; k += tstep) {
+        const int i0 = k * SPAN;
+        if constexpr (W == 2) {
+            // 4-bit: one group per lane, halves in the order (lane >> 2) & 1 first,
+            // so each quarter-warp's 16-byte loads fall in 8 distinct bank groups
+            const int i = i0 + lane;
+            const int c = task_column(U.ce, i0, SPAN, U.n, i);
+            if (i < U.n) {
+                const int h0 = (lane >> 2) & 1;
+                const uint4 va = lds_u32x4(U.pay + i * 32 + h0 * 16), vb = lds_u32x4(U.pay + i * 32 + (h0 ^ 1) * 16);
+                const uint32_t xa = smem_u32(T.x4s) + (c * 2 + h0) * XH * 4, xb = smem_u32(T.x4s) + (c * 2 + (h0 ^ 1)) * XH * 4;
+                const float2 aa = dot4_half(va, xa), ab = dot4_half(vb, xb);
+                const float4 z = lds_f32x4(smem_u32(T.x4z) + c * 16);     // (even, odd) of half 0, then of half 1
+                const float part = ((aa.x + ab.x) - 8.f * (z.x + z.z)) + ((aa.y + ab.y) - 8.f * (z.y + z.w));
+                red_shared(ys + 4 * lds_u8(U.row + i), (half_bits(lds_u16(U.sc + 2 * i)) * 0x1p100f) * part);
+            }
+        } else if constexpr (W == 3) {
+            // 8-bit: one group per lane, quarter (k + (lane >> 1)) & 3 in step k
+            // (conflict-free 16-byte loads for every quarter-warp)
+            const int i = i0 + lane;
+            const int c = task_column(U.ce, i0, SPAN, U.n, i);
+            if (i < U.n) {
+                const int q0 = lane >> 1;
+                float part = 0.f;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) ce[w] = lane < cols ? lds_u16(cc + 2 * (w * C + lane)) : 0xFFFFu;
-    const int t4 = (n2 + 15) >> 4, t48 = t4 + ((n3 + 7) >> 3), t482 = t48 + ((n1 + 31) >> 5);
-    const int ntask = t482 + ((n0 + 63) >> 6);
-    for (int t = t0; t < ntask; t += tstep) {
-        if (t < t4) {                                   // 4-bit: two lanes per group, one half each
-            const uint32_t pay = sblob + (h0.w & 0xFFFF) * 16, sc = sblob + (h1.y & 0xFFFF) * 16;
-            const uint32_t row = sblob + (h1.w & 0xFFFF) * 16;
-            // lanes l and l+16 share group l%16; the half is swizzled so that a
-            // quarter-warp reads 8 distinct 16-byte bank groups
-            const int e = lane & 15, hh = ((e >> 2) + (lane >> 4)) & 1;
-            const int i0 = t * 16, i = i0 + e;
-            const int cf = col_uniform(ce[2], i0), cl = col_uniform(ce[2], min(i0 + 15, n2 - 1));
-            const int c = col_within(ce[2], cf, cl, i);
-            float part = 0.f;
-            if (i < n2) {
-                const uint4 v = lds_u32x4(pay + i * 32 + hh * 16);
-                const float2 acc = dot4_half(v, x4s0 + (c * 2 + hh) * XH * 4);
-                const float2 z = lds_f32x2(x4z0 + (c * 2 + hh) * 8);
-                part = (acc.x - 8.f * z.x) + (acc.y - 8.f * z.y);
+                for (int step = 0; step < 4; ++step) {
+                    const int q = (step + q0) & 3;
+                    const uint4 v = lds_u32x4(U.pay + i * 64 + q * 16);
+                    part += dot8_quarter(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
+                }
+                red_shared(ys + 4 * lds_u8(U.row + i), half_bits(lds_u16(U.sc + 2 * i)) * part);
             }
-            part += __shfl_xor_sync(0xffffffffu, part, 16);
-            if (i < n2 && lane < 16)
-                red_shared(ys + 4 * lds_u8(row + i), (half_bits(lds_u16(sc + 2 * i)) * 0x1p100f) * part);
-        } else if (t < t48) {                           // 8-bit: four lanes per group, one quarter each
-            const uint32_t pay = sblob + (h0.w >> 16) * 16, sc = sblob + (h1.y >> 16) * 16;
-            const uint32_t row = sblob + (h1.w >> 16) * 16;
-            // lane 8k + e takes quarter ((e >> 1) + k) % 4 of group e: a quarter-warp
-            // reads 8 distinct 16-byte bank groups
-            const int e = lane & 7, q = ((e >> 1) + (lane >> 3)) & 3;
-            const int i0 = (t - t4) * 8, i = i0 + e;
-            const int cf = col_uniform(ce[3], i0), cl = col_uniform(ce[3], min(i0 + 7, n3 - 1));
-            const int c = col_within(ce[3], cf, cl, i);
-            float part = 0.f;
-            if (i < n3) {
-                const uint4 v = lds_u32x4(pay + i * 64 + q * 16);
-                part = dot8_quarter(v, xs0 + (c * 4 + q) * XQ * 4);
-            }
-            part += __shfl_xor_sync(0xffffffffu, part, 8);
-            part += __shfl_xor_sync(0xffffffffu, part, 16);
-            if (i < n3 && lane < 8)
-                red_shared(ys + 4 * lds_u8(row + i), half_bits(lds_u16(sc + 2 * i)) * part);
-        } else if (t < t482) {                          // 2-bit: one group per lane, both planes at once
-            const uint32_t pay = sblob + (h0.z >> 16) * 16, sc = sblob + (h1.x >> 16) * 16;
-            const uint32_t row = sblob + (h1.z >> 16) * 16;
-            const int i0 = (t - t48) * 32, i = i0 + lane;
-            const int cf = col_uniform(ce[1], i0), cl = col_uniform(ce[1], min(i0 + 31, n1 - 1));
-            const int c = col_within(ce[1], cf, cl, i);
-            if (i < n1) {
-                const uint4 pl = lds_u32x4(pay + i * 16);
-                const uint32_t tb = lut0 + c * LUT_COL_BYTES;
+        } else if constexpr (W == 1) {
+            // 2-bit: one group per lane, both planes at once
+            const int i = i0 + lane;
+            const int c = task_column(U.ce, i0, SPAN, U.n, i);
+            if (i < U.n) {
+                const uint4 pl = lds_u32x4(U.pay + i * 16);
+                const uint32_t tb = smem_u32(T.lut) + c * LUT_COL_BYTES;
                 float va[16], vb[16];
                 plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
                 plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
                 const float2 sp = tree16x2(va, vb);
-                red_shared(ys + 4 * lds_u8(row + i),
-                           half_bits(lds_u16(sc + 2 * i)) * (sp.x + 2.f * (sp.y - lds_f32r(xlut0 + 4 * c))));
+                red_shared(ys + 4 * lds_u8(U.row + i),
+                           half_bits(lds_u16(U.sc + 2 * i)) * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))));
             }
-        } else {                                        // 1-bit: two groups per lane, summed as a pair
-            const uint32_t pay = sblob + (h0.z & 0xFFFF) * 16, sc = sblob + (h1.x & 0xFFFF) * 16;
-            const uint32_t row = sblob + (h1.z & 0xFFFF) * 16;
-            const int i0 = (t - t482) * 64, i = i0 + 2 * lane;
-            const int cf = col_uniform(ce[0], i0), cl = col_uniform(ce[0], min(i0 + 63, n0 - 1));
+        } else {
+            // 1-bit: two groups per lane, summed as a pair
+            const int i = i0 + 2 * lane;
+            const int cf = col_uniform(U.ce, i0), cl = col_uniform(U.ce, min(i0 + SPAN - 1, U.n - 1));
             int ca = cf, cb = cf;
             if (cf != cl) {
-                ca = col_within(ce[0], cf, cl, i);
-                cb = col_within(ce[0], cf, cl, min(i + 1, n0 - 1));
+                ca = col_within(U.ce, cf, cl, i);
+                cb = col_within(U.ce, cf, cl, min(i + 1, U.n - 1));
             }
-            if (i < n0) {
-                const bool two = i + 1 < n0;
-                const uint4 v = lds_u32x4(pay + i * 8);
-                const uint32_t rows2 = lds_u16(row + i);
-                const uint32_t sc2 = lds_u32(sc + 2 * i);
+            if (i < U.n) {
+                const bool two = i + 1 < U.n;
+                const uint4 v = lds_u32x4(U.pay + i * 8);
+                const uint32_t rows2 = lds_u16(U.row + i);
+                const uint32_t sc2 = lds_u32(U.sc + 2 * i);
                 float va[16], vb[16];
-                plane_entries(lut0 + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
-                plane_entries(lut0 + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
+                plane_entries(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
+                plane_entries(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
                 const float2 sp = tree16x2(va, vb);
+                const uint32_t xl = smem_u32(T.xlut);
                 if (two)
-                    red_shared(ys + 4 * (rows2 >> 8), half_bits(sc2 >> 16) * (2.f * sp.y - lds_f32r(xlut0 + 4 * cb)));
-                red_shared(ys + 4 * (rows2 & 0xff), half_bits(sc2) * (2.f * sp.x - lds_f32r(xlut0 + 4 * ca)));
+                    red_shared(ys + 4 * (rows2 >> 8), half_bits(sc2 >> 16) * (2.f * sp.y - lds_f32r(xl + 4 * cb)));
+                red_shared(ys + 4 * (rows2 & 0xff), half_bits(sc2) * (2.f * sp.x - lds_f32r(xl + 4 * ca)));
             }
         }
+    }
+}
+
+// One consumer warp's share of a unit (blob at shared address sblob, cols
+// group columns). The unit's tasks are numbered 8-bit, 4-bit, 2-bit, 1-bit
+// (costliest first); this warp takes tasks t0, t0 + tstep, ... of that
+// sequence. Partials go to the row partials at shared address ys by
+// shared-memory reductions.
+__device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, int C, int cols, uint32_t ys,
+                                             int t0, int tstep, int lane) {
+    // UnitHeader fields, read as three 16-byte words
+    const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
+    const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
+    const int n[4] = {(int)(h0.x & 0xFFFF), (int)(h0.x >> 16), (int)(h0.y & 0xFFFF), (int)(h0.y >> 16)};
+    const uint32_t pay16[4] = {h0.z & 0xFFFF, h0.z >> 16, h0.w & 0xFFFF, h0.w >> 16};
+    const uint32_t sc16[4] = {h1.x & 0xFFFF, h1.x >> 16, h1.y & 0xFFFF, h1.y >> 16};
+    const uint32_t row16[4] = {h1.z & 0xFFFF, h1.z >> 16, h1.w & 0xFFFF, h1.w >> 16};
+    auto view = [&](int w) {
+        UnitView U;
+        U.pay = sblob + pay16[w] * 16;
+        U.sc = sblob + sc16[w] * 16;
+        U.row = sblob + row16[w] * 16;
+        U.ce = lane < cols ? lds_u16(cc + 2 * (w * C + lane)) : 0xFFFFu;
+        U.n = n[w];
+        return U;
+    };
+    // first task of each width for this warp: the width's tasks start at base b
+    // in the unit's sequence; this warp's next index at or after b is
+    // b + ((t0 - b) mod tstep)
+    int base = 0;
+    auto first = [&](int nt) {
+        int f = (t0 - base) % tstep;
+        if (f < 0) f += tstep;
+        base += nt;
+        return f;
+    };
+    {
+        const UnitView U = view(3);
+        run_width<3>(T, U, ys, first((U.n + 31) >> 5), tstep, lane);
+    }
+    {
+        const UnitView U = view(2);
+        run_width<2>(T, U, ys, first((U.n + 31) >> 5), tstep, lane);
+    }
+    {
+        const UnitView U = view(1);
+        run_width<1>(T, U, ys, first((U.n + 31) >> 5), tstep, lane);
+    }
+    {
+        const UnitView U = view(0);
+        run_width<0>(T, U, ys, first((U.n + 63) >> 6), tstep, lane);
     }
 }
 
@@ -480,7 +529,8 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
                 // tasks rotate over the team's warps from unit to unit, so no warp always draws the costly ones
-                const int t0 = (wt - (j >> lg_teams)) & (tw - 1);
+                int t0 = wt - (j >> lg_teams) % tw;
+                if (t0 < 0) t0 += tw;
                 consume_unit(T, stage0 + st * STAGE_BYTES, L.C, min(L.C, L.G - sj * L.C), smem_u32(T.ys[st]), t0,
                              tw, lane);
                 __syncwarp();

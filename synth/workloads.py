@@ -5,6 +5,12 @@ Table 2: a ~131M TinyStories decoder, ~1B and ~9B models) as plain linear
 stacks: per layer Q, K, V, O, gate, up, down, then the LM head. W is stored
 N x K (output features x input features); groups of 64 run along K.
 
+The "-fused" stacks hold the same projections with the ones that read the
+same input stacked into one matrix, as a decode step issues them: Q, K and V
+as one QKV matrix, gate and up as one matrix (4 products per layer instead of
+7). Their weights are drawn per fused matrix (same shapes, same
+distributions, their own seeds); O and down keep the per-projection seeds.
+
 Bit-width distributions are probabilities over widths (1, 2, 4, 8):
   * main:  the adaptive-search allocation of §5.1 (most groups at 1 bit),
            p = (0.69, 0.15, 0.11, 0.05), mean 1.83 bits;
@@ -58,23 +64,40 @@ class Workload:
 
 
 def _stack(config_id: int, d_model: int, n_layers: int, d_q: int, d_kv: int,
-           d_ff: int, vocab: int) -> List[MatrixSpec]:
+           d_ff: int, vocab: int, fused: bool = False) -> List[MatrixSpec]:
     mats: List[MatrixSpec] = []
     for layer in range(n_layers):
         mlp = DIST_MLP0 if layer == 0 else DIST_MAIN
-        projs = [
-            ("q", d_q, d_model, DIST_MAIN),
-            ("k", d_kv, d_model, DIST_MAIN),
-            ("v", d_kv, d_model, DIST_MAIN),
-            ("o", d_model, d_q, DIST_MAIN),
-            ("gate", d_ff, d_model, mlp),
-            ("up", d_ff, d_model, mlp),
-            ("down", d_model, d_ff, mlp),
-        ]
-        for pid, (pname, n, k, dist) in enumerate(projs):
+        # (name, n, k, dist, proj_id)
+        if fused:
+            projs = [
+                ("qkv", d_q + 2 * d_kv, d_model, DIST_MAIN, 7),
+                ("o", d_model, d_q, DIST_MAIN, 3),
+                ("gate_up", 2 * d_ff, d_model, mlp, 8),
+                ("down", d_model, d_ff, mlp, 6),
+            ]
+        else:
+            projs = [
+                ("q", d_q, d_model, DIST_MAIN, 0),
+                ("k", d_kv, d_model, DIST_MAIN, 1),
+                ("v", d_kv, d_model, DIST_MAIN, 2),
+                ("o", d_model, d_q, DIST_MAIN, 3),
+                ("gate", d_ff, d_model, mlp, 4),
+                ("up", d_ff, d_model, mlp, 5),
+                ("down", d_model, d_ff, mlp, 6),
+            ]
+        for pname, n, k, dist, pid in projs:
             mats.append(MatrixSpec(f"l{layer}.{pname}", n, k, dist, (config_id, layer, pid)))
     mats.append(MatrixSpec("head", vocab, d_model, DIST_HEAD, (config_id, n_layers, 0)))
     return mats
+
+
+# name -> (config_id, (d_model, n_layers, d_q, d_kv, d_ff, vocab))
+_STACKS = {
+    "stack131m": (1, (768, 12, 768, 768, 2048, 32000)),
+    "stack1b": (2, (2048, 22, 2048, 256, 5632, 32000)),
+    "stack9b": (3, (4096, 32, 4096, 1024, 14336, 128256)),
+}
 
 
 def workload(name: str, batch: int = 1) -> Workload:
@@ -84,17 +107,18 @@ def workload(name: str, batch: int = 1) -> Workload:
     stack131m   d_model 768, 12 layers, MLP 2048, head 32000 (85 GEMVs).
     stack1b     d_model 2048, 22 layers, Q/O 2048, K/V 256, MLP 5632, head 32000 (155 GEMVs).
     stack9b     d_model 4096, 32 layers, Q/O 4096, K/V 1024, MLP 14336, head 128256 (225 GEMVs).
+    <stack>-fused   the same stack with QKV and gate-up fused (131m: 49, 1b: 89, 9b: 129 GEMVs).
     sweep:<n>:<dist>  one n x n GEMV, dist in all1/all2/all4/all8/mixed.
     matrix:<n>:<k>:<dist>  one n x k GEMV (for profiling single shapes).
     """
+    if name.endswith("-fused") and name[:-6] in _STACKS:
+        cid, dims = _STACKS[name[:-6]]
+        return Workload(name, cid, batch, _stack(cid, *dims, fused=True))
+    if name in _STACKS:
+        cid, dims = _STACKS[name]
+        return Workload(name, cid, batch, _stack(cid, *dims))
     if name == "single768":
         return Workload(name, 0, batch, [MatrixSpec("w", 768, 768, DIST_MAIN, (0, 0, 0))])
-    if name == "stack131m":
-        return Workload(name, 1, batch, _stack(1, 768, 12, 768, 768, 2048, 32000))
-    if name == "stack1b":
-        return Workload(name, 2, batch, _stack(2, 2048, 22, 2048, 256, 5632, 32000))
-    if name == "stack9b":
-        return Workload(name, 3, batch, _stack(3, 4096, 32, 4096, 1024, 14336, 128256))
     if name.startswith("matrix:"):
         # matrix:N:K:dist, dist in main / mlp0 / head / all1 / all2 / all4 / all8
         _, n, k, dist = name.split(":")

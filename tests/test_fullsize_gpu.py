@@ -48,7 +48,8 @@ def _pack(spec, inp):
     return lay
 
 
-@pytest.mark.parametrize("name", ["single768", "stack131m", "stack1b", "stack9b"])
+@pytest.mark.parametrize("name", ["single768", "stack131m", "stack1b", "stack9b",
+                                  "stack131m-fused", "stack1b-fused", "stack9b-fused"])
 def test_stack_fullsize_sampled(name):
     work = synth.workload(name, 1)
     rng = np.random.default_rng(7)

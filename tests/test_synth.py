@@ -53,6 +53,24 @@ def test_stack_shapes():
         assert m.k % 64 == 0
 
 
+@pytest.mark.parametrize("name,layers", [("stack131m", 12), ("stack1b", 22), ("stack9b", 32)])
+def test_fused_stack_shapes(name, layers):
+    # same weights as the per-projection stack, 4 products per layer + the head
+    a, b = synth.workload(name), synth.workload(name + "-fused")
+    assert len(b.mats) == 4 * layers + 1 and b.weights == a.weights
+    per = {m.name: m for m in a.mats}
+    for m in b.mats:
+        layer, _, proj = m.name.rpartition(".")
+        if proj == "qkv":
+            parts = [per[f"{layer}.{p}"] for p in ("q", "k", "v")]
+        elif proj == "gate_up":
+            parts = [per[f"{layer}.{p}"] for p in ("gate", "up")]
+        else:
+            parts = [per[m.name]]
+            assert m.seed_path == parts[0].seed_path
+        assert m.n == sum(p.n for p in parts) and all(p.k == m.k and p.dist == m.dist for p in parts)
+
+
 def test_fmix32_tensor_matches_reference():
     # the int64-tensor formulation must equal the plain 32-bit definition
     key = gen.code_key((9, 9, 9))
