@@ -46,7 +46,7 @@ constexpr int GROUP = 64;        // weights per group (§3.1)
 constexpr int MAX_C = 16;        // max group columns per slab
 constexpr int MAX_BATCH = 16;
 constexpr int MAX_UNIT_ITEMS = RB * MAX_C;
-constexpr uint32_t MAX_BLOB_BYTES = 42 * 1024;   // a unit blob fits one shared-memory stage
+constexpr uint32_t MAX_BLOB_BYTES = 41 * 1024;   // a unit blob fits one shared-memory stage
 
 struct UnitHeader {
     uint16_t n[4];        // items per width index

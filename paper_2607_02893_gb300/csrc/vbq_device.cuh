@@ -24,6 +24,12 @@ __device__ __forceinline__ float lds_f32(uint32_t addr) {
     return v;
 }
 
+__device__ __forceinline__ void sts_f32(uint32_t addr, float v) {
+    asm volatile("st.shared.f32 [%0], %1;" :: "r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void sts_zero4(uint32_t addr) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" :: "r"(addr), "r"(0u) : "memory");
+}
 __device__ __forceinline__ float4 lds_f32x4(uint32_t addr) {
     float4 v;
     asm("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"

@@ -49,7 +49,7 @@ namespace {
 constexpr int NCW = 16;                  // consumer warps of the batch-1 kernel
 constexpr int NCT = 32 * NCW;            // consumer threads
 constexpr int MAX_TEAMS = 4;             // consumer teams (1, 2 or 4 by units per block); unit j goes to team j % teams
-static_assert(MAX_TEAMS == 4 && NCW % MAX_TEAMS == 0, "every team count splits the consumer warps evenly");
+static_assert(MAX_TEAMS == 4 && NCW == 16, "teams of 16, 8 or 4 warps: task steps are powers of two (masks, no division)");
 // Unit j uses stage j % NSTAGE and goes to team j % teams; with NSTAGE a
 // multiple of every team count, each stage serves one team only, and that team
 // waits the stage's phases in order (a parity wait never skips a phase).
@@ -70,14 +70,15 @@ struct __align__(16) Tables {
     float x4s[MAX_C * 2 * XH];           // x pre-scaled per 4-bit nibble slot (see dot4_half); half (c, h) at (c*2 + h) * XH
     float2 x4z[MAX_C][2];                // per column and half: sums of x * 2^-100, even / odd codes
     float xlut[MAX_C];                   // per column: sum of the all-ones entries, in lookup order
-    float ys[NSTAGE][RB];                // row partials of the unit in each stage
+    float slots[NSTAGE][RB * MAX_C];     // per stage: one value per (row, column) of the unit (see slot_addr)
     unsigned long long full[NSTAGE];     // blob landed (TMA transaction count)
     unsigned long long empty[NSTAGE];    // the unit's team is done (one arrival per team warp)
     int abort;                           // set by any role whose wait ran out
 };
 static_assert(offsetof(Tables, full) % 8 == 0, "mbarriers are 8-byte aligned");
 static_assert(offsetof(Tables, lut) == 0, "tables start at the aligned base");
-static_assert(offsetof(Tables, x4z) % 16 == 0 && offsetof(Tables, xs) % 16 == 0 && offsetof(Tables, x4s) % 16 == 0,
+static_assert(offsetof(Tables, x4z) % 16 == 0 && offsetof(Tables, xs) % 16 == 0 && offsetof(Tables, x4s) % 16 == 0 &&
+              offsetof(Tables, slots) % 16 == 0,
               "16-byte table reads");
 static_assert(RB % 32 == 0, "the copier flushes rows a warp at a time");
 static_assert(MAX_C <= 32, "a warp holds a unit's column ends one per lane");
@@ -94,6 +95,17 @@ static_assert(GEMV1_SMEM <= 227 * 1024, "one block per SM");
 // byte permute then merges one such byte with the upper bytes of tb, so every
 // lookup address costs one instruction.
 __device__ __forceinline__ uint32_t col_shift4(int c) { return (uint32_t)(c & 1) * 0x40404040u; }
+
+// Every (row, column) of a unit holds exactly one group, so each group's
+// scaled dot product has a slot of its own and is stored, not added: no
+// shared-memory atomics, and the row sums are taken later in a fixed order.
+// Row r's 16 slots are 64 contiguous bytes; column c sits at position
+// c ^ ((r >> 1) & 15), so a warp storing one column for up to 32 consecutive
+// rows touches 32 distinct banks.
+static_assert(MAX_C == 16, "16 slots per row");
+__device__ __forceinline__ uint32_t slot_addr(uint32_t slots, uint32_t r, int c) {
+    return slots + (r << 6) + (((uint32_t)c ^ ((r >> 1) & 15u)) << 2);
+}
 __device__ __forceinline__ void plane_entries(uint32_t tb, uint32_t sh4, uint32_t lo, uint32_t hi, float (&v)[16]) {
     const uint32_t M = 0x3C3C3C3Cu;
     const uint32_t le = ((lo << 2) & M) | sh4, lo_ = ((lo >> 2) & M) | sh4;
@@ -265,7 +277,7 @@ __device__ __forceinline__ int task_column(uint32_t ce, int i0, int span, int n,
 // k = first, first + tstep, ... of this width's nt tasks. Every lane holds
 // whole groups, so a task's bookkeeping is shared by 32 groups.
 template <int W>
-__device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, uint32_t ys, int first, int tstep,
+__device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, uint32_t slots, int first, int tstep,
                                           int lane) {
     constexpr int SPAN = W == 0 ? 64 : 32;
     const int nt = (U.n + SPAN - 1) / SPAN;
@@ -283,7 +295,7 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
                 const float2 aa = dot4_half(va, xa), ab = dot4_half(vb, xb);
                 const float4 z = lds_f32x4(smem_u32(T.x4z) + c * 16);     // (even, odd) of half 0, then of half 1
                 const float part = ((aa.x + ab.x) - 8.f * (z.x + z.z)) + ((aa.y + ab.y) - 8.f * (z.y + z.w));
-                red_shared(ys + 4 * lds_u8(U.row + i), (half_bits(lds_u16(U.sc + 2 * i)) * 0x1p100f) * part);
+                sts_f32(slot_addr(slots, lds_u8(U.row + i), c), (half_bits(lds_u16(U.sc + 2 * i)) * 0x1p100f) * part);
             }
         } else if constexpr (W == 3) {
             // 8-bit: one group per lane, quarter (k + (lane >> 1)) & 3 in step k
@@ -299,7 +311,7 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
                     const uint4 v = lds_u32x4(U.pay + i * 64 + q * 16);
                     part += dot8_quarter(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
                 }
-                red_shared(ys + 4 * lds_u8(U.row + i), half_bits(lds_u16(U.sc + 2 * i)) * part);
+                sts_f32(slot_addr(slots, lds_u8(U.row + i), c), half_bits(lds_u16(U.sc + 2 * i)) * part);
             }
         } else if constexpr (W == 1) {
             // 2-bit: one group per lane, both planes at once
@@ -312,8 +324,8 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
                 plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
                 plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
                 const float2 sp = tree16x2(va, vb);
-                red_shared(ys + 4 * lds_u8(U.row + i),
-                           half_bits(lds_u16(U.sc + 2 * i)) * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))));
+                sts_f32(slot_addr(slots, lds_u8(U.row + i), c),
+                        half_bits(lds_u16(U.sc + 2 * i)) * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))));
             }
         } else {
             // 1-bit: two groups per lane, summed as a pair
@@ -335,8 +347,8 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
                 const float2 sp = tree16x2(va, vb);
                 const uint32_t xl = smem_u32(T.xlut);
                 if (two)
-                    red_shared(ys + 4 * (rows2 >> 8), half_bits(sc2 >> 16) * (2.f * sp.y - lds_f32r(xl + 4 * cb)));
-                red_shared(ys + 4 * (rows2 & 0xff), half_bits(sc2) * (2.f * sp.x - lds_f32r(xl + 4 * ca)));
+                    sts_f32(slot_addr(slots, rows2 >> 8, cb), half_bits(sc2 >> 16) * (2.f * sp.y - lds_f32r(xl + 4 * cb)));
+                sts_f32(slot_addr(slots, rows2 & 0xff, ca), half_bits(sc2) * (2.f * sp.x - lds_f32r(xl + 4 * ca)));
             }
         }
     }
@@ -345,9 +357,9 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
 // One consumer warp's share of a unit (blob at shared address sblob, cols
 // group columns). The unit's tasks are numbered 8-bit, 4-bit, 2-bit, 1-bit
 // (costliest first); this warp takes tasks t0, t0 + tstep, ... of that
-// sequence. Partials go to the row partials at shared address ys by
-// shared-memory reductions.
-__device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, int C, int cols, uint32_t ys,
+// sequence (tstep a power of two). Each group's result goes to its slot in
+// the stage's slot array at shared address slots.
+__device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, int C, int cols, uint32_t slots,
                                              int t0, int tstep, int lane) {
     // UnitHeader fields, read as three 16-byte words
     const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
@@ -367,30 +379,13 @@ __device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, in
     };
     // first task of each width for this warp: the width's tasks start at base b
     // in the unit's sequence; this warp's next index at or after b is
-    // b + ((t0 - b) mod tstep)
-    int base = 0;
-    auto first = [&](int nt) {
-        int f = (t0 - base) % tstep;
-        if (f < 0) f += tstep;
-        base += nt;
-        return f;
-    };
-    {
-        const UnitView U = view(3);
-        run_width<3>(T, U, ys, first((U.n + 31) >> 5), tstep, lane);
-    }
-    {
-        const UnitView U = view(2);
-        run_width<2>(T, U, ys, first((U.n + 31) >> 5), tstep, lane);
-    }
-    {
-        const UnitView U = view(1);
-        run_width<1>(T, U, ys, first((U.n + 31) >> 5), tstep, lane);
-    }
-    {
-        const UnitView U = view(0);
-        run_width<0>(T, U, ys, first((U.n + 63) >> 6), tstep, lane);
-    }
+    // b + ((t0 - b) mod tstep), tstep a power of two
+    const int nt3 = (n[3] + 31) >> 5, nt2 = (n[2] + 31) >> 5, nt1 = (n[1] + 31) >> 5;
+    const int m = tstep - 1;
+    if (n[3]) run_width<3>(T, view(3), slots, t0 & m, tstep, lane);
+    if (n[2]) run_width<2>(T, view(2), slots, (t0 - nt3) & m, tstep, lane);
+    if (n[1]) run_width<1>(T, view(1), slots, (t0 - nt3 - nt2) & m, tstep, lane);
+    if (n[0]) run_width<0>(T, view(0), slots, (t0 - nt3 - nt2 - nt1) & m, tstep, lane);
 }
 
 __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
@@ -423,7 +418,9 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         T.abort = 0;
         fence_barrier_init();
     }
-    for (int i = tid; i < NSTAGE * RB; i += G1_THREADS) (&T.ys[0][0])[i] = 0.f;
+    // slots no group of a unit writes (rows past N, columns past the last
+    // slab's) must read as zero; the copier re-zeroes every slot it sums
+    for (int i = tid; i < NSTAGE * RB * MAX_C; i += G1_THREADS) (&T.slots[0][0])[i] = 0.f;
     __syncthreads();
     if (tid == 0) {
         const int first = n_units < NSTAGE ? n_units : NSTAGE;
@@ -471,14 +468,23 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         for (int j = 0; j < n_units; ++j) {
             if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 256)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
-                float* ys = T.ys[st];
+                const uint32_t sl = smem_u32(T.slots[st]);
                 const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
                 float* yr = y + (int64_t)rbw * RB;
 #pragma unroll
                 for (int q = 0; q < RB / 32; ++q) {
+                    // row r's 16 slots as four 16-byte chunks, chunk (k + (lane >> 1)) & 3
+                    // at step k (each quarter-warp touches 8 distinct bank groups);
+                    // summed as a tree, then zeroed for the stage's next unit
                     const int r = lane + 32 * q;
-                    const float v = ys[r];
-                    ys[r] = 0.f;
+                    const uint32_t ra = sl + (uint32_t)r * 64;
+                    float4 a[4];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) a[k] = lds_f32x4(ra + (((k + (lane >> 1)) & 3) << 4));
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) sts_zero4(ra + (((k + (lane >> 1)) & 3) << 4));
+                    const float v = (((a[0].x + a[0].y) + (a[0].z + a[0].w)) + ((a[1].x + a[1].y) + (a[1].z + a[1].w))) +
+                                    (((a[2].x + a[2].y) + (a[2].z + a[2].w)) + ((a[3].x + a[3].y) + (a[3].z + a[3].w)));
                     if (r < rows) {
                         if (L.S == 1) yr[r] = v;
                         else red_global(yr + r, v);
@@ -529,9 +535,8 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
                 // tasks rotate over the team's warps from unit to unit, so no warp always draws the costly ones
-                int t0 = wt - (j >> lg_teams) % tw;
-                if (t0 < 0) t0 += tw;
-                consume_unit(T, stage0 + st * STAGE_BYTES, L.C, min(L.C, L.G - sj * L.C), smem_u32(T.ys[st]), t0,
+                const int t0 = (wt - (j >> lg_teams)) & (tw - 1);
+                consume_unit(T, stage0 + st * STAGE_BYTES, L.C, min(L.C, L.G - sj * L.C), smem_u32(T.slots[st]), t0,
                              tw, lane);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty0 + 8 * st);
