@@ -5,15 +5,15 @@
 //
 // Batch 1 (gemv1_kernel): one persistent block per SM, warp-specialised.
 //   warp 0 (copier)    streams unit blobs into NSTAGE shared-memory stages with
-//                      TMA bulk copies and, once a unit is consumed, writes its
-//                      row partials to y and starts the copy of a later unit
+//                      TMA bulk copies and, once a unit is consumed, sums its
+//                      slots per row into y and starts the copy of a later unit
 //                      into the freed stage;
-//   warps 1.. (NCW)    consumers, in 1, 2 or 4 teams (more units per block,
-//                      more teams): unit j goes to team j % teams, whose warps
-//                      split its items into warp
-//                      tasks and accumulate the group dot products into the
-//                      stage's row partials; an item's column comes from the
-//                      blob's column ends (a ballot per task, see col_uniform).
+//   warps 1.. (NCW)    consumers, in 1 or 2 teams (2 from 4 units per block
+//                      on): unit j goes to team j % teams, whose warps split
+//                      its items into warp tasks and store each group's
+//                      scaled dot product in the stage's (row, column) slot;
+//                      an item's column comes from the blob's column ends (a
+//                      ballot per task, see col_uniform).
 // The roles hand stages to one another through two mbarriers per stage
 // (full: blob landed; empty: the unit's team is done), so no block-wide
 // barrier sits in the steady state and up to NSTAGE units are in flight per SM. Block p owns a contiguous range of units in
@@ -48,15 +48,15 @@ namespace {
 
 constexpr int NCW = 16;                  // consumer warps of the batch-1 kernel
 constexpr int NCT = 32 * NCW;            // consumer threads
-constexpr int MAX_TEAMS = 4;             // consumer teams (1, 2 or 4 by units per block); unit j goes to team j % teams
-static_assert(MAX_TEAMS == 4 && NCW == 16, "teams of 16, 8 or 4 warps: task steps are powers of two (masks, no division)");
+constexpr int MAX_TEAMS = 2;             // consumer teams (1 or 2 by units per block); unit j goes to team j % teams
+static_assert(MAX_TEAMS == 2 && NCW == 16, "teams of 16 or 8 warps: task steps are powers of two (masks, no division)");
 // Unit j uses stage j % NSTAGE and goes to team j % teams; with NSTAGE a
 // multiple of every team count, each stage serves one team only, and that team
 // waits the stage's phases in order (a parity wait never skips a phase).
 constexpr int G1_THREADS = 32 * (NCW + 1);
 constexpr int NSTAGE = 4;                // blob stages in flight per SM
 static_assert((NSTAGE & (NSTAGE - 1)) == 0, "power-of-two stage count");
-static_assert(NSTAGE % 4 == 0, "every team count (1, 2, 4) divides the stage count");
+static_assert(NSTAGE % MAX_TEAMS == 0, "every team count (1, 2) divides the stage count");
 constexpr int XQ = 20;                   // floats per 16-code quarter of x (16 + 4 pad: quarters use other banks)
 constexpr int XH = 36;                   // floats per 32-code half of the pre-scaled x (32 + 4 pad)
 constexpr int LUT_COL_BYTES = 1280;      // 16 tables x 64 bytes (+64 for odd columns), columns on 256-byte boundaries
@@ -270,6 +270,7 @@ struct UnitView {
 // Column of item i (tasks hold items i0 .. i0 + span - 1; lanes agree on i0).
 __device__ __forceinline__ int task_column(uint32_t ce, int i0, int span, int n, int i) {
     const int cf = col_uniform(ce, i0), cl = col_uniform(ce, min(i0 + span - 1, n - 1));
+    if (cl == cf + 1) return cf + (i >= (int)__shfl_sync(0xffffffffu, ce, cf));   // one column end inside
     return cf == cl ? cf : col_within(ce, cf, cl, i);
 }
 
@@ -332,7 +333,11 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
             const int i = i0 + 2 * lane;
             const int cf = col_uniform(U.ce, i0), cl = col_uniform(U.ce, min(i0 + SPAN - 1, U.n - 1));
             int ca = cf, cb = cf;
-            if (cf != cl) {
+            if (cl == cf + 1) {                         // one column end inside the task
+                const int e = (int)__shfl_sync(0xffffffffu, U.ce, cf);
+                ca = cf + (i >= e);
+                cb = cf + (i + 1 >= e);
+            } else if (cf != cl) {
                 ca = col_within(U.ce, cf, cl, i);
                 cb = col_within(U.ce, cf, cl, min(i + 1, U.n - 1));
             }
@@ -405,7 +410,9 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     const int s0 = u_begin / L.nrb, rb0 = u_begin - s0 * L.nrb;
     // more units per block -> more teams: each warp then covers more groups per
     // unit (less per-unit overhead); few units -> whole-block teams (less latency)
-    const int lg_teams = n_units >= 4 * MAX_TEAMS ? 2 : n_units >= 8 ? 1 : 0;
+    // two teams once the block has 4 units: each team then has NSTAGE / 2
+    // stages, so its next blob lands while it works on the current one
+    const int lg_teams = n_units >= 4 ? 1 : 0;
     const int teams = 1 << lg_teams, tw = NCW >> lg_teams;
 
     const uint32_t full0 = smem_u32(&T.full[0]), empty0 = smem_u32(&T.empty[0]);
