@@ -130,13 +130,15 @@ vbq_status_t vbq_gemv(const vbq_layout* layout, const uint16_t* x, float* y,
  *   Y  device, B x N floats, row-major; overwritten.
  *   B  1..16 (VBQ_ERR_UNSUPPORTED otherwise).
  * Same accuracy statement as vbq_gemv; the summation order is not fixed (results
- * can differ in the last bits between calls). B = 1 is vbq_gemv. For B >= 2 the
- * product runs on the tensor cores: activations are scaled per (row, group
- * column) by a power of two into fp16 range (values below 2^-14 of that
- * scale lose low bits), weights enter as exact levels, products and fp32
- * accumulation as in vbq_gemv. Y needs no zeroing; the same split-K workspace
- * and ordering rules as vbq_gemv apply (calls sharing a layout must not
- * overlap on the GPU), and the kernel is launched the same way.
+ * can differ in the last bits between calls). For B <= 3 each row is one
+ * vbq_gemv product (B launches of the batch-1 kernel, which is faster than
+ * the batched kernel there). For B >= 4 the product runs on the tensor cores:
+ * activations are scaled per (row, group column) by a power of two into fp16
+ * range (values below 2^-14 of that scale lose low bits), weights enter as
+ * exact levels, products and fp32 accumulation as in vbq_gemv. Y needs no
+ * zeroing; the same split-K workspace and ordering rules as vbq_gemv apply
+ * (calls sharing a layout must not overlap on the GPU), and the kernels are
+ * launched the same way.
  */
 vbq_status_t vbq_gemm_small(const vbq_layout* layout, const uint16_t* X, float* Y,
                             int B, void* stream);

@@ -42,10 +42,13 @@ constexpr int NCWB = 16;                 // consumer warps
 constexpr int NCTB = 32 * NCWB;
 constexpr int GB_THREADS = 32 * (NCWB + 1);
 constexpr int STAGE_BYTES_B = MAX_BLOB_BYTES;
+// Row partials of one batch row take RB + 1 floats, so the same row of eight
+// batch rows (the eight lane groups of an epilogue store) falls in eight banks.
+constexpr int YS_STRIDE = RB + 1;
 // Stages and consumer teams: with NB = 8 A rows the tables leave room for four
-// stages, so up to four teams (each team's units then use stages of their
-// own); NB = 16 fits three stages and one team.
-template <int NB> struct Pipe { static constexpr int stages = NB == 8 ? 4 : 3, max_teams = NB == 8 ? 4 : 1; };
+// stages, so up to two teams of two stages each (a team's next blob lands
+// while it works on the current one); NB = 16 fits three stages and one team.
+template <int NB> struct Pipe { static constexpr int stages = NB == 8 ? 4 : 3, max_teams = NB == 8 ? 2 : 1; };
 static_assert(Pipe<8>::stages % Pipe<8>::max_teams == 0 && Pipe<16>::stages % Pipe<16>::max_teams == 0,
               "each team's units use stages no other team uses");
 static_assert(STAGE_BYTES_B % 256 == 0, "stage alignment");
@@ -55,7 +58,7 @@ template <int NB>
 struct __align__(16) TablesB {
     uint32_t afr[MAX_C][32][NB];         // A fragments (fp16x2) per column and lane: NB/4 per k-step
     float e2[MAX_C][16];                 // per column and batch row: 2^E (0 for absent rows)
-    float ys[Pipe<NB>::stages][NB][RB];            // row partials of each stage, per batch row
+    float ys[Pipe<NB>::stages][NB][YS_STRIDE];     // row partials of each stage, per batch row
     unsigned long long full[Pipe<NB>::stages];     // blob landed
     unsigned long long empty[Pipe<NB>::stages];    // the unit's team is done
     int abort;
@@ -194,7 +197,7 @@ __device__ __forceinline__ void to_levels(uint32_t (&b)[8]) {
 // Tiles k0 .. k1-1 of one (column, width W) bucket: items bs + 8k .. of the
 // bucket [bs, be); pay / scb / rwb: the width's payload, scales and row bytes.
 template <int NB, int W>
-__device__ __forceinline__ void run_tiles(const uint32_t (&a)[NB], float e2g, float e2g8, uint32_t pay, uint32_t scb,
+__device__ __forceinline__ void run_tiles(const uint32_t (&A4)[4][4], float e2g, float e2g8, uint32_t pay, uint32_t scb,
                                           uint32_t rwb, int bs, int be, int k0, int k1, uint32_t ys, int B, int g,
                                           int t) {
     for (int k = k0; k < k1; ++k) {
@@ -211,22 +214,17 @@ __device__ __forceinline__ void run_tiles(const uint32_t (&a)[NB], float e2g, fl
         const int ra = lds_u8(rwb + ia), rb = lds_u8(rwb + ib);
         to_levels<W>(b);
         float d[4];
+        mma16816_z(d, A4[0], b[0], b[1]);
 #pragma unroll
-        for (int s2 = 0; s2 < 4; ++s2) {
-            uint32_t af[4];
-            if (NB == 16) { af[0] = a[4 * s2]; af[1] = a[4 * s2 + 1]; af[2] = a[4 * s2 + 2]; af[3] = a[4 * s2 + 3]; }
-            else { af[0] = a[2 * s2]; af[1] = 0u; af[2] = a[(2 * s2 + 1) % NB]; af[3] = 0u; }
-            if (s2 == 0) mma16816_z(d, af, b[0], b[1]);
-            else mma16816(d, af, b[2 * s2], b[2 * s2 + 1]);
-        }
+        for (int s2 = 1; s2 < 4; ++s2) mma16816(d, A4[s2], b[2 * s2], b[2 * s2 + 1]);
         // items 2t and 2t+1: scaled, added to the row partials of batch rows g and g + 8
         if (g < B) {
-            if (2 * t < nv) red_shared(ys + 4 * (g * RB + ra), d[0] * (sa * e2g));
-            if (2 * t + 1 < nv) red_shared(ys + 4 * (g * RB + rb), d[1] * (sb * e2g));
+            if (2 * t < nv) red_shared(ys + 4 * (g * YS_STRIDE + ra), d[0] * (sa * e2g));
+            if (2 * t + 1 < nv) red_shared(ys + 4 * (g * YS_STRIDE + rb), d[1] * (sb * e2g));
         }
         if (NB == 16 && g + 8 < B) {
-            if (2 * t < nv) red_shared(ys + 4 * ((g + 8) * RB + ra), d[2] * (sa * e2g8));
-            if (2 * t + 1 < nv) red_shared(ys + 4 * ((g + 8) * RB + rb), d[3] * (sb * e2g8));
+            if (2 * t < nv) red_shared(ys + 4 * ((g + 8) * YS_STRIDE + ra), d[2] * (sa * e2g8));
+            if (2 * t + 1 < nv) red_shared(ys + 4 * ((g + 8) * YS_STRIDE + rb), d[3] * (sb * e2g8));
         }
     }
 }
@@ -259,7 +257,8 @@ __device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sb
         if (lane >= o) incl += v;
     }
     const int total = __shfl_sync(0xffffffffu, incl, 31);
-    const int ta = (total * wt) / tw, tb = (total * (wt + 1)) / tw;
+    const int lg_tw = __popc(tw - 1);                  // tw is a power of two
+    const int ta = (total * wt) >> lg_tw, tb = (total * (wt + 1)) >> lg_tw;
     if (ta >= tb) return;
     const uint32_t pay[4] = {sblob + (h0.z & 0xFFFF) * 16, sblob + (h0.z >> 16) * 16, sblob + (h0.w & 0xFFFF) * 16,
                              sblob + (h0.w >> 16) * 16};
@@ -280,6 +279,14 @@ __device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sb
                 a[r] = v.x; a[r + 1] = v.y; a[r + 2] = v.z; a[r + 3] = v.w;
             }
         }
+        // the column's A operands, one register quad per k-step (NB = 8: rows
+        // 8..15 of the m16 shape are zero), set once for all of its tiles
+        uint32_t A4[4][4];
+#pragma unroll
+        for (int s2 = 0; s2 < 4; ++s2) {
+            if (NB == 16) { A4[s2][0] = a[4 * s2]; A4[s2][1] = a[4 * s2 + 1]; A4[s2][2] = a[4 * s2 + 2]; A4[s2][3] = a[4 * s2 + 3]; }
+            else { A4[s2][0] = a[2 * s2]; A4[s2][1] = 0u; A4[s2][2] = a[(2 * s2 + 1) % NB]; A4[s2][3] = 0u; }
+        }
         const float e2g = T.e2[c][g], e2g8 = T.e2[c][g + 8];
         int tile0 = c_begin;                            // global index of the bucket's first tile
 #pragma unroll
@@ -288,10 +295,10 @@ __device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sb
             const int k0 = max(ta - tile0, 0), k1 = min(tb - tile0, nt);
             if (k0 < k1) {
                 const int bs = __shfl_sync(0xffffffffu, start[w], c), be = __shfl_sync(0xffffffffu, end[w], c);
-                if (w == 0) run_tiles<NB, 0>(a, e2g, e2g8, pay[0], scb[0], rwb[0], bs, be, k0, k1, ys, B, g, t);
-                else if (w == 1) run_tiles<NB, 1>(a, e2g, e2g8, pay[1], scb[1], rwb[1], bs, be, k0, k1, ys, B, g, t);
-                else if (w == 2) run_tiles<NB, 2>(a, e2g, e2g8, pay[2], scb[2], rwb[2], bs, be, k0, k1, ys, B, g, t);
-                else run_tiles<NB, 3>(a, e2g, e2g8, pay[3], scb[3], rwb[3], bs, be, k0, k1, ys, B, g, t);
+                if (w == 0) run_tiles<NB, 0>(A4, e2g, e2g8, pay[0], scb[0], rwb[0], bs, be, k0, k1, ys, B, g, t);
+                else if (w == 1) run_tiles<NB, 1>(A4, e2g, e2g8, pay[1], scb[1], rwb[1], bs, be, k0, k1, ys, B, g, t);
+                else if (w == 2) run_tiles<NB, 2>(A4, e2g, e2g8, pay[2], scb[2], rwb[2], bs, be, k0, k1, ys, B, g, t);
+                else run_tiles<NB, 3>(A4, e2g, e2g8, pay[3], scb[3], rwb[3], bs, be, k0, k1, ys, B, g, t);
             }
             tile0 += nt;
         }
@@ -317,7 +324,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
     // stage j % stages and goes to team j % teams, and teams divides stages, so
     // each team waits the phases of its own stages in order (a parity wait that
     // skipped a phase could match an older completed one).
-    const int lg_teams = Pipe<NB>::max_teams == 4 ? (n_units >= 16 ? 2 : n_units >= 8 ? 1 : 0) : 0;
+    const int lg_teams = Pipe<NB>::max_teams == 2 && n_units >= 4 ? 1 : 0;
     const int teams = 1 << lg_teams, tw = NCWB >> lg_teams;
 
     const uint32_t full0 = smem_u32(&T.full[0]), empty0 = smem_u32(&T.empty[0]);
@@ -330,7 +337,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
         T.abort = 0;
         fence_barrier_init();
     }
-    for (int i = tid; i < NST * NB * RB; i += GB_THREADS) (&T.ys[0][0][0])[i] = 0.f;
+    for (int i = tid; i < NST * NB * YS_STRIDE; i += GB_THREADS) (&T.ys[0][0][0])[i] = 0.f;
     __syncthreads();
     if (tid == 0) {
         const int first = n_units < NST ? n_units : NST;
@@ -373,7 +380,12 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
         int st = 0, rbw = rb0, issued = n_units < NST ? n_units : NST;
         uint32_t par = 0;
         for (int j = 0; j < n_units; ++j) {
-            if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 256)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
+            // units here take microseconds: nap between polls, except on the
+            // block's last unit, whose rows end the block
+            if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, j + 1 < n_units ? 1024 : 0)) {
+                dead = true;
+                if (lane == 0) raise_abort(&T.abort);
+            }
             if (!dead) {
                 const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
                 for (int b = 0; b < B; ++b) {
@@ -423,7 +435,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
         build_tables_b(T, L, X, B, s0, ct);
         for (int j = team; j < n_units; j += teams) {
             while (cur < sj) build_tables_b(T, L, X, B, ++cur, ct);
-            const int st = j % NST;
+            const int st = j % NST;                      // NST is a compile-time constant
             const uint32_t par = (uint32_t)(j / NST) & 1u;
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {

@@ -664,8 +664,20 @@ cudaError_t launch_selftest_timeout(unsigned long long limit_ns, cudaStream_t s)
     return cudaGetLastError();
 }
 
+// Up to GEMV1_MAX_B rows run as that many batch-1 products: per row, the
+// batch-1 kernel's table lookups cost less than the batched kernel's
+// dequantisation into fragments and per-(row, group) epilogue (measured: B = 2
+// takes half the time this way, B = 3 three quarters; from B = 4 on the tensor
+// cores win).
+constexpr int GEMV1_MAX_B = 3;
+
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
-    return B <= 1 ? launch_gemv1(L, X, Y, s) : launch_gemm_small(L, X, Y, B, s);
+    if (B > GEMV1_MAX_B) return launch_gemm_small(L, X, Y, B, s);
+    for (int b = 0; b < B; ++b) {
+        const cudaError_t e = launch_gemv1(L, X + (int64_t)b * L.K, Y + (int64_t)b * L.N, s);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 }  // namespace vbq
