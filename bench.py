@@ -2,12 +2,18 @@
 
 One step = one token through every linear layer of the stack, each a packed
 VBQ GEMV run by libvbq.so on one stream, replayed from a CUDA graph. The
-default workload, stack9b-fused, issues the projections that read the same
-input as one matrix (per layer QKV, O, gate-up, down, then the LM head);
-`--workload stack9b` runs one GEMV per projection (Q, K, V, O, gate, up,
-down). Weights are random-but-seeded (synthetic) with the per-projection width
-distributions of the workload; every GEMV has its own resident BF16 activation
-vector.
+headline (default workload stack9b) is layer-serial: one GEMV per projection
+(Q, K, V, O, gate, up, down per layer, then the LM head), each launch ordered
+after the previous one. Weights are random-but-seeded (synthetic) with the
+per-projection width distributions of the workload; every GEMV has its own
+resident BF16 activation vector.
+
+`modes` reports, for a stack workload at batch 1, three companions measured in
+the same run: `fused` (the <stack>-fused workload: QKV and gate-up as single
+matrices, 4 GEMVs per layer), `grouped` (the headline's layouts as one
+vbq_gemv_group per step: independent products whose launches overlap, the
+streaming upper bound) and `cublas_bf16` (dense BF16 weights of the same
+shapes through torch.mv, i.e. cuBLAS, as a reference point).
 
 Printed JSON line (rank 0):
   value         algorithmic HBM GB/s of the whole step: sum over GEMVs of
@@ -59,9 +65,11 @@ def parse():
     p.add_argument("--steps", type=int, default=300)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--workload", default="stack9b-fused")
+    p.add_argument("--workload", default="stack9b")
     p.add_argument("--batch", type=int, default=1)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-modes", action="store_true",
+                   help="skip the fused, grouped and cuBLAS BF16 companion measurements")
     p.add_argument("--event-ring", type=int, default=4)
     return p.parse_args()
 
@@ -250,6 +258,77 @@ def setup_stack(work, batch, dev, min_bytes: int = 0):
     return layouts, xs, ys, nbytes, host_x, copies
 
 
+def time_graph(torch, stream, fn, steps: int, warmup: int) -> float:
+    """ms per replay of fn captured as one CUDA graph on stream."""
+    with torch.cuda.stream(stream):
+        fn()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        fn()
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(steps):
+            g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
+def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev, l2):
+    """The fused, grouped and cuBLAS BF16 companions of a batch-1 stack."""
+    import torch
+    import paper_2607_02893_gb300 as vbq
+    import synth
+    steps, warm = max(20, args.steps // 2), args.warmup
+    out = {}
+
+    def entry(ms, nbytes, cp, launches, note):
+        return {"ms_per_step": round(ms, 4), "value": round(nbytes / (ms * 1e-3) / 1e9, 1), "unit": "GB/s",
+                "tokens_per_s": round(cp / (ms * 1e-3), 1), "gemvs_per_step": launches, "note": note}
+
+    x0 = [x[0] for x in xs]
+    y0 = [y[0] for y in ys]
+    ms = time_graph(torch, stream, lambda: vbq.vbq_gemv_group(layouts, x0, y0, stream=stream), steps, warm)
+    out["grouped"] = entry(ms, step_bytes, copies, len(layouts),
+                           "the headline layouts as one vbq_gemv_group per step (independent products, "
+                           "overlapping launches): the streaming upper bound")
+    name = args.workload
+    if name in ("stack131m", "stack1b", "stack9b"):
+        fwork = synth.workload(name + "-fused", 1)
+        flays, fxs, fys, fnb, _, fcp = setup_stack(fwork, 1, dev, min_bytes=3 * l2)
+        ms = time_graph(torch, stream,
+                        lambda: [vbq.vbq_gemv(l, x[0], y[0], stream=stream) for l, x, y in zip(flays, fxs, fys)],
+                        steps, warm)
+        out["fused"] = entry(ms, sum(fnb), fcp, len(flays),
+                             "workload " + name + "-fused: QKV and gate-up as single matrices, layer-serial")
+        del flays, fxs, fys
+        torch.cuda.empty_cache()
+    # dense BF16 reference: the same shapes, one copy per packed copy so the
+    # weights stream from HBM too
+    g = torch.Generator(device=dev)
+    g.manual_seed(0)
+    dense, dx, dy, dbytes = [], [], [], 0
+    for _ in range(copies):
+        for spec in work.mats:
+            dense.append(torch.randn((spec.n, spec.k), generator=g, device=dev, dtype=torch.bfloat16) * 0.02)
+            dx.append(torch.randn(spec.k, generator=g, device=dev, dtype=torch.bfloat16))
+            dy.append(torch.empty(spec.n, device=dev, dtype=torch.bfloat16))
+            dbytes += 2 * spec.n * spec.k + 2 * spec.k + 2 * spec.n
+    ms = time_graph(torch, stream, lambda: [torch.mv(w, x, out=y) for w, x, y in zip(dense, dx, dy)], steps, warm)
+    out["cublas_bf16"] = entry(ms, dbytes, copies, len(dense),
+                               "dense BF16 weights of the same shapes, torch.mv (cuBLAS), layer-serial; "
+                               "value counts the BF16 weight bytes it streams")
+    del dense, dx, dy
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     import paper_2607_02893_gb300 as vbq
@@ -423,6 +502,8 @@ def run_ours(args, rank, world, local_rank):
         "gpu_launches": launches * args.steps,
         "clocks": clk,
     }
+    if B == 1 and not args.no_modes and world == 1:
+        result["modes"] = companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev, l2)
     return result, work
 
 

@@ -144,6 +144,27 @@ vbq_status_t vbq_gemm_small(const vbq_layout* layout, const uint16_t* X, float* 
                             int B, void* stream);
 
 /*
+ * vbq_gemv_group — count independent batch-1 products y_i = W_i x_i (§6
+ * product, several matrices). (The paper has no counterpart; this is an
+ * execution mode for products that do not feed one another, such as the
+ * projections of one decode step that read the same input.)
+ *   layouts, xs, ys  host arrays of count pointers: layouts, device x_i (K_i
+ *                    BF16 bit patterns), device y_i (N_i floats, overwritten).
+ *   count            >= 0; 0 does nothing.
+ * Product i runs exactly as vbq_gemv(layouts[i], xs[i], ys[i]) and satisfies
+ * its accuracy statement, but the launches overlap: launch i > 0 starts
+ * without waiting for launch i - 1 and waits for it only before completing.
+ * So no x_i may be written by another product of the same group, the layouts
+ * must be distinct and the outputs must not overlap (a repeated layout or
+ * output is VBQ_ERR_ARG; overlap of distinct output ranges is not checked).
+ * Work enqueued on the stream before the call is complete before any product
+ * reads its inputs, and work enqueued after it sees every output (it must
+ * order itself after the group's last kernel as after any kernel).
+ */
+vbq_status_t vbq_gemv_group(const vbq_layout* const* layouts, const uint16_t* const* xs, float* const* ys,
+                            int count, void* stream);
+
+/*
  * vbq_gemv_static — vbq_gemv for callers that must not allocate device memory.
  * (The paper has no counterpart; this is an operational variant.)
  *

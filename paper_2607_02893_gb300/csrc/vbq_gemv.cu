@@ -394,7 +394,7 @@ __device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, in
 }
 
 __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
-                                                              float* __restrict__ y) {
+                                                              float* __restrict__ y, int dep) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     // stages and tables on a 256-byte boundary: lookups merge a byte into table addresses
     unsigned char* base = smem_raw + ((256u - (smem_u32(smem_raw) & 255u)) & 255u);
@@ -442,8 +442,10 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         const int lines = (min(L.C, L.G - s0 * L.C) * GROUP * 2 + 127) / 128;
         if (tid >= 32 && tid - 32 < lines) prefetch_l2(x + k0 + (int64_t)(tid - 32) * 64);
     }
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    asm volatile("griddepcontrol.wait;" ::: "memory");
+    // Ordering against the previous kernel on the stream (see Dep):
+    if (dep != DEP_GROUP_FIRST) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    if (dep != DEP_GROUP_NEXT) asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (dep == DEP_GROUP_FIRST) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (warp == 0) {
         // ---- copier: split-K zeroing, then per unit: rows out, next copy in ----
@@ -524,6 +526,9 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                 st_volatile(L.ctl, epoch);
             }
         }
+        // a grouped product that started without waiting completes only after
+        // its predecessor, so completion stays in stream order
+        if (dep == DEP_GROUP_NEXT && lane == 0) asm volatile("griddepcontrol.wait;" ::: "memory");
     } else {
         // ---- consumers: team `team` takes units j = team, team + teams, ... ----
         const int cw = warp - 1, ct = tid - 32, team = cw / tw, wt = cw - team * tw;
@@ -557,7 +562,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
 
 int g_sms = 0;
 
-cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s) {
+cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s, int dep) {
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(gemv1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -579,7 +584,7 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, gemv1_kernel, L, x, y);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, gemv1_kernel, L, x, y, dep);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -619,7 +624,7 @@ cudaError_t launch_gemv1_static(const LayoutView& L, const uint16_t* x, float* y
     if ((e = cudaMemsetAsync(ctl + 1, 0, sizeof(uint32_t), s)) != cudaSuccess) return e;
     LayoutView Ls = L;
     Ls.ctl = ctl;
-    return launch_gemv1(Ls, x, y, s);
+    return launch_gemv1(Ls, x, y, s, DEP_BEFORE);
 }
 
 // ---------------------------------------------------------------------------
@@ -671,10 +676,20 @@ cudaError_t launch_selftest_timeout(unsigned long long limit_ns, cudaStream_t s)
 // cores win).
 constexpr int GEMV1_MAX_B = 3;
 
+cudaError_t launch_gemv_group(const LayoutView* const* Ls, const uint16_t* const* xs, float* const* ys, int count,
+                              cudaStream_t s) {
+    for (int i = 0; i < count; ++i) {
+        const int dep = count == 1 ? DEP_BEFORE : i == 0 ? DEP_GROUP_FIRST : DEP_GROUP_NEXT;
+        const cudaError_t e = launch_gemv1(*Ls[i], xs[i], ys[i], s, dep);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
     if (B > GEMV1_MAX_B) return launch_gemm_small(L, X, Y, B, s);
     for (int b = 0; b < B; ++b) {
-        const cudaError_t e = launch_gemv1(L, X + (int64_t)b * L.K, Y + (int64_t)b * L.N, s);
+        const cudaError_t e = launch_gemv1(L, X + (int64_t)b * L.K, Y + (int64_t)b * L.N, s, DEP_BEFORE);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

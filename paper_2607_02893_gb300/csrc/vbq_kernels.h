@@ -18,9 +18,26 @@ cudaError_t launch_scatter(const uint8_t* codes, const uint8_t* widths, const ui
 cudaError_t launch_dequant(const LayoutView& L, uint8_t* codes_out, uint8_t* widths_out,
                            uint16_t* scales_out, float* w_out, cudaStream_t s);
 
-// Products (vbq_gemv.cu). Y is B x N. When the layout has more than one slab
-// per row, units add into Y, which the caller must have zeroed.
+// Products (vbq_gemv.cu). Y is B x N, overwritten (no zeroing needed).
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s);
+
+// How a batch-1 launch orders itself against the previous kernel on its
+// stream (programmatic dependent launch):
+//   DEP_BEFORE       lets the next kernel launch at once, then waits for the
+//                    previous kernel before touching x, y or control words
+//                    (every product call: x may be the previous output);
+//   DEP_GROUP_FIRST  waits first, then lets the next kernel launch, so the
+//                    rest of a group starts only after earlier stream work;
+//   DEP_GROUP_NEXT   lets the next kernel launch and works without waiting
+//                    (its inputs predate the group), then waits for the
+//                    previous kernel before it completes, so kernels still
+//                    complete in stream order.
+enum Dep : int { DEP_BEFORE = 0, DEP_GROUP_FIRST = 1, DEP_GROUP_NEXT = 2 };
+
+// count independent batch-1 products (distinct layouts and outputs) as one
+// group: launch i > 0 overlaps the tail of launch i - 1.
+cudaError_t launch_gemv_group(const LayoutView* const* Ls, const uint16_t* const* xs, float* const* ys, int count,
+                              cudaStream_t s);
 
 // Batch 1 with the split-K control words in a fixed device array (no
 // allocation anywhere); usable for layouts with at most STATIC_CTL_WORDS - 2

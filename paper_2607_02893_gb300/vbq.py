@@ -35,6 +35,7 @@ SIGNATURES = {
     "vbq_gemv": (_I, [_P, _P, _P, _P]),
     "vbq_gemm_small": (_I, [_P, _P, _P, _I, _P]),
     "vbq_gemv_static": (_I, [_P, _P, _P, _P]),
+    "vbq_gemv_group": (_I, [ctypes.POINTER(_P), ctypes.POINTER(_P), ctypes.POINTER(_P), _I, _P]),
     "vbq_device_status": (_I, [_P]),
     "vbq_selftest_timeout": (_I, [_I, _P]),
     "vbq_free": (_I, [_P]),
@@ -162,6 +163,19 @@ def vbq_gemv_static(layout: Layout, x, y, stream=None) -> None:
     """vbq_gemv that allocates nothing: its split-K control words live in a
     fixed array inside the library (see include/vbq.h)."""
     _check(load().vbq_gemv_static(layout, _ptr(x), _ptr(y), _stream(stream, x, y)))
+
+
+def vbq_gemv_group(layouts, xs, ys, stream=None) -> None:
+    """Independent batch-1 products y_i = W_i x_i whose launches overlap
+    (distinct layouts and outputs; no x_i written inside the group)."""
+    n = len(layouts)
+    if len(xs) != n or len(ys) != n:
+        raise ValueError("layouts, xs and ys must have the same length")
+    arr = _P * max(n, 1)
+    la = arr(*[lay._as_parameter_ for lay in layouts])
+    xa = arr(*[_ptr(x) for x in xs])
+    ya = arr(*[_ptr(y) for y in ys])
+    _check(load().vbq_gemv_group(la, xa, ya, int(n), _stream(stream, *(list(xs) + list(ys)))))
 
 
 def vbq_gemm_small(layout: Layout, X, Y, B: Optional[int] = None, stream=None) -> None:

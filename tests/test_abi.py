@@ -76,6 +76,18 @@ def test_calls_reject_null_layout(lib):
     assert lib.vbq_free(None) == 0
 
 
+def test_group_rejects_bad_arguments_on_host(lib):
+    P = ctypes.c_void_p
+    arr = (P * 2)()
+    assert lib.vbq_gemv_group(None, None, None, 0, None) == 0           # empty group: nothing to do
+    assert lib.vbq_gemv_group(arr, arr, arr, -1, None) == -1             # negative count
+    assert lib.vbq_gemv_group(None, arr, arr, 2, None) == -1             # NULL arrays
+    assert lib.vbq_gemv_group(arr, arr, arr, 2, None) == -1              # NULL layout entries
+    assert b"layout 0 is NULL" in lib.vbq_last_error()
+    with pytest.raises(ValueError):
+        vbq.vbq_gemv_group([None], [], [])
+
+
 def test_binding_raises_typed_errors(lib):
     with pytest.raises(vbq.VbqError) as ei:
         vbq.vbq_pack(0, 0, 0, N=4, K=64, src_on_device=0)
