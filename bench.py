@@ -68,6 +68,9 @@ def parse():
     p.add_argument("--workload", default="stack9b")
     p.add_argument("--batch", type=int, default=1)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--sweep", action="store_true",
+                   help="print the roofline sweep (N = K in 4096/8192/16384, batch 1..16, five width "
+                        "distributions) as one JSON line instead of the stack benchmark")
     p.add_argument("--no-modes", action="store_true",
                    help="skip the fused, grouped and cuBLAS BF16 companion measurements")
     p.add_argument("--event-ring", type=int, default=4)
@@ -507,6 +510,55 @@ def run_ours(args, rank, world, local_rank):
     return result, work
 
 
+def run_sweep(args):
+    """Every point of the roofline sweep: per (N, distribution) as many packed
+    copies as it takes to exceed 3x L2, then per batch a CUDA graph of launches
+    cycling through the copies; device time per launch, algorithmic GB/s and
+    the fraction of the measured copy bandwidth."""
+    import torch
+    import paper_2607_02893_gb300 as vbq
+    import synth
+    from synth import gen
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    vbq.load()
+    l2 = int(getattr(torch.cuda.get_device_properties(dev), "L2_cache_size", 0)) or (129 << 20)
+    peak, peak_kind = measured_peak()
+    stream = torch.cuda.Stream(device=dev)
+    points = []
+    for n in (4096, 8192, 16384):
+        for dist in synth.SWEEP_DISTS:
+            spec = synth.workload(f"sweep:{n}:{dist}", 16).mats[0]
+            inp = gen.matrix_inputs(spec, 16)
+            wd = torch.from_numpy(inp["widths"]).to(dev)
+            sc = torch.from_numpy(inp["scales"].view(np.uint16).astype(np.int16)).to(dev)
+            one = algorithmic_bytes(inp["widths"], n, n, 1)
+            copies = max(1, -(-3 * l2 // one))
+            codes = gen.codes_torch(wd, inp["key"], n, device=dev)
+            lays = [vbq.vbq_pack(codes, wd, sc) for _ in range(copies)]
+            del codes
+            X = torch.from_numpy(inp["x_bits"].astype(np.uint16).view(np.int16).copy()).to(dev)
+            for b in (1, 2, 4, 8, 16):
+                Y = torch.empty((b, n), dtype=torch.float32, device=dev)
+                reps = 4 * copies
+                if b == 1:
+                    fn = lambda: [vbq.vbq_gemv(lays[i % copies], X[0], Y[0], stream=stream) for i in range(reps)]
+                else:
+                    fn = lambda: [vbq.vbq_gemm_small(lays[i % copies], X[:b], Y, b, stream=stream)
+                                  for i in range(reps)]
+                ms = time_graph(torch, stream, fn, steps=5, warmup=3) / reps
+                nb = algorithmic_bytes(inp["widths"], n, n, b)
+                gbs = nb / (ms * 1e-3) / 1e9
+                points.append({"n": n, "dist": dist, "batch": b, "us": round(ms * 1e3, 2),
+                               "GBs": round(gbs, 1), "frac": round(gbs / peak, 4),
+                               "tokens_per_s": round(b / (ms * 1e-3), 1)})
+            del lays
+            torch.cuda.empty_cache()
+    return {"sweep": points, "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
+            "note": "algorithmic bytes (payload + FP16 scales + BF16 x + FP32 y) per launch over its device time, "
+                    "inputs larger than L2 (copies cycled)"}
+
+
 def run_reference(args):
     """The CPU oracle as the reference arm: step s runs the oracle on a random
     row block of matrix s mod M, sized so that the whole run takes a few minutes."""
@@ -565,6 +617,11 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.sweep:
+        if rank == 0:
+            print(json.dumps(run_sweep(args)), flush=True)
+        return
 
     if args.impl == "reference":
         if rank == 0:

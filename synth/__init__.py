@@ -9,7 +9,7 @@ random numbers for them.
 
 from .workloads import (  # noqa: F401
     DIST_MAIN, DIST_MLP0, DIST_HEAD, DIST_ALL1, DIST_ALL2, DIST_ALL4, DIST_ALL8,
-    MatrixSpec, Workload, workload, workload_names, sweep_points,
+    SWEEP_DISTS, MatrixSpec, Workload, workload, workload_names, sweep_points,
 )
 from .gen import (  # noqa: F401
     draw_widths, draw_scales, draw_x_bf16, bf16_bits_to_f32, f32_to_bf16_bits,
