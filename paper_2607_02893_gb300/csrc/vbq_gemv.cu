@@ -289,45 +289,45 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
             // so each quarter-warp's 16-byte loads fall in 8 distinct bank groups
             const int i = i0 + lane;
             const int c = task_column(U.ce, i0, SPAN, U.n, i);
-            if (i < U.n) {
-                const int h0 = (lane >> 2) & 1;
-                const uint4 va = lds_u32x4(U.pay + i * 32 + h0 * 16), vb = lds_u32x4(U.pay + i * 32 + (h0 ^ 1) * 16);
-                const uint32_t xa = smem_u32(T.x4s) + (c * 2 + h0) * XH * 4, xb = smem_u32(T.x4s) + (c * 2 + (h0 ^ 1)) * XH * 4;
-                const float2 aa = dot4_half(va, xa), ab = dot4_half(vb, xb);
-                const float4 z = lds_f32x4(smem_u32(T.x4z) + c * 16);     // (even, odd) of half 0, then of half 1
-                const float part = ((aa.x + ab.x) - 8.f * (z.x + z.z)) + ((aa.y + ab.y) - 8.f * (z.y + z.w));
-                sts_f32(slot_addr(slots, lds_u8(U.row + i), c), (half_bits(lds_u16(U.sc + 2 * i)) * 0x1p100f) * part);
-            }
+            const bool on = i < U.n;
+            const int ii = on ? i : 0;                  // lanes past the end redo item 0 and store nothing
+            const int h0 = (lane >> 2) & 1;
+            const uint4 va = lds_u32x4(U.pay + ii * 32 + h0 * 16), vb = lds_u32x4(U.pay + ii * 32 + (h0 ^ 1) * 16);
+            const uint32_t xa = smem_u32(T.x4s) + (c * 2 + h0) * XH * 4, xb = smem_u32(T.x4s) + (c * 2 + (h0 ^ 1)) * XH * 4;
+            const float2 aa = dot4_half(va, xa), ab = dot4_half(vb, xb);
+            const float4 z = lds_f32x4(smem_u32(T.x4z) + c * 16);         // (even, odd) of half 0, then of half 1
+            const float part = ((aa.x + ab.x) - 8.f * (z.x + z.z)) + ((aa.y + ab.y) - 8.f * (z.y + z.w));
+            sts_f32_if(slot_addr(slots, lds_u8(U.row + ii), c), (half_bits(lds_u16(U.sc + 2 * ii)) * 0x1p100f) * part, on);
         } else if constexpr (W == 3) {
             // 8-bit: one group per lane, quarter (k + (lane >> 1)) & 3 in step k
             // (conflict-free 16-byte loads for every quarter-warp)
             const int i = i0 + lane;
             const int c = task_column(U.ce, i0, SPAN, U.n, i);
-            if (i < U.n) {
-                const int q0 = lane >> 1;
-                float part = 0.f;
+            const bool on = i < U.n;
+            const int ii = on ? i : 0;
+            const int q0 = lane >> 1;
+            float part = 0.f;
 #pragma unroll
-                for (int step = 0; step < 4; ++step) {
-                    const int q = (step + q0) & 3;
-                    const uint4 v = lds_u32x4(U.pay + i * 64 + q * 16);
-                    part += dot8_quarter(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
-                }
-                sts_f32(slot_addr(slots, lds_u8(U.row + i), c), half_bits(lds_u16(U.sc + 2 * i)) * part);
+            for (int step = 0; step < 4; ++step) {
+                const int q = (step + q0) & 3;
+                const uint4 v = lds_u32x4(U.pay + ii * 64 + q * 16);
+                part += dot8_quarter(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
             }
+            sts_f32_if(slot_addr(slots, lds_u8(U.row + ii), c), half_bits(lds_u16(U.sc + 2 * ii)) * part, on);
         } else if constexpr (W == 1) {
             // 2-bit: one group per lane, both planes at once
             const int i = i0 + lane;
             const int c = task_column(U.ce, i0, SPAN, U.n, i);
-            if (i < U.n) {
-                const uint4 pl = lds_u32x4(U.pay + i * 16);
-                const uint32_t tb = smem_u32(T.lut) + c * LUT_COL_BYTES;
-                float va[16], vb[16];
-                plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
-                plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
-                const float2 sp = tree16x2(va, vb);
-                sts_f32(slot_addr(slots, lds_u8(U.row + i), c),
-                        half_bits(lds_u16(U.sc + 2 * i)) * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))));
-            }
+            const bool on = i < U.n;
+            const int ii = on ? i : 0;
+            const uint4 pl = lds_u32x4(U.pay + ii * 16);
+            const uint32_t tb = smem_u32(T.lut) + c * LUT_COL_BYTES;
+            float va[16], vb[16];
+            plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
+            plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
+            const float2 sp = tree16x2(va, vb);
+            sts_f32_if(slot_addr(slots, lds_u8(U.row + ii), c),
+                       half_bits(lds_u16(U.sc + 2 * ii)) * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))), on);
         } else {
             // 1-bit: two groups per lane, summed as a pair
             const int i = i0 + 2 * lane;
@@ -341,20 +341,19 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
                 ca = col_within(U.ce, cf, cl, i);
                 cb = col_within(U.ce, cf, cl, min(i + 1, U.n - 1));
             }
-            if (i < U.n) {
-                const bool two = i + 1 < U.n;
-                const uint4 v = lds_u32x4(U.pay + i * 8);
-                const uint32_t rows2 = lds_u16(U.row + i);
-                const uint32_t sc2 = lds_u32(U.sc + 2 * i);
-                float va[16], vb[16];
-                plane_entries(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
-                plane_entries(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
-                const float2 sp = tree16x2(va, vb);
-                const uint32_t xl = smem_u32(T.xlut);
-                if (two)
-                    sts_f32(slot_addr(slots, rows2 >> 8, cb), half_bits(sc2 >> 16) * (2.f * sp.y - lds_f32r(xl + 4 * cb)));
-                sts_f32(slot_addr(slots, rows2 & 0xff, ca), half_bits(sc2) * (2.f * sp.x - lds_f32r(xl + 4 * ca)));
-            }
+            // branch-free: lanes past the end redo item 0 (always present) and store nothing
+            const bool one = i < U.n, two = i + 1 < U.n;
+            const int ii = one ? i : 0;
+            const uint4 v = lds_u32x4(U.pay + ii * 8);
+            const uint32_t rows2 = lds_u16(U.row + ii);
+            const uint32_t sc2 = lds_u32(U.sc + 2 * ii);
+            float va[16], vb[16];
+            plane_entries(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
+            plane_entries(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
+            const float2 sp = tree16x2(va, vb);
+            const uint32_t xl = smem_u32(T.xlut);
+            sts_f32_if(slot_addr(slots, rows2 >> 8, cb), half_bits(sc2 >> 16) * (2.f * sp.y - lds_f32r(xl + 4 * cb)), two);
+            sts_f32_if(slot_addr(slots, rows2 & 0xff, ca), half_bits(sc2) * (2.f * sp.x - lds_f32r(xl + 4 * ca)), one);
         }
     }
 }
