@@ -261,6 +261,26 @@ def setup_stack(work, batch, dev, min_bytes: int = 0):
     return layouts, xs, ys, nbytes, host_x, copies
 
 
+def max_over_ranks(vals, device=None):
+    """Element-wise maximum of vals over the ranks of the default process group
+    (the values themselves on a single process)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in vals]
+    t = torch.tensor([float(v) for v in vals], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
+
+
+def job_throughput(step_bytes: int, copies: int, batch: int, world: int, ms_max: float):
+    """Whole-job GB/s and tokens/s: every rank streams its own replica of the
+    step, so the job moves world times the bytes in the slowest rank's time."""
+    gbs = step_bytes * world / (ms_max * 1e-3) / 1e9
+    tok_s = batch * copies * world / (ms_max * 1e-3)
+    return gbs, tok_s
+
+
 def time_graph(torch, stream, fn, steps: int, warmup: int) -> float:
     """ms per replay of fn captured as one CUDA graph on stream."""
     with torch.cuda.stream(stream):
@@ -443,15 +463,8 @@ def run_ours(args, rank, world, local_rank):
     e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
     barrier()
 
-    ms_max, e2e_max = ms, e2e_ms
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_max, e2e_max = float(t[0]), float(t[1])
-
-    gbs = step_bytes * world / (ms_max * 1e-3) / 1e9
-    tok_s = B * copies * world / (ms_max * 1e-3)
+    ms_max, e2e_max = max_over_ranks([ms, e2e_ms], device=dev)
+    gbs, tok_s = job_throughput(step_bytes, copies, B, world, ms_max)
     peak, peak_kind = measured_peak()
     kernel_gbs = step_bytes / (kernel_ms_per_step * 1e-3) / 1e9
     launches = len(layouts)
@@ -496,11 +509,11 @@ def run_ours(args, rank, world, local_rank):
             "avg_launch_us": round(kernel_ms_per_step * 1e3 / launches, 3),
         },
         "e2e": {
-            "value": round(step_bytes * world / (e2e_max * 1e-3) / 1e9, 1),
+            "value": round(job_throughput(step_bytes, copies, B, world, e2e_max)[0], 1),
             "unit": "GB/s",
             "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h),
-            "tokens_per_s": round(B * copies * world / (e2e_max * 1e-3), 1),
+            "tokens_per_s": round(job_throughput(step_bytes, copies, B, world, e2e_max)[1], 1),
         },
         "gpu_launches": launches * args.steps,
         "clocks": clk,
