@@ -36,7 +36,10 @@
 // shared-memory partial; a unit's rows then go to y directly (one slab per
 // row) or through atomics (several slabs).
 //
-// Batch 2..16 runs on the tensor cores in vbq_gemm.cu.
+// The same kernel takes two activation vectors per launch (NX = 2, batches of
+// 2..4 as one or two launches): the second vector's tables sit a fixed
+// distance after the first's, so each lookup address, masked code and level
+// serves both. Batches of 5..16 run on the tensor cores in vbq_gemm.cu.
 #include <cstddef>
 #include <mutex>
 
@@ -48,15 +51,7 @@ namespace {
 
 constexpr int NCW = 16;                  // consumer warps of the batch-1 kernel
 constexpr int NCT = 32 * NCW;            // consumer threads
-constexpr int MAX_TEAMS = 2;             // consumer teams (1 or 2 by units per block); unit j goes to team j % teams
-static_assert(MAX_TEAMS == 2 && NCW == 16, "teams of 16 or 8 warps: task steps are powers of two (masks, no division)");
-// Unit j uses stage j % NSTAGE and goes to team j % teams; with NSTAGE a
-// multiple of every team count, each stage serves one team only, and that team
-// waits the stage's phases in order (a parity wait never skips a phase).
 constexpr int G1_THREADS = 32 * (NCW + 1);
-constexpr int NSTAGE = 4;                // blob stages in flight per SM
-static_assert((NSTAGE & (NSTAGE - 1)) == 0, "power-of-two stage count");
-static_assert(NSTAGE % MAX_TEAMS == 0, "every team count (1, 2) divides the stage count");
 constexpr int XQ = 20;                   // floats per 16-code quarter of x (16 + 4 pad: quarters use other banks)
 constexpr int XH = 36;                   // floats per 32-code half of the pre-scaled x (32 + 4 pad)
 constexpr int LUT_COL_BYTES = 1280;      // 16 tables x 64 bytes (+64 for odd columns), columns on 256-byte boundaries
@@ -64,27 +59,57 @@ constexpr int STAGE_BYTES = MAX_BLOB_BYTES;   // holds the largest unit blob (th
 static_assert(STAGE_BYTES % 256 == 0, "stages keep the tables 256-byte aligned");
 static_assert(LUT_COL_BYTES % 256 == 0 && 64 + 16 * 64 <= LUT_COL_BYTES, "column tables: 256-byte aligned, room for the odd shift");
 
-struct __align__(16) Tables {
-    uint8_t lut[MAX_C * LUT_COL_BYTES];  // column c, nibble j, entry m at c*1280 + (c&1)*64 + j*64 + m*4
-    float xs[MAX_C * 4 * XQ];            // x as fp32; quarter (c, q) at (c*4 + q) * XQ
-    float x4s[MAX_C * 2 * XH];           // x pre-scaled per 4-bit nibble slot (see dot4_half); half (c, h) at (c*2 + h) * XH
-    float2 x4z[MAX_C][2];                // per column and half: sums of x * 2^-100, even / odd codes
-    float xlut[MAX_C];                   // per column: sum of the all-ones entries, in lookup order
-    float slots[NSTAGE][RB * MAX_C];     // per stage: one value per (row, column) of the unit (see slot_addr)
-    unsigned long long full[NSTAGE];     // blob landed (TMA transaction count)
-    unsigned long long empty[NSTAGE];    // the unit's team is done (one arrival per team warp)
+// One kernel serves NX = 1 or 2 activation vectors (batch rows) per launch.
+// With two, every table lookup address serves both: the second vector's
+// tables sit a fixed distance after the first's, reached by the load's
+// immediate offset. Per vector (byte strides between the vectors' copies):
+constexpr int LUT_BYTES = MAX_C * LUT_COL_BYTES;          // nibble lookup tables
+constexpr int XS_FLOATS = MAX_C * 4 * XQ;                 // x as fp32
+constexpr int X4S_FLOATS = MAX_C * 2 * XH;                // pre-scaled 4-bit slots
+constexpr int SLOT_FLOATS = RB * MAX_C;                   // (row, column) slots of a unit
+static_assert(LUT_BYTES % 256 == 0, "the second vector's tables keep the byte-merge alignment");
+
+// Stages and consumer teams per vector count. Unit j uses stage j % nstage and
+// goes to team j % teams; with nstage a multiple of every team count, each
+// stage serves one team only, and that team waits the stage's phases in order
+// (a parity wait never skips a phase). Two teams give each team two stages,
+// so its next blob lands while it works on the current one; two vectors'
+// tables leave room for two stages and one team.
+template <int NX> struct Geo {
+    static constexpr int nstage = NX == 1 ? 4 : 2;
+    static constexpr int max_teams = NX == 1 ? 2 : 1;
+    static_assert((nstage & (nstage - 1)) == 0, "power-of-two stage count");
+    static_assert(nstage % max_teams == 0 && nstage / max_teams >= 2, "each team owns at least two stages");
+};
+static_assert(NCW == 16, "teams of 16 or 8 warps: task steps are powers of two (masks, no division)");
+
+template <int NX>
+struct __align__(16) TablesT {
+    uint8_t lut[NX * LUT_BYTES];         // vector v, column c, nibble j, entry m at v*LUT_BYTES + c*1280 + (c&1)*64 + j*64 + m*4
+    float xs[NX * XS_FLOATS];            // x as fp32; quarter (c, q) at (c*4 + q) * XQ
+    float x4s[NX * X4S_FLOATS];          // x pre-scaled per 4-bit nibble slot (see dot4_half); half (c, h) at (c*2 + h) * XH
+    float2 x4z[NX][MAX_C][2];            // per column and half: sums of x * 2^-100, even / odd codes
+    float xlut[NX][MAX_C];               // per column: sum of the all-ones entries, in lookup order
+    float slots[Geo<NX>::nstage][NX][SLOT_FLOATS];   // per stage and vector: one value per (row, column) (see slot_addr)
+    unsigned long long full[Geo<NX>::nstage];        // blob landed (TMA transaction count)
+    unsigned long long empty[Geo<NX>::nstage];       // the unit's team is done (one arrival per team warp)
     int abort;                           // set by any role whose wait ran out
 };
-static_assert(offsetof(Tables, full) % 8 == 0, "mbarriers are 8-byte aligned");
-static_assert(offsetof(Tables, lut) == 0, "tables start at the aligned base");
-static_assert(offsetof(Tables, x4z) % 16 == 0 && offsetof(Tables, xs) % 16 == 0 && offsetof(Tables, x4s) % 16 == 0 &&
-              offsetof(Tables, slots) % 16 == 0,
-              "16-byte table reads");
+template <int NX> struct TablesCheck {
+    using T = TablesT<NX>;
+    static_assert(offsetof(T, full) % 8 == 0, "mbarriers are 8-byte aligned");
+    static_assert(offsetof(T, lut) == 0, "tables start at the aligned base");
+    static_assert(offsetof(T, x4z) % 16 == 0 && offsetof(T, xs) % 16 == 0 && offsetof(T, x4s) % 16 == 0 &&
+                  offsetof(T, slots) % 16 == 0, "16-byte table reads");
+    static constexpr bool ok = true;
+};
+static_assert(TablesCheck<1>::ok && TablesCheck<2>::ok, "table layout");
 static_assert(RB % 32 == 0, "the copier flushes rows a warp at a time");
 static_assert(MAX_C <= 32, "a warp holds a unit's column ends one per lane");
 
-constexpr size_t GEMV1_SMEM = 256 /* alignment slack */ + (size_t)NSTAGE * STAGE_BYTES + sizeof(Tables);
-static_assert(GEMV1_SMEM <= 227 * 1024, "one block per SM");
+template <int NX>
+constexpr size_t gemv1_smem() { return 256 /* alignment slack */ + (size_t)Geo<NX>::nstage * STAGE_BYTES + sizeof(TablesT<NX>); }
+static_assert(gemv1_smem<1>() <= 227 * 1024 && gemv1_smem<2>() <= 227 * 1024, "one block per SM");
 
 // The 16 table entries that a 64-bit bit plane (words lo, hi) selects from a
 // column's tables at tb (256-byte aligned): nibble p of the plane picks entry
@@ -185,75 +210,168 @@ __device__ __forceinline__ float dot8_quarter(uint4 v, uint32_t xa) {
     return (ca.x + ca.y) + (cb.x + cb.y);
 }
 
+// Two activation vectors: the same 16 lookups of a plane, each address
+// reading the first vector's entry (.x) and the second's, LUT_BYTES further
+// (.y).
+template <int OFF>
+__device__ __forceinline__ float2 lds_pair(uint32_t a) { return f2(lds_f32<OFF>(a), lds_f32<OFF + LUT_BYTES>(a)); }
+__device__ __forceinline__ void plane_entries2(uint32_t tb, uint32_t sh4, uint32_t lo, uint32_t hi, float2 (&v)[16]) {
+    const uint32_t M = 0x3C3C3C3Cu;
+    const uint32_t le = ((lo << 2) & M) | sh4, lo_ = ((lo >> 2) & M) | sh4;
+    const uint32_t he = ((hi << 2) & M) | sh4, ho = ((hi >> 2) & M) | sh4;
+    v[0] = lds_pair<0>(__byte_perm(le, tb, 0x7650));
+    v[1] = lds_pair<64>(__byte_perm(lo_, tb, 0x7650));
+    v[2] = lds_pair<128>(__byte_perm(le, tb, 0x7651));
+    v[3] = lds_pair<192>(__byte_perm(lo_, tb, 0x7651));
+    v[4] = lds_pair<256>(__byte_perm(le, tb, 0x7652));
+    v[5] = lds_pair<320>(__byte_perm(lo_, tb, 0x7652));
+    v[6] = lds_pair<384>(__byte_perm(le, tb, 0x7653));
+    v[7] = lds_pair<448>(__byte_perm(lo_, tb, 0x7653));
+    v[8] = lds_pair<512>(__byte_perm(he, tb, 0x7650));
+    v[9] = lds_pair<576>(__byte_perm(ho, tb, 0x7650));
+    v[10] = lds_pair<640>(__byte_perm(he, tb, 0x7651));
+    v[11] = lds_pair<704>(__byte_perm(ho, tb, 0x7651));
+    v[12] = lds_pair<768>(__byte_perm(he, tb, 0x7652));
+    v[13] = lds_pair<832>(__byte_perm(ho, tb, 0x7652));
+    v[14] = lds_pair<896>(__byte_perm(he, tb, 0x7653));
+    v[15] = lds_pair<960>(__byte_perm(ho, tb, 0x7653));
+}
+// Sums of 16 pairs in the order tree16x2 adds each of its two operands.
+__device__ __forceinline__ float2 tree16_pairs(const float2 (&a)[16]) {
+    float2 p[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) p[i] = __fadd2_rn(a[2 * i], a[2 * i + 1]);
+    const float2 q0 = __fadd2_rn(p[0], p[1]), q1 = __fadd2_rn(p[2], p[3]);
+    const float2 q2 = __fadd2_rn(p[4], p[5]), q3 = __fadd2_rn(p[6], p[7]);
+    return __fadd2_rn(__fadd2_rn(q0, q1), __fadd2_rn(q2, q3));
+}
+// dot4_half for two vectors: the masked codes are shared, each vector's
+// pre-scaled slots are X4S_FLOATS after the previous one's.
+__device__ __forceinline__ void dot4_half2(uint4 v, uint32_t xa, float2& r0, float2& r1) {
+    float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f), da = f2(0.f, 0.f), db = f2(0.f, 0.f);
+    const uint32_t words[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+        const uint32_t w = words[t], w2 = w >> 24;
+        const float4 xa4 = lds_f32x4(xa + t * 32), xb4 = lds_f32x4(xa + t * 32 + 16);
+        const float4 ya4 = lds_f32x4(xa + 4 * X4S_FLOATS + t * 32), yb4 = lds_f32x4(xa + 4 * X4S_FLOATS + t * 32 + 16);
+        const float2 u0 = f2(__uint_as_float(w & 0xFu), __uint_as_float(w & 0xF0u));
+        const float2 u1 = f2(__uint_as_float(w & 0xF00u), __uint_as_float(w & 0xF000u));
+        const float2 u2 = f2(__uint_as_float(w & 0xF0000u), __uint_as_float(w & 0xF00000u));
+        const float2 u3 = f2(__uint_as_float(w2 & 0xFu), __uint_as_float(w2 & 0xF0u));
+        float2& c = (t & 1) ? cb : ca;
+        float2& d = (t & 1) ? db : da;
+        c = __ffma2_rn(u0, f2(xa4.x, xa4.y), c);
+        c = __ffma2_rn(u1, f2(xa4.z, xa4.w), c);
+        c = __ffma2_rn(u2, f2(xb4.x, xb4.y), c);
+        c = __ffma2_rn(u3, f2(xb4.z, xb4.w), c);
+        d = __ffma2_rn(u0, f2(ya4.x, ya4.y), d);
+        d = __ffma2_rn(u1, f2(ya4.z, ya4.w), d);
+        d = __ffma2_rn(u2, f2(yb4.x, yb4.y), d);
+        d = __ffma2_rn(u3, f2(yb4.z, yb4.w), d);
+    }
+    r0 = __fadd2_rn(ca, cb);
+    r1 = __fadd2_rn(da, db);
+}
+// dot8_quarter for two vectors (levels shared; each vector's fp32 x is
+// XS_FLOATS after the previous one's). Returns (vector 0, vector 1).
+__device__ __forceinline__ float2 dot8_quarter2(uint4 v, uint32_t xa) {
+    const float2 off = f2(-8388736.f, -8388736.f);          // -(2^23 + 128)
+    const uint32_t M = 0x4B000000u;
+    float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f), da = f2(0.f, 0.f), db = f2(0.f, 0.f);
+    const uint32_t words[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+        const uint32_t w = words[t];
+        const float4 x4 = lds_f32x4(xa + t * 16), y4 = lds_f32x4(xa + 4 * XS_FLOATS + t * 16);
+        const float2 l0 = __fadd2_rn(f2(__uint_as_float(__byte_perm(w, M, 0x7540)),
+                                        __uint_as_float(__byte_perm(w, M, 0x7541))), off);
+        const float2 l1 = __fadd2_rn(f2(__uint_as_float(__byte_perm(w, M, 0x7542)),
+                                        __uint_as_float(__byte_perm(w, M, 0x7543))), off);
+        ca = __ffma2_rn(l0, f2(x4.x, x4.y), ca);
+        cb = __ffma2_rn(l1, f2(x4.z, x4.w), cb);
+        da = __ffma2_rn(l0, f2(y4.x, y4.y), da);
+        db = __ffma2_rn(l1, f2(y4.z, y4.w), db);
+    }
+    return f2((ca.x + ca.y) + (cb.x + cb.y), (da.x + da.y) + (db.x + db.y));
+}
+
 // Consumer warps only (named barrier 1).
 __device__ __forceinline__ void consumer_sync() {
     asm volatile("bar.sync 1, %0;" :: "n"(NCT) : "memory");
 }
 
-// Activations of slab s: x as fp32, the pre-scaled x of the 4-bit slots, the
-// nibble lookup tables, and the per-column sums in lookup order. Consumer
+// Activations of slab s (per vector, for NX vectors stored K apart): x as fp32,
+// the pre-scaled x of the 4-bit slots, the nibble lookup tables, and the
+// per-column sums in lookup order. Consumer
 // threads only (ct = 0 .. NCT-1), one thread per (column, 4 weights): each
 // reads its 4 activations from global memory (L2), so the whole build is one
 // phase between two consumer barriers. The column sum of the all-ones entries
 // (xlut) is added over the column's half-warp in the pairs tree16x2 uses.
-__device__ void build_tables(Tables& T, const LayoutView& L, const uint16_t* __restrict__ x, int s, int ct) {
+template <int NX>
+__device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t* __restrict__ x, int s, int ct) {
     const int cols = min(L.C, L.G - s * L.C);
-    const uint16_t* xg = x + (int64_t)s * L.C * GROUP;
     consumer_sync();                // nobody still reads the old tables
     if (ct < cols * 16) {
         const int c = ct >> 4, jn = ct & 15, jj = 4 * jn;
-        const uint2 four = __ldg(reinterpret_cast<const uint2*>(xg + c * GROUP + jj));
-        const float x0 = __uint_as_float(four.x << 16), x1 = __uint_as_float(four.x & 0xFFFF0000u);
-        const float x2 = __uint_as_float(four.y << 16), x3 = __uint_as_float(four.y & 0xFFFF0000u);
-        *reinterpret_cast<float4*>(&T.xs[(c * 4 + (jj >> 4)) * XQ + (jj & 15)]) = make_float4(x0, x1, x2, x3);
-        // 4-bit slot shifts: nibble slots 0..5 of a word keep their place, 6 and 7 come down by 24
-        float p4[4];
-        const float xv4[4] = {x0, x1, x2, x3};
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int slot = (jj + i) & 7, e = slot < 6 ? 4 * slot : 4 * (slot - 6);
-            p4[i] = xv4[i] * __uint_as_float((uint32_t)(127 + 49 - e) << 23);
-        }
-        *reinterpret_cast<float4*>(&T.x4s[(c * 2 + (jj >> 5)) * XH + (jj & 31)]) = make_float4(p4[0], p4[1], p4[2], p4[3]);
-        const float t3 = x0 + x1, t12 = x3 + x2;
-        float4* dst = reinterpret_cast<float4*>(T.lut + c * LUT_COL_BYTES + (c & 1) * 64 + jn * 64);
-        dst[0] = make_float4(0.f, x0, x1, t3);
-        dst[1] = make_float4(x2, x2 + x0, x2 + x1, x2 + t3);
-        dst[2] = make_float4(x3, x3 + x0, x3 + x1, x3 + t3);
-        dst[3] = make_float4(t12, t12 + x0, t12 + x1, t12 + t3);
-        // xlut: balanced tree over the column's 16 all-ones entries (xor 1, 2, 4, 8
-        // pair them as tree16x2 pairs the lookups)
-        const unsigned half = (ct & 16) ? 0xFFFF0000u : 0x0000FFFFu;
-        float v = t12 + t3;
-        v += __shfl_xor_sync(half, v, 1);
-        v += __shfl_xor_sync(half, v, 2);
-        v += __shfl_xor_sync(half, v, 4);
-        v += __shfl_xor_sync(half, v, 8);
-        if (jn == 0) T.xlut[c] = v;
-        // X for the 4-bit zero level of half hh, summed as dot4_half accumulates
-        if ((jn & 7) == 0) {
-            const int hh = jn >> 3;
-            const uint4* src = reinterpret_cast<const uint4*>(xg + c * GROUP + 32 * hh);
-            float xh[32];
+        for (int v = 0; v < NX; ++v) {
+            const uint16_t* xg = x + (int64_t)v * L.K + (int64_t)s * L.C * GROUP;
+            float* xs = T.xs + v * XS_FLOATS;
+            float* x4s = T.x4s + v * X4S_FLOATS;
+            const uint2 four = __ldg(reinterpret_cast<const uint2*>(xg + c * GROUP + jj));
+            const float x0 = __uint_as_float(four.x << 16), x1 = __uint_as_float(four.x & 0xFFFF0000u);
+            const float x2 = __uint_as_float(four.y << 16), x3 = __uint_as_float(four.y & 0xFFFF0000u);
+            *reinterpret_cast<float4*>(&xs[(c * 4 + (jj >> 4)) * XQ + (jj & 15)]) = make_float4(x0, x1, x2, x3);
+            // 4-bit slot shifts: nibble slots 0..5 of a word keep their place, 6 and 7 come down by 24
+            float p4[4];
+            const float xv4[4] = {x0, x1, x2, x3};
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint4 w = __ldg(src + q);
-                const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+            for (int i = 0; i < 4; ++i) {
+                const int slot = (jj + i) & 7, e = slot < 6 ? 4 * slot : 4 * (slot - 6);
+                p4[i] = xv4[i] * __uint_as_float((uint32_t)(127 + 49 - e) << 23);
+            }
+            *reinterpret_cast<float4*>(&x4s[(c * 2 + (jj >> 5)) * XH + (jj & 31)]) = make_float4(p4[0], p4[1], p4[2], p4[3]);
+            const float t3 = x0 + x1, t12 = x3 + x2;
+            float4* dst = reinterpret_cast<float4*>(T.lut + v * LUT_BYTES + c * LUT_COL_BYTES + (c & 1) * 64 + jn * 64);
+            dst[0] = make_float4(0.f, x0, x1, t3);
+            dst[1] = make_float4(x2, x2 + x0, x2 + x1, x2 + t3);
+            dst[2] = make_float4(x3, x3 + x0, x3 + x1, x3 + t3);
+            dst[3] = make_float4(t12, t12 + x0, t12 + x1, t12 + t3);
+            // xlut: balanced tree over the column's 16 all-ones entries (xor 1, 2, 4, 8
+            // pair them as tree16x2 pairs the lookups)
+            const unsigned half = (ct & 16) ? 0xFFFF0000u : 0x0000FFFFu;
+            float sv = t12 + t3;
+            sv += __shfl_xor_sync(half, sv, 1);
+            sv += __shfl_xor_sync(half, sv, 2);
+            sv += __shfl_xor_sync(half, sv, 4);
+            sv += __shfl_xor_sync(half, sv, 8);
+            if (jn == 0) T.xlut[v][c] = sv;
+            // X for the 4-bit zero level of half hh, summed as dot4_half accumulates
+            if ((jn & 7) == 0) {
+                const int hh = jn >> 3;
+                const uint4* src = reinterpret_cast<const uint4*>(xg + c * GROUP + 32 * hh);
+                float xh[32];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    xh[8 * q + 2 * i] = __uint_as_float(ws[i] << 16);
-                    xh[8 * q + 2 * i + 1] = __uint_as_float(ws[i] & 0xFFFF0000u);
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 w = __ldg(src + q);
+                    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        xh[8 * q + 2 * i] = __uint_as_float(ws[i] << 16);
+                        xh[8 * q + 2 * i + 1] = __uint_as_float(ws[i] & 0xFFFF0000u);
+                    }
                 }
-            }
-            float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
+                float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
 #pragma unroll
-            for (int t4 = 0; t4 < 4; ++t4) {
-                float2& cc = (t4 & 1) ? cb : ca;
+                for (int t4 = 0; t4 < 4; ++t4) {
+                    float2& cc = (t4 & 1) ? cb : ca;
 #pragma unroll
-                for (int e = 0; e < 8; e += 2)
-                    cc = __ffma2_rn(f2(xh[8 * t4 + e], xh[8 * t4 + e + 1]), f2(0x1p-100f, 0x1p-100f), cc);
+                    for (int e = 0; e < 8; e += 2)
+                        cc = __ffma2_rn(f2(xh[8 * t4 + e], xh[8 * t4 + e + 1]), f2(0x1p-100f, 0x1p-100f), cc);
+                }
+                T.x4z[v][c][hh] = __fadd2_rn(ca, cb);
             }
-            T.x4z[c][hh] = __fadd2_rn(ca, cb);
         }
     }
     consumer_sync();
@@ -277,10 +395,11 @@ __device__ __forceinline__ int task_column(uint32_t ce, int i0, int span, int n,
 // Tasks of one width: items are taken 32 (64 for 1-bit) at a time, task
 // k = first, first + tstep, ... of this width's nt tasks. Every lane holds
 // whole groups, so a task's bookkeeping is shared by 32 groups.
-template <int W>
-__device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, uint32_t slots, int first, int tstep,
+template <int W, int NX>
+__device__ __forceinline__ void run_width(const TablesT<NX>& T, const UnitView& U, uint32_t slots, int first, int tstep,
                                           int lane) {
     constexpr int SPAN = W == 0 ? 64 : 32;
+    constexpr uint32_t SLOT_V = SLOT_FLOATS * 4;      // bytes between the vectors' slot arrays
     const int nt = (U.n + SPAN - 1) / SPAN;
     for (int k = first; k < nt; k += tstep) {
         const int i0 = k * SPAN;
@@ -294,10 +413,23 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
             const int h0 = (lane >> 2) & 1;
             const uint4 va = lds_u32x4(U.pay + ii * 32 + h0 * 16), vb = lds_u32x4(U.pay + ii * 32 + (h0 ^ 1) * 16);
             const uint32_t xa = smem_u32(T.x4s) + (c * 2 + h0) * XH * 4, xb = smem_u32(T.x4s) + (c * 2 + (h0 ^ 1)) * XH * 4;
-            const float2 aa = dot4_half(va, xa), ab = dot4_half(vb, xb);
-            const float4 z = lds_f32x4(smem_u32(T.x4z) + c * 16);         // (even, odd) of half 0, then of half 1
-            const float part = ((aa.x + ab.x) - 8.f * (z.x + z.z)) + ((aa.y + ab.y) - 8.f * (z.y + z.w));
-            sts_f32_if(slot_addr(slots, lds_u8(U.row + ii), c), (half_bits(lds_u16(U.sc + 2 * ii)) * 0x1p100f) * part, on);
+            const uint32_t sa = slot_addr(slots, lds_u8(U.row + ii), c);
+            const float scl = half_bits(lds_u16(U.sc + 2 * ii)) * 0x1p100f;
+            if constexpr (NX == 1) {
+                const float2 aa = dot4_half(va, xa), ab = dot4_half(vb, xb);
+                const float4 z = lds_f32x4(smem_u32(T.x4z) + c * 16);     // (even, odd) of half 0, then of half 1
+                const float part = ((aa.x + ab.x) - 8.f * (z.x + z.z)) + ((aa.y + ab.y) - 8.f * (z.y + z.w));
+                sts_f32_if(sa, scl * part, on);
+            } else {
+                float2 aa0, aa1, ab0, ab1;
+                dot4_half2(va, xa, aa0, aa1);
+                dot4_half2(vb, xb, ab0, ab1);
+                const float4 z0 = lds_f32x4(smem_u32(T.x4z) + c * 16), z1 = lds_f32x4(smem_u32(T.x4z) + MAX_C * 16 + c * 16);
+                const float p0 = ((aa0.x + ab0.x) - 8.f * (z0.x + z0.z)) + ((aa0.y + ab0.y) - 8.f * (z0.y + z0.w));
+                const float p1 = ((aa1.x + ab1.x) - 8.f * (z1.x + z1.z)) + ((aa1.y + ab1.y) - 8.f * (z1.y + z1.w));
+                sts_f32_if(sa, scl * p0, on);
+                sts_f32_if(sa + SLOT_V, scl * p1, on);
+            }
         } else if constexpr (W == 3) {
             // 8-bit: one group per lane, quarter (k + (lane >> 1)) & 3 in step k
             // (conflict-free 16-byte loads for every quarter-warp)
@@ -306,14 +438,30 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
             const bool on = i < U.n;
             const int ii = on ? i : 0;
             const int q0 = lane >> 1;
-            float part = 0.f;
+            const uint32_t sa = slot_addr(slots, lds_u8(U.row + ii), c);
+            const float scl = half_bits(lds_u16(U.sc + 2 * ii));
+            if constexpr (NX == 1) {
+                float part = 0.f;
 #pragma unroll
-            for (int step = 0; step < 4; ++step) {
-                const int q = (step + q0) & 3;
-                const uint4 v = lds_u32x4(U.pay + ii * 64 + q * 16);
-                part += dot8_quarter(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
+                for (int step = 0; step < 4; ++step) {
+                    const int q = (step + q0) & 3;
+                    const uint4 v = lds_u32x4(U.pay + ii * 64 + q * 16);
+                    part += dot8_quarter(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
+                }
+                sts_f32_if(sa, scl * part, on);
+            } else {
+                float p0 = 0.f, p1 = 0.f;
+#pragma unroll
+                for (int step = 0; step < 4; ++step) {
+                    const int q = (step + q0) & 3;
+                    const uint4 v = lds_u32x4(U.pay + ii * 64 + q * 16);
+                    const float2 d = dot8_quarter2(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
+                    p0 += d.x;
+                    p1 += d.y;
+                }
+                sts_f32_if(sa, scl * p0, on);
+                sts_f32_if(sa + SLOT_V, scl * p1, on);
             }
-            sts_f32_if(slot_addr(slots, lds_u8(U.row + ii), c), half_bits(lds_u16(U.sc + 2 * ii)) * part, on);
         } else if constexpr (W == 1) {
             // 2-bit: one group per lane, both planes at once
             const int i = i0 + lane;
@@ -322,12 +470,24 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
             const int ii = on ? i : 0;
             const uint4 pl = lds_u32x4(U.pay + ii * 16);
             const uint32_t tb = smem_u32(T.lut) + c * LUT_COL_BYTES;
-            float va[16], vb[16];
-            plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
-            plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
-            const float2 sp = tree16x2(va, vb);
-            sts_f32_if(slot_addr(slots, lds_u8(U.row + ii), c),
-                       half_bits(lds_u16(U.sc + 2 * ii)) * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))), on);
+            const uint32_t sa = slot_addr(slots, lds_u8(U.row + ii), c);
+            const float scl = half_bits(lds_u16(U.sc + 2 * ii));
+            if constexpr (NX == 1) {
+                float va[16], vb[16];
+                plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
+                plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
+                const float2 sp = tree16x2(va, vb);
+                sts_f32_if(sa, scl * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))), on);
+            } else {
+                float2 pv[16];
+                plane_entries2(tb, col_shift4(c), pl.x, pl.y, pv);
+                const float2 s0 = tree16_pairs(pv);                       // plane 0, both vectors
+                plane_entries2(tb, col_shift4(c), pl.z, pl.w, pv);
+                const float2 s1 = tree16_pairs(pv);                       // plane 1
+                const uint32_t xl = smem_u32(T.xlut) + 4 * c;
+                sts_f32_if(sa, scl * (s0.x + 2.f * (s1.x - lds_f32r(xl))), on);
+                sts_f32_if(sa + SLOT_V, scl * (s0.y + 2.f * (s1.y - lds_f32r(xl + 4 * MAX_C))), on);
+            }
         } else {
             // 1-bit: two groups per lane, summed as a pair
             const int i = i0 + 2 * lane;
@@ -347,13 +507,27 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
             const uint4 v = lds_u32x4(U.pay + ii * 8);
             const uint32_t rows2 = lds_u16(U.row + ii);
             const uint32_t sc2 = lds_u32(U.sc + 2 * ii);
-            float va[16], vb[16];
-            plane_entries(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
-            plane_entries(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
-            const float2 sp = tree16x2(va, vb);
             const uint32_t xl = smem_u32(T.xlut);
-            sts_f32_if(slot_addr(slots, rows2 >> 8, cb), half_bits(sc2 >> 16) * (2.f * sp.y - lds_f32r(xl + 4 * cb)), two);
-            sts_f32_if(slot_addr(slots, rows2 & 0xff, ca), half_bits(sc2) * (2.f * sp.x - lds_f32r(xl + 4 * ca)), one);
+            const uint32_t sb = slot_addr(slots, rows2 >> 8, cb), sa = slot_addr(slots, rows2 & 0xff, ca);
+            const float scb = half_bits(sc2 >> 16), sca = half_bits(sc2);
+            if constexpr (NX == 1) {
+                float va[16], vb[16];
+                plane_entries(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
+                plane_entries(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
+                const float2 sp = tree16x2(va, vb);
+                sts_f32_if(sb, scb * (2.f * sp.y - lds_f32r(xl + 4 * cb)), two);
+                sts_f32_if(sa, sca * (2.f * sp.x - lds_f32r(xl + 4 * ca)), one);
+            } else {
+                float2 pv[16];
+                plane_entries2(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, pv);
+                const float2 sx = tree16_pairs(pv);                       // item i, both vectors
+                sts_f32_if(sa, sca * (2.f * sx.x - lds_f32r(xl + 4 * ca)), one);
+                sts_f32_if(sa + SLOT_V, sca * (2.f * sx.y - lds_f32r(xl + 4 * MAX_C + 4 * ca)), one);
+                plane_entries2(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, pv);
+                const float2 sy = tree16_pairs(pv);                       // item i + 1
+                sts_f32_if(sb, scb * (2.f * sy.x - lds_f32r(xl + 4 * cb)), two);
+                sts_f32_if(sb + SLOT_V, scb * (2.f * sy.y - lds_f32r(xl + 4 * MAX_C + 4 * cb)), two);
+            }
         }
     }
 }
@@ -363,7 +537,8 @@ __device__ __forceinline__ void run_width(const Tables& T, const UnitView& U, ui
 // (costliest first); this warp takes tasks t0, t0 + tstep, ... of that
 // sequence (tstep a power of two). Each group's result goes to its slot in
 // the stage's slot array at shared address slots.
-__device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, int C, int cols, uint32_t slots,
+template <int NX>
+__device__ __forceinline__ void consume_unit(const TablesT<NX>& T, uint32_t sblob, int C, int cols, uint32_t slots,
                                              int t0, int tstep, int lane) {
     // UnitHeader fields, read as three 16-byte words
     const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
@@ -386,18 +561,21 @@ __device__ __forceinline__ void consume_unit(const Tables& T, uint32_t sblob, in
     // b + ((t0 - b) mod tstep), tstep a power of two
     const int nt3 = (n[3] + 31) >> 5, nt2 = (n[2] + 31) >> 5, nt1 = (n[1] + 31) >> 5;
     const int m = tstep - 1;
-    if (n[3]) run_width<3>(T, view(3), slots, t0 & m, tstep, lane);
-    if (n[2]) run_width<2>(T, view(2), slots, (t0 - nt3) & m, tstep, lane);
-    if (n[1]) run_width<1>(T, view(1), slots, (t0 - nt3 - nt2) & m, tstep, lane);
-    if (n[0]) run_width<0>(T, view(0), slots, (t0 - nt3 - nt2 - nt1) & m, tstep, lane);
+    if (n[3]) run_width<3, NX>(T, view(3), slots, t0 & m, tstep, lane);
+    if (n[2]) run_width<2, NX>(T, view(2), slots, (t0 - nt3) & m, tstep, lane);
+    if (n[1]) run_width<1, NX>(T, view(1), slots, (t0 - nt3 - nt2) & m, tstep, lane);
+    if (n[0]) run_width<0, NX>(T, view(0), slots, (t0 - nt3 - nt2 - nt1) & m, tstep, lane);
 }
 
+// NX activation vectors x (NX x K, row-major) and outputs y (NX x N).
+template <int NX>
 __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
                                                               float* __restrict__ y, int dep) {
+    constexpr int NSTAGE = Geo<NX>::nstage;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     // stages and tables on a 256-byte boundary: lookups merge a byte into table addresses
     unsigned char* base = smem_raw + ((256u - (smem_u32(smem_raw) & 255u)) & 255u);
-    Tables& T = *reinterpret_cast<Tables*>(base + (size_t)NSTAGE * STAGE_BYTES);
+    TablesT<NX>& T = *reinterpret_cast<TablesT<NX>*>(base + (size_t)NSTAGE * STAGE_BYTES);
     const uint32_t stage0 = smem_u32(base);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int P = gridDim.x, p = blockIdx.x;
@@ -411,7 +589,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     // unit (less per-unit overhead); few units -> whole-block teams (less latency)
     // two teams once the block has 4 units: each team then has NSTAGE / 2
     // stages, so its next blob lands while it works on the current one
-    const int lg_teams = n_units >= 4 ? 1 : 0;
+    const int lg_teams = Geo<NX>::max_teams == 2 && n_units >= 4 ? 1 : 0;
     const int teams = 1 << lg_teams, tw = NCW >> lg_teams;
 
     const uint32_t full0 = smem_u32(&T.full[0]), empty0 = smem_u32(&T.empty[0]);
@@ -426,7 +604,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     }
     // slots no group of a unit writes (rows past N, columns past the last
     // slab's) must read as zero; the copier re-zeroes every slot it sums
-    for (int i = tid; i < NSTAGE * RB * MAX_C; i += G1_THREADS) (&T.slots[0][0])[i] = 0.f;
+    for (int i = tid; i < NSTAGE * NX * SLOT_FLOATS; i += G1_THREADS) (&T.slots[0][0][0])[i] = 0.f;
     __syncthreads();
     if (tid == 0) {
         const int first = n_units < NSTAGE ? n_units : NSTAGE;
@@ -439,7 +617,10 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     {
         const int64_t k0 = (int64_t)s0 * L.C * GROUP;
         const int lines = (min(L.C, L.G - s0 * L.C) * GROUP * 2 + 127) / 128;
-        if (tid >= 32 && tid - 32 < lines) prefetch_l2(x + k0 + (int64_t)(tid - 32) * 64);
+        if (tid >= 32 && tid - 32 < NX * lines) {
+            const int v = (tid - 32) / lines, ln = (tid - 32) - v * lines;
+            prefetch_l2(x + (int64_t)v * L.K + k0 + (int64_t)ln * 64);
+        }
     }
     // Ordering against the previous kernel on the stream (see Dep):
     if (dep != DEP_GROUP_FIRST) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -455,9 +636,12 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             epoch = ld_volatile(L.ctl) + 1u;
             const int z_end = min(u_end, L.nrb);
             for (int u = u_begin; u < z_end; ++u) {
-                float* dst = y + (int64_t)u * RB;
                 const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
-                for (int r = lane; r < rows; r += 32) dst[r] = 0.f;
+#pragma unroll
+                for (int v = 0; v < NX; ++v) {
+                    float* dst = y + (int64_t)v * L.N + (int64_t)u * RB;
+                    for (int r = lane; r < rows; r += 32) dst[r] = 0.f;
+                }
             }
             __syncwarp();
             if (lane == 0 && u_begin < z_end) {
@@ -476,11 +660,13 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         for (int j = 0; j < n_units; ++j) {
             if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 256)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
-                const uint32_t sl = smem_u32(T.slots[st]);
                 const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
-                float* yr = y + (int64_t)rbw * RB;
+#pragma unroll
+                for (int v = 0; v < NX; ++v)            // per vector: its slots into its row of y
 #pragma unroll
                 for (int q = 0; q < RB / 32; ++q) {
+                    const uint32_t sl = smem_u32(T.slots[st][v]);
+                    float* yr = y + (int64_t)v * L.N + (int64_t)rbw * RB;
                     // row r's 16 slots as four 16-byte chunks, chunk (k + (lane >> 1)) & 3
                     // at step k (each quarter-warp touches 8 distinct bank groups);
                     // summed as a tree, then zeroed for the stage's next unit
@@ -491,11 +677,11 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                     for (int k = 0; k < 4; ++k) a[k] = lds_f32x4(ra + (((k + (lane >> 1)) & 3) << 4));
 #pragma unroll
                     for (int k = 0; k < 4; ++k) sts_zero4(ra + (((k + (lane >> 1)) & 3) << 4));
-                    const float v = (((a[0].x + a[0].y) + (a[0].z + a[0].w)) + ((a[1].x + a[1].y) + (a[1].z + a[1].w))) +
-                                    (((a[2].x + a[2].y) + (a[2].z + a[2].w)) + ((a[3].x + a[3].y) + (a[3].z + a[3].w)));
+                    const float sum = (((a[0].x + a[0].y) + (a[0].z + a[0].w)) + ((a[1].x + a[1].y) + (a[1].z + a[1].w))) +
+                                      (((a[2].x + a[2].y) + (a[2].z + a[2].w)) + ((a[3].x + a[3].y) + (a[3].z + a[3].w)));
                     if (r < rows) {
-                        if (L.S == 1) yr[r] = v;
-                        else red_global(yr + r, v);
+                        if (L.S == 1) yr[r] = sum;
+                        else red_global(yr + r, sum);
                     }
                 }
                 __syncwarp();
@@ -536,36 +722,37 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         int cur = s0;
         int rbj = rb0 + team, sj = s0;                  // row block and slab of unit j
         while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
-        build_tables(T, L, x, s0, ct);
+        build_tables<NX>(T, L, x, s0, ct);
         for (int j = team; j < n_units; j += teams) {
             // every consumer warp rebuilds the tables at every slab boundary of the
             // block's range, in order (the rebuild's named barrier waits for all)
-            while (cur < sj) build_tables(T, L, x, ++cur, ct);
+            while (cur < sj) build_tables<NX>(T, L, x, ++cur, ct);
             const int st = j & (NSTAGE - 1);
             const uint32_t par = (uint32_t)(j / NSTAGE) & 1u;
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
                 // tasks rotate over the team's warps from unit to unit, so no warp always draws the costly ones
                 const int t0 = (wt - (j >> lg_teams)) & (tw - 1);
-                consume_unit(T, stage0 + st * STAGE_BYTES, L.C, min(L.C, L.G - sj * L.C), smem_u32(T.slots[st]), t0,
-                             tw, lane);
+                consume_unit<NX>(T, stage0 + st * STAGE_BYTES, L.C, min(L.C, L.G - sj * L.C), smem_u32(T.slots[st][0]),
+                                 t0, tw, lane);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty0 + 8 * st);
             }
             rbj += teams;
             while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
         }
-        while (cur < s_last) build_tables(T, L, x, ++cur, ct);   // boundaries past this team's last unit
+        while (cur < s_last) build_tables<NX>(T, L, x, ++cur, ct);   // boundaries past this team's last unit
     }
 }
 
 int g_sms = 0;
 
+template <int NX>
 cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s, int dep) {
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemv1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)GEMV1_SMEM);
+        cudaError_t e = cudaFuncSetAttribute(gemv1_kernel<NX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)gemv1_smem<NX>());
         if (e != cudaSuccess) return e;
         int dev = 0;
         if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
@@ -576,14 +763,14 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(G1_THREADS);
-    cfg.dynamicSmemBytes = GEMV1_SMEM;
+    cfg.dynamicSmemBytes = gemv1_smem<NX>();
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, gemv1_kernel, L, x, y, dep);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, gemv1_kernel<NX>, L, x, y, dep);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -623,7 +810,7 @@ cudaError_t launch_gemv1_static(const LayoutView& L, const uint16_t* x, float* y
     if ((e = cudaMemsetAsync(ctl + 1, 0, sizeof(uint32_t), s)) != cudaSuccess) return e;
     LayoutView Ls = L;
     Ls.ctl = ctl;
-    return launch_gemv1(Ls, x, y, s, DEP_BEFORE);
+    return launch_gemv1<1>(Ls, x, y, s, DEP_BEFORE);
 }
 
 // ---------------------------------------------------------------------------
@@ -668,18 +855,18 @@ cudaError_t launch_selftest_timeout(unsigned long long limit_ns, cudaStream_t s)
     return cudaGetLastError();
 }
 
-// Up to GEMV1_MAX_B rows run as that many batch-1 products: per row, the
-// batch-1 kernel's table lookups cost less than the batched kernel's
-// dequantisation into fragments and per-(row, group) epilogue (measured: B = 2
-// takes half the time this way, B = 3 three quarters; from B = 4 on the tensor
-// cores win).
-constexpr int GEMV1_MAX_B = 3;
+// Up to GEMV1_MAX_B rows run on the table kernel, two rows per launch (the
+// two-vector variant shares every lookup address and masked code between its
+// rows) plus one single row for an odd count: per row, table lookups cost less
+// than the batched kernel's dequantisation into fragments and per-(row, group)
+// epilogue at these sizes.
+constexpr int GEMV1_MAX_B = 4;
 
 cudaError_t launch_gemv_group(const LayoutView* const* Ls, const uint16_t* const* xs, float* const* ys, int count,
                               cudaStream_t s) {
     for (int i = 0; i < count; ++i) {
         const int dep = count == 1 ? DEP_BEFORE : i == 0 ? DEP_GROUP_FIRST : DEP_GROUP_NEXT;
-        const cudaError_t e = launch_gemv1(*Ls[i], xs[i], ys[i], s, dep);
+        const cudaError_t e = launch_gemv1<1>(*Ls[i], xs[i], ys[i], s, dep);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
@@ -687,10 +874,12 @@ cudaError_t launch_gemv_group(const LayoutView* const* Ls, const uint16_t* const
 
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
     if (B > GEMV1_MAX_B) return launch_gemm_small(L, X, Y, B, s);
-    for (int b = 0; b < B; ++b) {
-        const cudaError_t e = launch_gemv1(L, X + (int64_t)b * L.K, Y + (int64_t)b * L.N, s, DEP_BEFORE);
+    int b = 0;
+    for (; b + 2 <= B; b += 2) {
+        const cudaError_t e = launch_gemv1<2>(L, X + (int64_t)b * L.K, Y + (int64_t)b * L.N, s, DEP_BEFORE);
         if (e != cudaSuccess) return e;
     }
+    if (b < B) return launch_gemv1<1>(L, X + (int64_t)b * L.K, Y + (int64_t)b * L.N, s, DEP_BEFORE);
     return cudaSuccess;
 }
 
