@@ -16,7 +16,8 @@
 //                      ballot per task, see col_uniform).
 // The roles hand stages to one another through two mbarriers per stage
 // (full: blob landed; empty: the unit's team is done), so no block-wide
-// barrier sits in the steady state and up to NSTAGE units are in flight per SM. Block p owns a contiguous range of units in
+// barrier sits in the steady state and up to NSTAGE units are in flight per
+// SM. Block p owns a contiguous range of units in
 // slab-major order, so consecutive units share their activations; on a slab
 // change the consumer warps rebuild, under a named barrier of their own, the
 // per-slab activation tables: x as fp32 and, for every 4 consecutive weights of
@@ -32,9 +33,9 @@
 //   b = 8  same with a byte permute and 2^23 + 128.
 // X is summed from the tables in the same order as the lookups, so a group
 // whose codes are all at the zero level contributes exactly 0. Each group's
-// fp32 dot product is scaled once by its FP16 scale and added to its row's
-// shared-memory partial; a unit's rows then go to y directly (one slab per
-// row) or through atomics (several slabs).
+// fp32 dot product is scaled once by its FP16 scale and stored in its
+// (row, column) slot; the copier sums a row's slots in a fixed order and
+// writes y directly (one slab per row) or through atomics (several slabs).
 //
 // The same kernel takes two activation vectors per launch (NX = 2, batches of
 // 2..4 as one or two launches): the second vector's tables sit a fixed
