@@ -130,11 +130,13 @@ vbq_status_t vbq_gemv(const vbq_layout* layout, const uint16_t* x, float* y,
  *   Y  device, B x N floats, row-major; overwritten.
  *   B  1..16 (VBQ_ERR_UNSUPPORTED otherwise).
  * Same accuracy statement as vbq_gemv; the summation order is not fixed (results
- * can differ in the last bits between calls). For B <= 4 the rows run on the
+ * can differ in the last bits between calls). For B = 2..4 the library picks,
+ * from the layout's group count per width, the cheaper of two paths: the
  * batch-1 table kernel, two rows per launch (both rows share every lookup
- * address and decoded code) and a single row for an odd count; each row's
- * result is computed as vbq_gemv computes it. For B >= 5 the product runs on
- * the tensor cores:
+ * address and decoded code) and a single row for an odd count, each row
+ * computed as vbq_gemv computes it; or the tensor cores (chosen for layouts
+ * heavy in 4- and 8-bit groups). For B >= 5 the product runs on the tensor
+ * cores:
  * activations are scaled per (row, group column) by a power of two into fp16
  * range (values below 2^-14 of that scale lose low bits), weights enter as
  * exact levels, products and fp32 accumulation as in vbq_gemv. Y needs no

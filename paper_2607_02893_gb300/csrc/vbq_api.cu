@@ -225,6 +225,7 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     V.S = (int)S;
     V.nrb = (int)nrb;
     V.units = (int)units;
+    for (int w = 0; w < 4; ++w) V.items[w] = (int64_t)real_items[w];
     V.max_blob16 = (int)max16;
 
     if ((e = cudaMemsetAsync(L->base, 0, alloc_bytes, s)) != cudaSuccess) return bail(VBQ_ERR_CUDA, "memset", e);

@@ -66,6 +66,7 @@ struct LayoutView {
     int64_t N, K;
     int G, C, S, nrb, units;
     int max_blob16;             // largest blob, in 16-byte units
+    int64_t items[4];           // groups per width index (1, 2, 4, 8 bits): host-side launch choices
 };
 
 __host__ __device__ inline int width_of(int w) { return 1 << w; }
