@@ -8,9 +8,11 @@ after the previous one. Weights are random-but-seeded (synthetic) with the
 per-projection width distributions of the workload; every GEMV has its own
 resident BF16 activation vector.
 
-`modes` reports, for a stack workload at batch 1, three companions measured in
-the same run: `fused` (the <stack>-fused workload: QKV and gate-up as single
-matrices, 4 GEMVs per layer), `grouped` (the headline's layouts as one
+`modes` reports, for a stack workload at batch 1, companions measured in the
+same run: `grouped_by_input` (the headline's products in decode order, those
+that read the same input, Q/K/V and gate/up, issued as one vbq_gemv_group),
+`fused` (the <stack>-fused workload: QKV and gate-up as single matrices, 4
+GEMVs per layer), `grouped` (all of the headline's layouts as one
 vbq_gemv_group per step: independent products whose launches overlap, the
 streaming upper bound) and `cublas_bf16` (dense BF16 weights of the same
 shapes through torch.mv, i.e. cuBLAS, as a reference point).
@@ -321,6 +323,28 @@ def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev
     out["grouped"] = entry(ms, step_bytes, copies, len(layouts),
                            "the headline layouts as one vbq_gemv_group per step (independent products, "
                            "overlapping launches): the streaming upper bound")
+    # the decode order with products that read the same input issued as one
+    # group: per layer (Q, K, V) together, O, (gate, up) together, down
+    names = [m.name for m in work.mats] * copies
+    steps_list, i = [], 0
+    while i < len(names):
+        proj = names[i].rpartition(".")[2]
+        span = 3 if proj == "q" else 2 if proj == "gate" else 1
+        steps_list.append(list(range(i, i + span)))
+        i += span
+    if any(len(st) > 1 for st in steps_list):
+        def by_input():
+            for st in steps_list:
+                if len(st) == 1:
+                    vbq.vbq_gemv(layouts[st[0]], x0[st[0]], y0[st[0]], stream=stream)
+                else:
+                    xin = x0[st[0]]
+                    vbq.vbq_gemv_group([layouts[j] for j in st], [xin] * len(st), [y0[j] for j in st], stream=stream)
+        ms = time_graph(torch, stream, by_input, steps, warm)
+        out["grouped_by_input"] = entry(ms, step_bytes, copies, len(layouts),
+                                        "the headline's products in decode order, those that read the same input "
+                                        "(Q, K, V; gate, up) issued as one vbq_gemv_group: "
+                                        f"{len(steps_list)} dependent steps per token")
     name = args.workload
     if name in ("stack131m", "stack1b", "stack9b"):
         fwork = synth.workload(name + "-fused", 1)

@@ -177,8 +177,8 @@ vbq_status_t vbq_gemv_group(const vbq_layout* const* layouts, const uint16_t* co
  * allocation calls, or a host framework whose allocator must own every
  * device byte. This entry point allocates nothing, on the device or the host.
  * It runs the same batch-1 kernel as vbq_gemv, but keeps the kernel's split-K
- * control words (a call epoch, a finished-block count and one flag per row
- * block) in a fixed array inside this library instead of in the layout.
+ * control words (a call counter and one flag per row block) in a fixed array
+ * inside this library instead of in the layout.
  *
  *   layout  a layout with at most 8192 row blocks of 128 rows (N <= 1048576);
  *           larger layouts give VBQ_ERR_UNSUPPORTED.
@@ -188,10 +188,11 @@ vbq_status_t vbq_gemv_group(const vbq_layout* const* layouts, const uint16_t* co
  * library holds it until the process exits. The first call on a device looks
  * up the array's address with that device current, so make the first call
  * on each device before any stream capture. Every call on a device shares the
- * array and leaves its contents for the next call: the finished-block count
- * is cleared on `stream` before each launch, and the epoch only grows, so
- * flags left behind never match a later call. Calls that overlap on the GPU
- * race on the array: order them on one stream.
+ * array and leaves its contents for the next call: each call adds the same
+ * amount to the counter, whatever its grid, so the epoch its flags carry only
+ * grows and flags left behind never match a later call. Calls that overlap on
+ * the GPU race on the array: order them on one stream. Nothing is enqueued
+ * besides the kernel.
  */
 vbq_status_t vbq_gemv_static(const vbq_layout* layout, const uint16_t* x, float* y,
                              void* stream);

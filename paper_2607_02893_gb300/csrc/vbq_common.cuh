@@ -62,7 +62,7 @@ static_assert(sizeof(UnitHeader) == 48, "header is 48 bytes");
 struct LayoutView {
     const uint8_t* blobs;       // blob area
     const uint32_t* blob_off;   // units + 1 offsets, in 16-byte units
-    uint32_t* ctl;              // [0] call epoch, [1] blocks finished in this call, [2 + rb] y-zeroed flags
+    uint32_t* ctl;              // [0..1] 64-bit call counter (see call_epoch), [2 + rb] y-zeroed flags
     int64_t N, K;
     int G, C, S, nrb, units;
     int max_blob16;             // largest blob, in 16-byte units

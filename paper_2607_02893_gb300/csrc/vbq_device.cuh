@@ -106,13 +106,25 @@ __device__ __forceinline__ void prefetch_l2(const void* p) {
 __device__ __forceinline__ void fence_release_gpu() {
     asm volatile("fence.acq_rel.gpu;" ::: "memory");
 }
-// Atomic add with acquire-release ordering at GPU scope; returns the old value.
-__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
-    uint32_t old;
-    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
-    return old;
-}
 
+// Split-K call counter, control words 0-1 (one 64-bit word): every call adds
+// exactly 2^CALL_SHIFT in all, split over its blocks, so (counter >>
+// CALL_SHIFT) counts the calls before this one; a block that reads it while
+// other blocks of the same call have already added their shares still sees
+// fewer than 2^CALL_SHIFT of them. The call's epoch (the value its zeroed-row
+// flags carry) is that count + 1. The additions need no reply, so no block
+// waits on them before it exits.
+constexpr int CALL_SHIFT = 20;
+__device__ __forceinline__ uint32_t call_epoch(const uint32_t* ctl) {
+    unsigned long long c;
+    asm volatile("ld.volatile.global.u64 %0, [%1];" : "=l"(c) : "l"(ctl) : "memory");
+    return (uint32_t)(c >> CALL_SHIFT) + 1u;
+}
+__device__ __forceinline__ void call_done(uint32_t* ctl) {     // one thread per block, once per call
+    const unsigned long long q = (1ull << CALL_SHIFT) / gridDim.x;
+    const unsigned long long share = blockIdx.x == 0 ? (1ull << CALL_SHIFT) - q * (gridDim.x - 1) : q;
+    asm volatile("red.relaxed.gpu.global.add.u64 [%0], %1;" :: "l"(ctl), "l"(share) : "memory");
+}
 __device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) {
     return *reinterpret_cast<const volatile uint32_t*>(p);
 }

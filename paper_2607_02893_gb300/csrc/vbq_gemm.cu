@@ -356,7 +356,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
         // ---- copier: split-K zeroing, then per unit: rows out, next copy in ----
         uint32_t epoch = 0;
         if (L.S > 1) {
-            epoch = ld_volatile(L.ctl) + 1u;
+            epoch = call_epoch(L.ctl);
             const int z_end = min(u_end, L.nrb);
             for (int u = u_begin; u < z_end; ++u) {
                 const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
@@ -417,14 +417,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
                 mbar_wait_bounded(full0 + 8 * i, (uint32_t)((jl / NST) & 1));
             }
         }
-        if (L.S > 1 && lane == 0) {
-            // (acquire-release: this block's read of the epoch comes before its
-            // count, and the last block's epoch write after every count)
-            if (atom_add_acq_rel(L.ctl + 1, 1u) == gridDim.x - 1) {
-                st_volatile(L.ctl + 1, 0u);
-                st_volatile(L.ctl, epoch);
-            }
-        }
+        if (L.S > 1 && lane == 0) call_done(L.ctl);      // this block's share of the call count
     } else {
         // ---- consumers: team `team` takes units j = team, team + teams, ... ----
         const int cw = warp - 1, ct = tid - 32, team = cw / tw, wt = cw - team * tw;

@@ -634,7 +634,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         if (L.S > 1) {
             // this call's epoch; zero y for the row blocks whose slab 0 this block
             // owns (units u < nrb) and publish them
-            epoch = ld_volatile(L.ctl) + 1u;
+            epoch = call_epoch(L.ctl);
             const int z_end = min(u_end, L.nrb);
             for (int u = u_begin; u < z_end; ++u) {
                 const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
@@ -703,15 +703,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                 mbar_wait_bounded(full0 + 8 * i, (uint32_t)((jl / NSTAGE) & 1));
             }
         }
-        if (L.S > 1 && lane == 0) {
-            // the last block of the call advances the epoch for the next call
-            // (acquire-release: this block's read of the epoch comes before its
-            // count, and the last block's epoch write after every count)
-            if (atom_add_acq_rel(L.ctl + 1, 1u) == gridDim.x - 1) {
-                st_volatile(L.ctl + 1, 0u);
-                st_volatile(L.ctl, epoch);
-            }
-        }
+        if (L.S > 1 && lane == 0) call_done(L.ctl);      // this block's share of the call count
         // a grouped product that started without waiting completes only after
         // its predecessor, so completion stays in stream order
         if (dep == DEP_GROUP_NEXT && lane == 0) asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -782,10 +774,10 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
 // Batch 1 with the split-K control words in a fixed device array instead of
 // the layout's own allocation (for callers that cannot allocate device
 // memory; see vbq_gemv_static in vbq.h). Every call on a device shares the
-// array: word 0 is the call epoch, word 1 the count of finished blocks
-// (cleared on the stream before every launch), words 2.. the per-row-block
-// zeroed flags. Epochs only grow, so flags left by earlier calls never match
-// the current one. Calls that overlap on the GPU race on the array.
+// array: words 0-1 the call counter (each call adds exactly 2^CALL_SHIFT,
+// whatever its grid), words 2.. the per-row-block zeroed flags. Epochs only
+// grow, so flags left by earlier calls never match the current one. Calls
+// that overlap on the GPU race on the array.
 // ---------------------------------------------------------------------------
 
 static __device__ __align__(256) uint32_t g_static_ctl[STATIC_CTL_WORDS];
@@ -808,7 +800,6 @@ cudaError_t launch_gemv1_static(const LayoutView& L, const uint16_t* x, float* y
         }
         ctl = addr[dev];
     }
-    if ((e = cudaMemsetAsync(ctl + 1, 0, sizeof(uint32_t), s)) != cudaSuccess) return e;
     LayoutView Ls = L;
     Ls.ctl = ctl;
     return launch_gemv1<1>(Ls, x, y, s, DEP_BEFORE);
