@@ -659,7 +659,11 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         int st = 0, rbw = rb0, issued = n_units < NSTAGE ? n_units : NSTAGE;
         uint32_t par = 0;
         for (int j = 0; j < n_units; ++j) {
-            if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 256)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
+            // nap between polls, except on the block's last unit, whose rows end the block
+            if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, j + 1 < n_units ? 256 : 0)) {
+                dead = true;
+                if (lane == 0) raise_abort(&T.abort);
+            }
             if (!dead) {
                 const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
 #pragma unroll
