@@ -304,11 +304,14 @@ __device__ __forceinline__ void consumer_sync() {
 
 // Activations of slab s (per vector, for NX vectors stored K apart): x as fp32,
 // the pre-scaled x of the 4-bit slots, the nibble lookup tables, and the
-// per-column sums in lookup order. Consumer
-// threads only (ct = 0 .. NCT-1), one thread per (column, 4 weights): each
-// reads its 4 activations from global memory (L2), so the whole build is one
-// phase between two consumer barriers. The column sum of the all-ones entries
-// (xlut) is added over the column's half-warp in the pairs tree16x2 uses.
+// per-column sums in lookup order. Consumer threads only (ct = 0 .. NCT-1):
+// threads 0 .. 16 MAX_C - 1 one per (column, 4 weights), each reading its 4
+// activations from global memory (L2); the next 2 MAX_C threads one per
+// (column, half) for the 4-bit zero-level sums, reading their 32 activations
+// at the same time. So the whole build is one phase between two consumer
+// barriers. The column sum of the all-ones entries (xlut) is added over the
+// column's half-warp in the pairs tree16x2 uses.
+static_assert(NCT >= 16 * MAX_C + 2 * MAX_C, "threads for the tables and the zero-level sums");
 template <int NX>
 __device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t* __restrict__ x, int s, int ct) {
     const int cols = min(L.C, L.G - s * L.C);
@@ -348,31 +351,35 @@ __device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t
             sv += __shfl_xor_sync(half, sv, 4);
             sv += __shfl_xor_sync(half, sv, 8);
             if (jn == 0) T.xlut[v][c] = sv;
-            // X for the 4-bit zero level of half hh, summed as dot4_half accumulates
-            if ((jn & 7) == 0) {
-                const int hh = jn >> 3;
-                const uint4* src = reinterpret_cast<const uint4*>(xg + c * GROUP + 32 * hh);
-                float xh[32];
+        }
+    } else if (ct >= 16 * MAX_C && ct < 16 * MAX_C + cols * 2) {
+        // X for the 4-bit zero level of half hh of column c, summed as
+        // dot4_half accumulates (threads the lookup tables leave idle)
+        const int z = ct - 16 * MAX_C, c = z >> 1, hh = z & 1;     // c < cols, hh < 2
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint4 w = __ldg(src + q);
-                    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+        for (int v = 0; v < NX; ++v) {
+            const uint16_t* xg = x + (int64_t)v * L.K + (int64_t)s * L.C * GROUP;
+            const uint4* src = reinterpret_cast<const uint4*>(xg + c * GROUP + 32 * hh);
+            float xh[32];
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        xh[8 * q + 2 * i] = __uint_as_float(ws[i] << 16);
-                        xh[8 * q + 2 * i + 1] = __uint_as_float(ws[i] & 0xFFFF0000u);
-                    }
+            for (int q = 0; q < 4; ++q) {
+                const uint4 w = __ldg(src + q);
+                const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    xh[8 * q + 2 * i] = __uint_as_float(ws[i] << 16);
+                    xh[8 * q + 2 * i + 1] = __uint_as_float(ws[i] & 0xFFFF0000u);
                 }
-                float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
-#pragma unroll
-                for (int t4 = 0; t4 < 4; ++t4) {
-                    float2& cc = (t4 & 1) ? cb : ca;
-#pragma unroll
-                    for (int e = 0; e < 8; e += 2)
-                        cc = __ffma2_rn(f2(xh[8 * t4 + e], xh[8 * t4 + e + 1]), f2(0x1p-100f, 0x1p-100f), cc);
-                }
-                T.x4z[v][c][hh] = __fadd2_rn(ca, cb);
             }
+            float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
+#pragma unroll
+            for (int t4 = 0; t4 < 4; ++t4) {
+                float2& cc = (t4 & 1) ? cb : ca;
+#pragma unroll
+                for (int e = 0; e < 8; e += 2)
+                    cc = __ffma2_rn(f2(xh[8 * t4 + e], xh[8 * t4 + e + 1]), f2(0x1p-100f, 0x1p-100f), cc);
+            }
+            T.x4z[v][c][hh] = __fadd2_rn(ca, cb);
         }
     }
     consumer_sync();
