@@ -103,8 +103,17 @@ __device__ __forceinline__ void prefetch_l2(const void* p) {
 // Order this thread's earlier writes (and those it has observed) before its
 // later ones, GPU-wide: the release half of __threadfence, without waiting for
 // sequential consistency.
-__device__ __forceinline__ void fence_release_gpu() {
-    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+// Release store / acquire load at GPU scope: the split-K zeroed-row flags.
+// A warp's zero stores, ordered before lane 0 by the warp barrier, are visible
+// to whoever acquires the flag; the acquiring lanes order the warp's later
+// additions after it by another warp barrier.
+__device__ __forceinline__ void st_release_gpu(uint32_t* p, uint32_t v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
 }
 
 // Split-K call counter, control words 0-1 (one 64-bit word): every call adds
@@ -125,13 +134,6 @@ __device__ __forceinline__ void call_done(uint32_t* ctl) {     // one thread per
     const unsigned long long share = blockIdx.x == 0 ? (1ull << CALL_SHIFT) - q * (gridDim.x - 1) : q;
     asm volatile("red.relaxed.gpu.global.add.u64 [%0], %1;" :: "l"(ctl), "l"(share) : "memory");
 }
-__device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) {
-    return *reinterpret_cast<const volatile uint32_t*>(p);
-}
-__device__ __forceinline__ void st_volatile(uint32_t* p, uint32_t v) {
-    *reinterpret_cast<volatile uint32_t*>(p) = v;
-}
-
 __device__ __forceinline__ float half_bits(uint32_t bits) { return __half2float(__ushort_as_half((uint16_t)bits)); }
 
 // ---------------------------------------------------------------------------
@@ -239,7 +241,7 @@ __device__ __forceinline__ int col_within(uint32_t ce, int cf, int cl, int i) { 
 // Split-K: true once every row block this block adds a slab s > 0 into has
 // been zeroed in this call (flag == epoch), within the wait limit. A whole warp:
 // lane i watches units u_begin + i, + 32, ..., so one round trip covers them
-// all; ends with an acquire fence.
+// all; the flags are read with acquire loads.
 __device__ __forceinline__ bool split_k_flags_ready(const LayoutView& L, uint32_t epoch, int u_begin, int u_end,
                                                     int lane) {
     bool seen = true;
@@ -247,11 +249,11 @@ __device__ __forceinline__ bool split_k_flags_ready(const LayoutView& L, uint32_
     for (int u = u_begin + lane; u < u_end && seen; u += 32) {
         if (u >= L.nrb) {               // slab > 0
             const uint32_t* f = L.ctl + 2 + (u % L.nrb);
-            while (!(seen = ld_volatile(f) == epoch))
+            while (!(seen = ld_acquire_gpu(f) == epoch))
                 if (global_ns() - t0 > WAIT_LIMIT_NS) break;
         }
     }
-    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+    __syncwarp();                       // every lane's later additions after every acquire
     return __all_sync(0xffffffffu, seen);
 }
 

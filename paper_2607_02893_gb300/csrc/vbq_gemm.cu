@@ -367,8 +367,8 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             }
             __syncwarp();
             if (lane == 0 && u_begin < z_end) {
-                fence_release_gpu();        // the zeros before the flags
-                for (int u = u_begin; u < z_end; ++u) st_volatile(L.ctl + 2 + u, epoch);
+                // release stores: the warp's zeros (ordered by __syncwarp) before the flags
+                for (int u = u_begin; u < z_end; ++u) st_release_gpu(L.ctl + 2 + u, epoch);
             }
         }
         bool dead = false;
