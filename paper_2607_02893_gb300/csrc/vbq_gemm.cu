@@ -366,10 +366,9 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
                 }
             }
             __syncwarp();
-            if (lane == 0 && u_begin < z_end) {
-                // release stores: the warp's zeros (ordered by __syncwarp) before the flags
-                for (int u = u_begin; u < z_end; ++u) st_release_gpu(L.ctl + 2 + u, epoch);
-            }
+            // release stores, one unit per lane in parallel: the warp's zeros
+            // (ordered by __syncwarp) before each flag
+            for (int u = u_begin + lane; u < z_end; u += 32) st_release_gpu(L.ctl + 2 + u, epoch);
         }
         bool dead = false;
         if (L.S > 1 && !split_k_flags_ready(L, epoch, u_begin, u_end, lane)) {
