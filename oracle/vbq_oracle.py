@@ -29,7 +29,10 @@ Readings of points the paper leaves open (each also listed in the design notes):
 * sign(0) = +1 (one bit cannot encode zero).
 * The scale is computed in fp64, rounded to FP16 (round to nearest even),
   and the codes are computed with the rounded scale; clip absorbs overshoot.
-  Scales above 65504 saturate to 65504.
+  Scales above 65504 saturate to 65504. The 1-bit mean sums |w| in fp64 as a
+  balanced pairwise tree over neighbouring weights (pairwise_sum), then
+  divides by the group size. NaN weights are rejected; +-inf quantise like
+  any value above the saturated scale.
 * An all-zero group (or one whose scale rounds to 0) gets s = 0 and codes
   u = 2^(b-1) (b >= 2) or u = 1 (b = 1); it dequantises to zeros.
 * Activations are BF16; the reference product is exact-input fp64:
@@ -127,15 +130,33 @@ def _to_fp16_scale(s: float) -> np.float16:
     return np.float16(s)
 
 
+def pairwise_sum(v) -> float:
+    """fp64 sum of v as a balanced tree over neighbours: (v0 + v1), (v2 + v3),
+    ... then pairs of those, and so on (an odd element is carried up a level).
+    The paper fixes the mean of the 1-bit rule, not a summation order; this is
+    the order the quantiser uses, written out."""
+    level = [float(t) for t in v]
+    if not level:
+        return 0.0
+    while len(level) > 1:
+        nxt = [level[i] + level[i + 1] for i in range(0, len(level) - 1, 2)]
+        if len(level) % 2:
+            nxt.append(level[-1])
+        level = nxt
+    return level[0]
+
+
 def quantize_group(w, b: int, fp16_scale: bool = True):
     """Quantise one group of weights at width b.
 
     Returns (codes uint8[len(w)], scale) where scale is np.float16 if
-    fp16_scale else the unrounded fp64 value.
+    fp16_scale else the unrounded fp64 value. NaN weights are rejected.
     """
     w = np.asarray(w, dtype=np.float64)
+    if np.isnan(w).any():
+        raise ValueError("NaN weight")
     if b == 1:
-        s = float(np.mean(np.abs(w)))
+        s = pairwise_sum(np.abs(w)) / w.size if w.size else 0.0
         s_used = _to_fp16_scale(s) if fp16_scale else s
         codes = (w >= 0).astype(np.uint8)          # sign(0) = +1
         return codes, s_used

@@ -117,6 +117,25 @@ def pin_quantizer_invariants(O, seed=2):
         _check(float(s) == float(np.float16(np.mean(np.abs(w)))), "1-bit scale != mean|w|")
 
 
+def pin_one_bit_mean_order(O):
+    """The 1-bit scale is FP16(mean |w|) (§3.1) with the mean summed as a
+    balanced fp64 tree. Hand-derived case where the order decides the FP16 bits:
+    w0 = 1 + 2^-11 (the FP16 midpoint between 1 and 1 + 2^-10, times 64 later)
+    and 63 weights of 2^-54. Exactly, sum = 1 + 2^-11 + 63 * 2^-54, above the
+    midpoint, so FP16(sum / 64) = 2^-6 (1 + 2^-10) = 0x2401. The tree loses
+    the first 2^-54 (w0 + w1 rounds to w0), and (w0 + w1) + (w2 + w3) is a tie
+    that rounds to even (w0); then it adds 2^-52, 2^-51, 2^-50 and 2^-49
+    exactly: 1 + 2^-11 + 15 * 2^-52, still above the midpoint: 0x2401. A
+    left-to-right sum loses every 2^-54 (each is below half an ulp of 1),
+    lands on the midpoint and rounds to even: 0x2400."""
+    w = np.full(64, 2.0 ** -54)
+    w[0] = 1.0 + 2.0 ** -11
+    codes, s = O.quantize_group(w, 1)
+    _check(int(np.float16(s).view(np.uint16)) == 0x2401, f"1-bit mean order: scale {np.float16(s)}")
+    _check(np.array_equal(codes, np.ones(64, np.uint8)), "1-bit mean order: codes")
+    _check(O.pairwise_sum([1.0, 2.0, 3.0]) == 6.0 and O.pairwise_sum([]) == 0.0, "pairwise_sum edge cases")
+
+
 def pin_group_size_one(O, seed=3):
     """§3.1: with one weight per group every width reconstructs w exactly
     (unrounded scale)."""
@@ -212,5 +231,5 @@ def pin_payload_accounting(O, seed=6):
 
 
 ALL_PINS = [pin_eq1_golden, pin_level_grid, pin_grid_roundtrip, pin_quantizer_invariants,
-            pin_group_size_one, pin_integer_gemv, pin_exact_rational, pin_enumerated_codes,
+            pin_one_bit_mean_order, pin_group_size_one, pin_integer_gemv, pin_exact_rational, pin_enumerated_codes,
             pin_payload_accounting]

@@ -49,7 +49,9 @@ MUTATIONS = {
     "unrounded_scale_for_codes": ("sf = float(s_used)", "sf = float(s)"),
     "qmax_too_large": ("qmax = (1 << (b - 1)) - 1\n    z = 1 << (b - 1)\n    m =",
                        "qmax = (1 << (b - 1))\n    z = 1 << (b - 1)\n    m ="),
-    "one_bit_max_scale": ("s = float(np.mean(np.abs(w)))", "s = float(np.max(np.abs(w)))"),
+    "one_bit_max_scale": ("s = pairwise_sum(np.abs(w)) / w.size", "s = float(np.max(np.abs(w))) / 1.0"),
+    "one_bit_sequential_sum": ("s = pairwise_sum(np.abs(w)) / w.size",
+                               "s = float(np.cumsum(np.abs(w))[-1]) / w.size"),
     "sign_zero_negative": ("codes = (w >= 0).astype(np.uint8)", "codes = (w > 0).astype(np.uint8)"),
     "pack_msb_first": ("acc |= int(codes[r, g * GROUP + i]) << (i * b)",
                        "acc |= int(codes[r, g * GROUP + i]) << ((GROUP - 1 - i) * b)"),
