@@ -373,6 +373,35 @@ def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev
                                "value counts the BF16 weight bytes it streams")
     del dense, dx, dy
     torch.cuda.empty_cache()
+    # the export step: vbq_quantize of the stack's largest non-head matrix,
+    # whole calls (device validation, host read-back of its flags, then the
+    # quantisation kernel), timed with events on the stream
+    cands = [m for m in work.mats if not m.name.startswith("head")] or list(work.mats)
+    big = max(cands, key=lambda m: m.n * m.k)
+    w = torch.randn((big.n, big.k), generator=g, device=dev, dtype=torch.float32) * 0.02
+    wd = torch.tensor([1, 2, 4, 8], dtype=torch.uint8, device=dev)[
+        torch.multinomial(torch.tensor(synth.DIST_MAIN, device=dev), big.n * (big.k // 64), replacement=True,
+                          generator=g)].reshape(big.n, big.k // 64)
+    qc = torch.empty((big.n, big.k), dtype=torch.uint8, device=dev)
+    qs = torch.empty((big.n, big.k // 64), dtype=torch.int16, device=dev)
+    for _ in range(3):
+        vbq.vbq_quantize(w, wd, qc, qs, stream=stream)
+    reps = 10
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        vbq.vbq_quantize(w, wd, qc, qs, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    qms = e0.elapsed_time(e1) / reps
+    qbytes = big.n * big.k * 5 + (big.n * big.k // 64) * 3      # fp32 in, codes out; width in, scale out
+    out["quantize"] = {"ms_per_call": round(qms, 4), "value": round(qbytes / (qms * 1e-3) / 1e9, 1), "unit": "GB/s",
+                       "weights_per_s": round(big.n * big.k / (qms * 1e-3), 1), "shape": [big.n, big.k],
+                       "note": "vbq_quantize (Eq. 1 / 1-bit absmean per group) of an FP32 matrix at the main width "
+                               "mix, whole calls: device validation pass and its flag read-back, then the "
+                               "quantisation kernel; value counts 4 B in and 1 B out per weight"}
+    del w, wd, qc, qs
+    torch.cuda.empty_cache()
     return out
 
 

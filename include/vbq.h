@@ -58,6 +58,37 @@ enum {
 typedef struct vbq_layout vbq_layout;
 
 /*
+ * vbq_quantize — quantise a dense matrix group by group (§3.1), the step that
+ * produces vbq_pack's inputs (§6 export).
+ *
+ *   w           device, N x K float32, row-major. +-inf allowed, NaN is
+ *               VBQ_ERR_ARG.
+ *   bitwidths   device, N x (K/64) uint8, each in {1, 2, 4, 8}
+ *               (VBQ_ERR_WIDTH otherwise).
+ *   N, K        K % 64 == 0, N * K <= 2^40.
+ *   codes_out   device, N x K uint8: the codes vbq_pack takes.
+ *   scales_out  device, N x (K/64) FP16 bit patterns.
+ *   stream      stream for the device work.
+ *
+ * Per group of 64 weights w_j at width b (FP16() rounds to nearest even and
+ * saturates above 65504 to 65504):
+ *   b >= 2 (Eq. 1): qmax = 2^(b-1) - 1, s = FP16(max_j |w_j| / qmax) with the
+ *          quotient in fp64; q_j = clip(round(w_j / s), -qmax, qmax), round
+ *          half to even of the exact quotient; u_j = q_j + 2^(b-1). A group
+ *          whose s is 0 gets u_j = 2^(b-1).
+ *   b = 1  (absmean sign rule): s = FP16(mean_j |w_j|), the sum of |w_j| in
+ *          fp64 as a balanced pairwise tree over neighbouring weights
+ *          ((|w_0| + |w_1|) + (|w_2| + |w_3|), ...); u_j = 1 if w_j >= 0
+ *          (including -0), else 0.
+ * So codes and scales are a pure function of w and the widths. The call
+ * validates widths and NaNs on the device first and synchronises `stream`
+ * (outputs are untouched on an error), then enqueues the quantisation and
+ * returns without waiting. It allocates a 4-byte temporary.
+ */
+vbq_status_t vbq_quantize(const float* w, const uint8_t* bitwidths, int64_t N, int64_t K,
+                          uint8_t* codes_out, uint16_t* scales_out, void* stream);
+
+/*
  * vbq_pack — build the packed device layout of one matrix (§6: the export
  * step that turns per-group codes into packed storage; §3.1 groups of 64).
  *

@@ -257,6 +257,35 @@ vbq_status_t vbq_layout_shape(const vbq_layout* L, int64_t* N, int64_t* K) {
     return VBQ_OK;
 }
 
+vbq_status_t vbq_quantize(const float* w, const uint8_t* bitwidths, int64_t N, int64_t K, uint8_t* codes_out,
+                          uint16_t* scales_out, void* stream) {
+    g_err[0] = 0;
+    if (!w || !bitwidths || !codes_out || !scales_out)
+        return fail(VBQ_ERR_ARG, "w, bitwidths, codes_out and scales_out must be non-NULL");
+    if (N < 1 || K < vbq::GROUP || K % vbq::GROUP != 0)
+        return fail(VBQ_ERR_SHAPE, "need N >= 1 and K a positive multiple of 64 (N=%lld K=%lld)",
+                    (long long)N, (long long)K);
+    if (N > (1LL << 40) / K) return fail(VBQ_ERR_UNSUPPORTED, "N x K above 2^40 weights");
+    if (!aligned16(w) || !aligned16(bitwidths) || !aligned16(codes_out) || !aligned16(scales_out))
+        return fail(VBQ_ERR_ALIGN, "device arrays must be 16-byte aligned");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    // the flag word is a stream-ordered allocation (no device-wide sync on free)
+    void* d_err = nullptr;
+    VBQ_CUDA(cudaMallocAsync(&d_err, sizeof(uint32_t), s));
+    uint32_t h_err = 0;
+    cudaError_t e = cudaMemsetAsync(d_err, 0, sizeof(uint32_t), s);
+    if (e == cudaSuccess) e = vbq::launch_quant_validate(w, bitwidths, N, K, static_cast<uint32_t*>(d_err), s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&h_err, d_err, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
+    const cudaError_t ef = cudaFreeAsync(d_err, s);
+    if (e == cudaSuccess) e = ef;
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    VBQ_CUDA(e);
+    if (h_err & 1u) return fail(VBQ_ERR_WIDTH, "a bit-width is not in {1,2,4,8}");
+    if (h_err & 2u) return fail(VBQ_ERR_ARG, "a weight is NaN");
+    VBQ_CUDA(vbq::launch_quantize(w, bitwidths, N, K, codes_out, scales_out, s));
+    return VBQ_OK;
+}
+
 vbq_status_t vbq_dequant(const vbq_layout* L, uint8_t* codes_out, uint8_t* bitwidths_out,
                          uint16_t* scales_out, float* w_out, void* stream) {
     g_err[0] = 0;

@@ -18,6 +18,13 @@ cudaError_t launch_scatter(const uint8_t* codes, const uint8_t* widths, const ui
 cudaError_t launch_dequant(const LayoutView& L, uint8_t* codes_out, uint8_t* widths_out,
                            uint16_t* scales_out, float* w_out, cudaStream_t s);
 
+// Quantisation (vbq_quant.cu): validation (bit 0 of err: a width outside
+// {1,2,4,8}; bit 1: a NaN weight), then codes and FP16 scales per group.
+cudaError_t launch_quant_validate(const float* w, const uint8_t* widths, int64_t N, int64_t K, uint32_t* err,
+                                  cudaStream_t s);
+cudaError_t launch_quantize(const float* w, const uint8_t* widths, int64_t N, int64_t K, uint8_t* codes,
+                            uint16_t* scales, cudaStream_t s);
+
 // Products (vbq_gemv.cu). Y is B x N, overwritten (no zeroing needed).
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s);
 

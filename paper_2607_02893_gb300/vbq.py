@@ -28,6 +28,7 @@ _I = ctypes.c_int
 _SZP = ctypes.POINTER(ctypes.c_size_t)
 _I64P = ctypes.POINTER(ctypes.c_int64)
 SIGNATURES = {
+    "vbq_quantize": (_I, [_P, _P, _I64, _I64, _P, _P, _P]),
     "vbq_pack": (_I, [_P, _P, _P, _I64, _I64, _I, _P, ctypes.POINTER(_P)]),
     "vbq_packed_bytes": (_I, [_P, _SZP, _SZP, _SZP]),
     "vbq_layout_shape": (_I, [_P, _I64P, _I64P]),
@@ -121,6 +122,21 @@ class Layout:
         if not self.handle:
             raise ValueError("layout already freed")
         return ctypes.c_void_p(self.handle)
+
+
+def vbq_quantize(w, bitwidths, codes_out=None, scales_out=None, stream=None):
+    """Quantise w (N x K float32, device) at per-group widths (N x K/64 uint8,
+    device) into codes (N x K uint8) and FP16 scale bit patterns (N x K/64,
+    int16 storage); returns (codes, scales). Outputs are allocated when not given."""
+    import torch
+    n, k = int(w.shape[0]), int(w.shape[1])
+    if codes_out is None:
+        codes_out = torch.empty((n, k), dtype=torch.uint8, device=w.device)
+    if scales_out is None:
+        scales_out = torch.empty((n, k // 64), dtype=torch.int16, device=w.device)
+    _check(load().vbq_quantize(_ptr(w), _ptr(bitwidths), n, k, _ptr(codes_out), _ptr(scales_out),
+                               _stream(stream, w)))
+    return codes_out, scales_out
 
 
 def vbq_pack(codes, bitwidths, scales_fp16, N: Optional[int] = None, K: Optional[int] = None,

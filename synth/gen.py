@@ -43,6 +43,17 @@ def draw_scales(n: int, g: int, rng: np.random.Generator) -> np.ndarray:
     return (np.abs(rng.normal(0.0, 0.02, size=(n, g))) + 1e-4).astype(np.float16)
 
 
+def draw_dense_weights(n: int, k: int, rng: np.random.Generator) -> np.ndarray:
+    """Dense float32 weights for the quantiser: N(0, 0.02) scaled per 64-column
+    group by exp(N(0, 0.5)) (groups of different magnitude), with 1% of the
+    weights eight times larger (outliers)."""
+    g = k // 64
+    w = rng.normal(0.0, 0.02, size=(n, k))
+    w *= np.repeat(np.exp(rng.normal(0.0, 0.5, size=(n, g))), 64, axis=1)
+    w *= np.where(rng.random((n, k)) < 0.01, 8.0, 1.0)
+    return w.astype(np.float32)
+
+
 def f32_to_bf16_bits(a: np.ndarray) -> np.ndarray:
     """Round float32 values to bfloat16 (round to nearest even); return the bit patterns."""
     bits = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)

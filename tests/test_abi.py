@@ -67,6 +67,19 @@ def test_pack_rejects_bad_arguments_on_host(lib):
     assert b"16-byte" in lib.vbq_last_error()
 
 
+def test_quantize_rejects_bad_arguments_on_host(lib):
+    buf = ctypes.create_string_buffer(256)
+    p = (ctypes.addressof(buf) + 15) // 16 * 16
+    assert lib.vbq_quantize(None, p, 1, 64, p, p, None) == -1            # w NULL
+    assert lib.vbq_quantize(p, p, 1, 64, p, None, None) == -1            # scales NULL
+    assert lib.vbq_quantize(p, p, 0, 64, p, p, None) == -2               # N < 1
+    assert lib.vbq_quantize(p, p, 2, 96, p, p, None) == -2               # K % 64
+    assert lib.vbq_quantize(p, p, 1 << 30, 1 << 20, p, p, None) == -7    # over 2^40 weights
+    assert lib.vbq_quantize(p + 4, p, 1, 64, p, p, None) == -5           # misaligned
+    assert lib.vbq_quantize(p, p, 1, 64, p + 2, p, None) == -5
+    assert b"16-byte" in lib.vbq_last_error()
+
+
 def test_calls_reject_null_layout(lib):
     assert lib.vbq_gemv(None, None, None, None) == -1
     assert lib.vbq_gemm_small(None, None, None, 4, None) == -1
