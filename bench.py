@@ -356,6 +356,17 @@ def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev
                              "workload " + name + "-fused: QKV and gate-up as single matrices, layer-serial")
         del flays, fxs, fys
         torch.cuda.empty_cache()
+        rwork = synth.workload(name + "-recipe", 1)
+        rlays, rxs, rys, rnb, _, rcp = setup_stack(rwork, 1, dev, min_bytes=3 * l2)
+        ms = time_graph(torch, stream,
+                        lambda: [vbq.vbq_gemv(l, x[0], y[0], stream=stream) for l, x, y in zip(rlays, rxs, rys)],
+                        steps, warm)
+        out["recipe"] = entry(ms, sum(rnb), rcp, len(rlays),
+                              "workload " + name + "-recipe: the fixed recipe's widths (§3.4; layer-0 MLP "
+                              "4-bit, other projections 2-bit, head tiered per row, mean 1.18 bits), "
+                              "layer-serial, same shapes as the headline")
+        del rlays, rxs, rys
+        torch.cuda.empty_cache()
     # dense BF16 reference: the same shapes, one copy per packed copy so the
     # weights stream from HBM too
     g = torch.Generator(device=dev)
@@ -696,7 +707,7 @@ def algorithmic_bytes_est(spec, batch: int) -> int:
     """Algorithmic bytes of one matrix from its drawn widths."""
     from synth import gen
     rng = gen.rng_for(spec.seed_path)
-    widths = gen.draw_widths(spec.n, spec.k // 64, spec.dist, rng)
+    widths = gen.spec_widths(spec, rng)
     return algorithmic_bytes(widths, spec.n, spec.k, batch)
 
 

@@ -13,5 +13,5 @@ from .workloads import (  # noqa: F401
 )
 from .gen import (  # noqa: F401
     draw_widths, draw_scales, draw_x_bf16, bf16_bits_to_f32, f32_to_bf16_bits,
-    code_key, codes_torch, matrix_inputs, fmix32_py,
+    code_key, codes_torch, matrix_inputs, fmix32_py, tiered_widths, spec_widths,
 )

@@ -3,6 +3,8 @@
 Draw order per matrix, from one PCG64 stream seeded by
 SeedSequence([0, config_id, layer, proj_id]):
   1. widths  rng.choice([1,2,4,8], size=(N, G), p=dist)           (uint8)
+             (a tiered matrix, the recipe's head, draws nothing here: its
+             widths are fixed per row by tier)
   2. scales  |rng.normal(0, 0.02, (N, G))| + 1e-4 -> float16 (RNE)  (float16)
   3. x       rng.normal(0, 1, (B, K)) float32 -> bfloat16 (RNE)     (uint16 bits)
 
@@ -132,11 +134,34 @@ def codes_torch(widths, key: int, k: int, row0: int = 0, nrows: Optional[int] = 
     return out
 
 
+def tiered_widths(n: int, g: int, tiers) -> np.ndarray:
+    """Per-row widths from (cumulative fraction of rows, width) tiers in row
+    order, every group of a row at its row's width. Tier boundaries are
+    round(fraction * n)."""
+    w = np.empty(n, dtype=np.uint8)
+    start = 0
+    for frac, b in tiers:
+        end = n if frac >= 1.0 else min(n, int(round(frac * n)))
+        w[start:end] = b
+        start = max(start, end)
+    return np.repeat(w[:, None], g, axis=1)
+
+
+def spec_widths(spec, rng: np.random.Generator) -> np.ndarray:
+    """A matrix's widths: per-row tiers when the spec has them (no random
+    draw), else drawn i.i.d. per group from its distribution."""
+    g = spec.k // 64
+    tiers = getattr(spec, "tiers", None)
+    if tiers:
+        return tiered_widths(spec.n, g, tiers)
+    return draw_widths(spec.n, g, spec.dist, rng)
+
+
 def matrix_inputs(spec, batch: int):
     """Widths, scales and x of one matrix (numpy), plus its code key."""
     rng = rng_for(spec.seed_path)
     g = spec.k // 64
-    widths = draw_widths(spec.n, g, spec.dist, rng)
+    widths = spec_widths(spec, rng)
     scales = draw_scales(spec.n, g, rng)
     x_bits = draw_x_bf16(batch, spec.k, rng)
     return {"widths": widths, "scales": scales, "x_bits": x_bits,

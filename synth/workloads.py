@@ -23,7 +23,7 @@ Bit-width distributions are probabilities over widths (1, 2, 4, 8):
 from __future__ import annotations
 
 from dataclasses import dataclass, field
-from typing import List, Tuple
+from typing import Optional, List, Tuple
 
 WIDTHS = (1, 2, 4, 8)
 
@@ -43,12 +43,18 @@ SWEEP_DISTS = {
 
 @dataclass(frozen=True)
 class MatrixSpec:
-    """One weight matrix of a workload: W is n x k, groups of 64 along k."""
+    """One weight matrix of a workload: W is n x k, groups of 64 along k.
+
+    Widths are drawn i.i.d. per group from dist, unless tiers is set: then
+    every group of a row takes its row's tier width, tiers given as
+    (cumulative fraction of rows, width) in row order (the recipe's
+    frequency-tiered head, rows sorted by token frequency)."""
     name: str
     n: int
     k: int
     dist: Tuple[float, float, float, float]
     seed_path: Tuple[int, ...]   # (config_id, layer, proj_id) for the seed sequence
+    tiers: Optional[Tuple[Tuple[float, int], ...]] = None
 
 
 @dataclass
@@ -63,32 +69,44 @@ class Workload:
         return sum(m.n * m.k for m in self.mats)
 
 
+# The fixed VBQ recipe (§3.4): the first block's MLP at 4 bits, every other
+# projection at 2 bits, the LM head tiered per row by token-frequency rank:
+# top 0.5% of rows at 8 bits, next 1.5% at 4, next 10% at 2, the last 88% at 1.
+RECIPE_HEAD_TIERS = ((0.005, 8), (0.02, 4), (0.12, 2), (1.0, 1))
+
+
 def _stack(config_id: int, d_model: int, n_layers: int, d_q: int, d_kv: int,
-           d_ff: int, vocab: int, fused: bool = False) -> List[MatrixSpec]:
+           d_ff: int, vocab: int, fused: bool = False, recipe: bool = False) -> List[MatrixSpec]:
     mats: List[MatrixSpec] = []
+    if recipe:
+        config_id += 100            # its own seeds
+    main = DIST_ALL2 if recipe else DIST_MAIN
     for layer in range(n_layers):
-        mlp = DIST_MLP0 if layer == 0 else DIST_MAIN
+        mlp = (DIST_ALL4 if recipe else DIST_MLP0) if layer == 0 else main
         # (name, n, k, dist, proj_id)
         if fused:
             projs = [
-                ("qkv", d_q + 2 * d_kv, d_model, DIST_MAIN, 7),
-                ("o", d_model, d_q, DIST_MAIN, 3),
+                ("qkv", d_q + 2 * d_kv, d_model, main, 7),
+                ("o", d_model, d_q, main, 3),
                 ("gate_up", 2 * d_ff, d_model, mlp, 8),
                 ("down", d_model, d_ff, mlp, 6),
             ]
         else:
             projs = [
-                ("q", d_q, d_model, DIST_MAIN, 0),
-                ("k", d_kv, d_model, DIST_MAIN, 1),
-                ("v", d_kv, d_model, DIST_MAIN, 2),
-                ("o", d_model, d_q, DIST_MAIN, 3),
+                ("q", d_q, d_model, main, 0),
+                ("k", d_kv, d_model, main, 1),
+                ("v", d_kv, d_model, main, 2),
+                ("o", d_model, d_q, main, 3),
                 ("gate", d_ff, d_model, mlp, 4),
                 ("up", d_ff, d_model, mlp, 5),
                 ("down", d_model, d_ff, mlp, 6),
             ]
         for pname, n, k, dist, pid in projs:
             mats.append(MatrixSpec(f"l{layer}.{pname}", n, k, dist, (config_id, layer, pid)))
-    mats.append(MatrixSpec("head", vocab, d_model, DIST_HEAD, (config_id, n_layers, 0)))
+    if recipe:
+        mats.append(MatrixSpec("head", vocab, d_model, DIST_HEAD, (config_id, n_layers, 0), RECIPE_HEAD_TIERS))
+    else:
+        mats.append(MatrixSpec("head", vocab, d_model, DIST_HEAD, (config_id, n_layers, 0)))
     return mats
 
 
@@ -108,12 +126,17 @@ def workload(name: str, batch: int = 1) -> Workload:
     stack1b     d_model 2048, 22 layers, Q/O 2048, K/V 256, MLP 5632, head 32000 (155 GEMVs).
     stack9b     d_model 4096, 32 layers, Q/O 4096, K/V 1024, MLP 14336, head 128256 (225 GEMVs).
     <stack>-fused   the same stack with QKV and gate-up fused (131m: 49, 1b: 89, 9b: 129 GEMVs).
+    <stack>-recipe  the same shapes with the fixed recipe's widths (§3.4): layer-0 MLP all
+                    4-bit, other projections all 2-bit, head tiered per row (mean 1.18 bits).
     sweep:<n>:<dist>  one n x n GEMV, dist in all1/all2/all4/all8/mixed.
     matrix:<n>:<k>:<dist>  one n x k GEMV (for profiling single shapes).
     """
     if name.endswith("-fused") and name[:-6] in _STACKS:
         cid, dims = _STACKS[name[:-6]]
         return Workload(name, cid, batch, _stack(cid, *dims, fused=True))
+    if name.endswith("-recipe") and name[:-7] in _STACKS:
+        cid, dims = _STACKS[name[:-7]]
+        return Workload(name, cid, batch, _stack(cid, *dims, recipe=True))
     if name in _STACKS:
         cid, dims = _STACKS[name]
         return Workload(name, cid, batch, _stack(cid, *dims))

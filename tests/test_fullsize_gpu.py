@@ -49,7 +49,8 @@ def _pack(spec, inp):
 
 
 @pytest.mark.parametrize("name", ["single768", "stack131m", "stack1b", "stack9b",
-                                  "stack131m-fused", "stack1b-fused", "stack9b-fused"])
+                                  "stack131m-fused", "stack1b-fused", "stack9b-fused",
+                                  "stack131m-recipe", "stack1b-recipe", "stack9b-recipe"])
 def test_stack_fullsize_sampled(name):
     work = synth.workload(name, 1)
     rng = np.random.default_rng(7)

@@ -98,6 +98,29 @@ def test_codes_in_range_and_uniform():
     assert np.array_equal(sub, codes[100:107])
 
 
+def test_recipe_stacks():
+    """The fixed recipe (§3.4): layer-0 MLP all 4-bit, every other projection
+    all 2-bit, the head tiered per row 8/4/2/1 bits over the top 0.5% / next
+    1.5% / next 10% / last 88% of rows (mean 1.18 bits)."""
+    for name, vocab in (("stack9b-recipe", 128256), ("stack131m-recipe", 32000)):
+        work = synth.workload(name)
+        plain = synth.workload(name[:-7])
+        assert [(m.n, m.k) for m in work.mats] == [(m.n, m.k) for m in plain.mats]
+        for spec in work.mats[:-1]:
+            w = gen.matrix_inputs(spec, 1)["widths"]
+            mlp0 = spec.name.split(".")[0] == "l0" and spec.name.split(".")[1] in ("gate", "up", "down")
+            assert (w == (4 if mlp0 else 2)).all(), spec.name
+        head = work.mats[-1]
+        w = gen.matrix_inputs(head, 1)["widths"]
+        assert head.n == vocab and (w == w[:, :1]).all()          # one width per row
+        rows = w[:, 0]
+        b8, b4, b2 = round(0.005 * vocab), round(0.02 * vocab), round(0.12 * vocab)
+        assert (rows[:b8] == 8).all() and (rows[b8:b4] == 4).all() and (rows[b4:b2] == 2).all()
+        assert (rows[b2:] == 1).all()
+        assert abs(rows.astype(float).mean() - 1.18) < 0.005
+    assert gen.tiered_widths(3, 2, ((0.5, 8), (1.0, 1))).tolist() == [[8, 8], [8, 8], [1, 1]]
+
+
 def test_generators_deterministic():
     spec = synth.workload("stack131m").mats[3]
     a = gen.matrix_inputs(spec, 2)
