@@ -17,6 +17,9 @@ What it defines (paper: "Variable Bit-width Quantization", arXiv 2607.02893):
   boundaries"), i.e. 8*b bytes, plus its scale.
 * The inference product (§6): y = W_hat x with the weights never widened in
   memory; here simply the plain dense definition in fp64.
+* SwiGLU on a gate-up product (the models' MLP, §4; §6 relies on
+  silu(0) * u = 0): h = silu(gate) * up with silu(z) = z / (1 + exp(-z)),
+  gate and up rows alternating (row 2i gate i, row 2i + 1 up i), fp64.
 
 Readings of points the paper leaves open (each also listed in the design notes):
 
@@ -118,6 +121,46 @@ def gemv(codes: np.ndarray, widths: np.ndarray, scales_fp16: np.ndarray, x: np.n
 def within_bound(y, y_ref, a_ref, rel: float = 2e-3, floor: float = 1e-5) -> np.ndarray:
     """Acceptance test of a computed y: |y - y_ref| <= rel * A + floor, elementwise."""
     return np.abs(np.asarray(y, np.float64) - y_ref) <= rel * a_ref + floor
+
+
+# ---------------------------------------------------------------------------
+# SwiGLU on a gate-up product (§4 models; §6: zero-padded intermediates are
+# inert because silu(0) * u = 0)
+# ---------------------------------------------------------------------------
+
+SILU_SLOPE_MAX = 1.1        # max |d silu / dz| (about 1.0998, at z near 2.4)
+
+
+def silu(z):
+    """silu(z) = z * sigmoid(z) = z / (1 + exp(-z)), fp64."""
+    z = np.asarray(z, dtype=np.float64)
+    with np.errstate(over="ignore"):
+        return z / (1.0 + np.exp(-z))
+
+
+def swiglu(y):
+    """h = silu(gate) * up for a gate-up product whose rows alternate: row 2i
+    is gate i, row 2i + 1 is up i. y: (B, N) with N even -> h: (B, N / 2)."""
+    y = np.atleast_2d(np.asarray(y, dtype=np.float64))
+    if y.shape[1] % 2:
+        raise ValueError("a gate-up product has an even number of rows")
+    return silu(y[:, 0::2]) * y[:, 1::2]
+
+
+def swiglu_within_bound(h, y_ref, a_ref, rel: float = 2e-3, floor: float = 1e-5) -> np.ndarray:
+    """True where h (rounded to BF16 by the kernel) is within the error that
+    follows from a gate-up product within within_bound: with eg, eu the
+    product bounds of g and u, |silu(g') u' - silu(g) u| <= 1.1 eg (|u| + eu)
+    + |silu(g)| eu, plus the BF16 rounding of the result (2^-8 relative, here
+    2^-7 for the fp32 evaluation as well)."""
+    y_ref = np.atleast_2d(y_ref)
+    a_ref = np.atleast_2d(a_ref)
+    g, u = y_ref[:, 0::2], y_ref[:, 1::2]
+    eg, eu = rel * a_ref[:, 0::2] + floor, rel * a_ref[:, 1::2] + floor
+    h_ref = swiglu(y_ref)
+    e = SILU_SLOPE_MAX * eg * (np.abs(u) + eu) + np.abs(silu(g)) * eu
+    tol = e * (1.0 + 2.0 ** -7) + 2.0 ** -7 * np.abs(h_ref)
+    return np.abs(np.atleast_2d(h) - h_ref) <= tol
 
 
 # ---------------------------------------------------------------------------

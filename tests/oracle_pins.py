@@ -218,6 +218,30 @@ def pin_enumerated_codes(O):
                 _check(list(got) == expect, f"b={b} pos {pos}")
 
 
+def pin_swiglu(O):
+    """SwiGLU (§4 models; §6 silu(0) * u = 0) by closed forms and identities:
+    silu(0) = 0, silu(1) = e / (1 + e), silu(z) - silu(-z) = z (the sigmoid's
+    symmetry), silu(z) -> z for large z and -> 0 for very negative z; the
+    pairing puts gate on even rows and up on odd rows; the slope bound the
+    tolerance uses holds on a dense grid."""
+    import math
+    _check(float(O.silu(0.0)) == 0.0, "silu(0)")
+    _check(abs(float(O.silu(1.0)) - math.e / (1.0 + math.e)) <= 1e-16, "silu(1)")
+    z = np.linspace(-30, 30, 6001)
+    _check(np.allclose(O.silu(z) - O.silu(-z), z, rtol=0, atol=1e-13), "silu odd part")
+    _check(float(O.silu(60.0)) == 60.0 and abs(float(O.silu(-60.0))) < 1e-20, "silu tails")
+    _check(np.isfinite(O.silu(np.array([-1000.0, 1000.0]))).all(), "silu overflow")
+    h = O.swiglu(np.array([[2.0, 3.0, -1.0, 5.0, 0.0, 7.0]]))
+    exp = [2.0 / (1.0 + math.exp(-2.0)) * 3.0, -1.0 / (1.0 + math.exp(1.0)) * 5.0, 0.0]
+    _check(np.allclose(h[0], exp, rtol=1e-15, atol=0), f"swiglu pairing {h}")
+    d = np.diff(O.silu(np.linspace(-20, 20, 400001))) / 1e-4
+    _check(np.abs(d).max() <= O.SILU_SLOPE_MAX and np.abs(d).max() > 1.09, "silu slope bound")
+    y = np.array([[1.5, -2.0, 0.25, 4.0]])
+    a = np.abs(y) + 1.0
+    _check(O.swiglu_within_bound(O.swiglu(y), y, a).all(), "bound admits the exact value")
+    _check(not O.swiglu_within_bound(O.swiglu(y) + 0.1, y, a).any(), "bound rejects a gross error")
+
+
 def pin_payload_accounting(O, seed=6):
     rng = np.random.default_rng(seed)
     n, k = 7, 320
@@ -232,4 +256,4 @@ def pin_payload_accounting(O, seed=6):
 
 ALL_PINS = [pin_eq1_golden, pin_level_grid, pin_grid_roundtrip, pin_quantizer_invariants,
             pin_one_bit_mean_order, pin_group_size_one, pin_integer_gemv, pin_exact_rational, pin_enumerated_codes,
-            pin_payload_accounting]
+            pin_swiglu, pin_payload_accounting]

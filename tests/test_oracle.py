@@ -55,6 +55,8 @@ MUTATIONS = {
     "sign_zero_negative": ("codes = (w >= 0).astype(np.uint8)", "codes = (w > 0).astype(np.uint8)"),
     "pack_msb_first": ("acc |= int(codes[r, g * GROUP + i]) << (i * b)",
                        "acc |= int(codes[r, g * GROUP + i]) << ((GROUP - 1 - i) * b)"),
+    "swiglu_swapped": ("return silu(y[:, 0::2]) * y[:, 1::2]", "return silu(y[:, 1::2]) * y[:, 0::2]"),
+    "silu_sign": ("return z / (1.0 + np.exp(-z))", "return z / (1.0 + np.exp(z))"),
     "scale_bytes_one": ("return 2 * int(np.asarray(widths).size)",
                         "return int(np.asarray(widths).size)"),
 }
