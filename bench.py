@@ -12,7 +12,12 @@ resident BF16 activation vector.
 same run: `grouped_by_input` (the headline's products in decode order, those
 that read the same input, Q/K/V and gate/up, issued as one vbq_gemv_group),
 `fused` (the <stack>-fused workload: QKV and gate-up as single matrices, 4
-GEMVs per layer), `grouped` (all of the headline's layouts as one
+GEMVs per layer), `fused_swiglu` (the same with the gate-up product's SwiGLU
+epilogue in its kernel, vbq_gemv_swiglu, whose BF16 output is the down
+projection's input: the MLP as one dependent chain), `fused_swiglu_in` (the
+same chain with the SwiGLU applied by the down projection as it stages its
+activations from the gate-up product's fp32 output, vbq_gemv_swiglu_in),
+`grouped` (all of the headline's layouts as one
 vbq_gemv_group per step: independent products whose launches overlap, the
 streaming upper bound) and `cublas_bf16` (dense BF16 weights of the same
 shapes through torch.mv, i.e. cuBLAS, as a reference point).
@@ -354,6 +359,43 @@ def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev
                         steps, warm)
         out["fused"] = entry(ms, sum(fnb), fcp, len(flays),
                              "workload " + name + "-fused: QKV and gate-up as single matrices, layer-serial")
+        # the same chain with the MLP's SwiGLU fused into the products, so the
+        # down projection consumes the gate-up product: (a) as the gate-up
+        # kernel's epilogue (vbq_gemv_swiglu writes BF16 h, the down
+        # projection reads it); (b) in the down projection's activation
+        # staging (vbq_gemv_swiglu_in reads the gate-up product's fp32 output)
+        calls, prev = [], None
+        for i, nm in enumerate([m.name for m in fwork.mats] * fcp):
+            proj = nm.rpartition(".")[2]
+            if proj == "gate_up":
+                prev = (i, torch.empty(flays[i].N // 2, dtype=torch.int16, device=dev))
+                calls.append((i, "gate_up", prev))
+            elif proj == "down" and prev is not None:
+                calls.append((i, "down", prev))
+                prev = None
+            else:
+                calls.append((i, "gemv", None))
+
+        def swiglu_chain(epilogue):
+            for i, kind, link in calls:
+                if kind == "gate_up" and epilogue:
+                    vbq.vbq_gemv_swiglu(flays[i], fxs[i][0], fys[i][0], link[1], stream=stream)
+                elif kind == "down" and epilogue:
+                    vbq.vbq_gemv(flays[i], link[1], fys[i][0], stream=stream)
+                elif kind == "down":
+                    vbq.vbq_gemv_swiglu_in(flays[i], fys[link[0]][0], fys[i][0], stream=stream)
+                else:
+                    vbq.vbq_gemv(flays[i], fxs[i][0], fys[i][0], stream=stream)
+        ms = time_graph(torch, stream, lambda: swiglu_chain(True), steps, warm)
+        out["fused_swiglu"] = entry(ms, sum(fnb), fcp, len(flays),
+                                    "workload " + name + "-fused with vbq_gemv_swiglu for gate-up (SwiGLU "
+                                    "epilogue in the product kernel, BF16 h) feeding the down projection, "
+                                    "layer-serial")
+        ms = time_graph(torch, stream, lambda: swiglu_chain(False), steps, warm)
+        out["fused_swiglu_in"] = entry(ms, sum(fnb), fcp, len(flays),
+                                       "workload " + name + "-fused, the down projection as vbq_gemv_swiglu_in on "
+                                       "the gate-up product's fp32 output (SwiGLU while staging activations, h "
+                                       "never stored), layer-serial")
         del flays, fxs, fys
         torch.cuda.empty_cache()
         rwork = synth.workload(name + "-recipe", 1)

@@ -179,6 +179,49 @@ vbq_status_t vbq_gemm_small(const vbq_layout* layout, const uint16_t* X, float* 
                             int B, void* stream);
 
 /*
+ * vbq_gemv_swiglu — the MLP's gate-up product with its SwiGLU epilogue fused
+ * in (§4: the models' MLPs are SwiGLU; §6: the fused kernels stream the
+ * packed gate and up projections, and zero-padded intermediates are inert
+ * because silu(0) * u = 0).
+ *   layout  a gate-up matrix whose rows alternate: row 2i is the gate
+ *           projection of feature i, row 2i + 1 its up projection (N even,
+ *           VBQ_ERR_SHAPE otherwise). Any layout from vbq_pack with even N.
+ *   x       device, K BF16 bit patterns.
+ *   y       device, N floats; overwritten with W x (rows interleaved as in W),
+ *           exactly as vbq_gemv writes it. It is also the kernel's
+ *           accumulator when a row spans several slabs.
+ *   h       device, N/2 BF16 bit patterns; overwritten with
+ *           h_i = silu(y_2i) * y_2i+1, silu(z) = z / (1 + e^-z), evaluated in
+ *           fp32 on the kernel's y and rounded to nearest even. This is the
+ *           down projection's input.
+ * Accuracy: y as vbq_gemv; h within the error that the bound on y implies
+ * (|d silu/dz| <= 1.1) plus its BF16 rounding. One launch: when a row spans
+ * several slabs, each row block's outputs are written by the block that adds
+ * its last slab. Same ordering rules as vbq_gemv (calls sharing a layout must
+ * not overlap on the GPU; the kernel is launched with programmatic dependent
+ * launch).
+ */
+vbq_status_t vbq_gemv_swiglu(const vbq_layout* layout, const uint16_t* x, float* y, uint16_t* h,
+                             void* stream);
+
+/*
+ * vbq_gemv_swiglu_in — the MLP's down projection applied to the SwiGLU of a
+ * gate-up product, y = W h with h_k = silu(gu[2k]) * gu[2k+1] (§4 SwiGLU
+ * MLPs; §6 fused packed products, padded features inert since
+ * silu(0) * u = 0). h is computed in fp32 as the kernel stages its
+ * activations and never reaches memory.
+ *   layout  the down projection, N x K.
+ *   gu      device, 2K floats: gate and up of feature k at 2k and 2k + 1, i.e.
+ *           the y of a vbq_gemv over a gate-up matrix whose rows alternate.
+ *   y       device, N floats; overwritten.
+ * Per output, |y - y_exact| stays within 2e-3 * sum_k |w_nk h_k| + 1e-5, with
+ * h and y_exact exact functions of gu (h's fp32 evaluation adds a few ulps).
+ * Same ordering rules as vbq_gemv; gu is read only after the previous kernel
+ * on the stream has finished, so it may be that kernel's output.
+ */
+vbq_status_t vbq_gemv_swiglu_in(const vbq_layout* layout, const float* gu, float* y, void* stream);
+
+/*
  * vbq_gemv_group — count independent batch-1 products y_i = W_i x_i (§6
  * product, several matrices). (The paper has no counterpart; this is an
  * execution mode for products that do not feed one another, such as the

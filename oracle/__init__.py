@@ -6,6 +6,6 @@ import this package. The CUDA library and its Python binding never do.
 
 from .vbq_oracle import (  # noqa: F401
     GROUP, WIDTHS, level, check_inputs, dequant, gemv, within_bound,
-    silu, swiglu, swiglu_within_bound, SILU_SLOPE_MAX,
+    silu, swiglu, swiglu_error_bound, swiglu_within_bound, SILU_SLOPE_MAX,
     quantize_group, quantize, payload_bytes, scale_bytes, pack_lsb, unpack_lsb,
 )

@@ -147,18 +147,25 @@ def swiglu(y):
     return silu(y[:, 0::2]) * y[:, 1::2]
 
 
-def swiglu_within_bound(h, y_ref, a_ref, rel: float = 2e-3, floor: float = 1e-5) -> np.ndarray:
-    """True where h (rounded to BF16 by the kernel) is within the error that
-    follows from a gate-up product within within_bound: with eg, eu the
-    product bounds of g and u, |silu(g') u' - silu(g) u| <= 1.1 eg (|u| + eu)
-    + |silu(g)| eu, plus the BF16 rounding of the result (2^-8 relative, here
-    2^-7 for the fp32 evaluation as well)."""
+def swiglu_error_bound(y_ref, a_ref, rel: float = 2e-3, floor: float = 1e-5) -> np.ndarray:
+    """Largest |silu(g') u' - silu(g) u| over gate-up values g', u' that are
+    within the product bound of within_bound from the exact g, u: with eg, eu
+    those bounds, 1.1 eg (|u| + eu) + |silu(g)| eu (mean value theorem on silu,
+    whose slope is at most 1.1 in magnitude). Shape (B, N / 2)."""
     y_ref = np.atleast_2d(y_ref)
     a_ref = np.atleast_2d(a_ref)
     g, u = y_ref[:, 0::2], y_ref[:, 1::2]
     eg, eu = rel * a_ref[:, 0::2] + floor, rel * a_ref[:, 1::2] + floor
+    return SILU_SLOPE_MAX * eg * (np.abs(u) + eu) + np.abs(silu(g)) * eu
+
+
+def swiglu_within_bound(h, y_ref, a_ref, rel: float = 2e-3, floor: float = 1e-5) -> np.ndarray:
+    """True where h (rounded to BF16 by the kernel) is within the error that
+    follows from a gate-up product within within_bound (swiglu_error_bound),
+    plus the BF16 rounding of the result (2^-8 relative, here 2^-7 for the
+    fp32 evaluation as well)."""
     h_ref = swiglu(y_ref)
-    e = SILU_SLOPE_MAX * eg * (np.abs(u) + eu) + np.abs(silu(g)) * eu
+    e = swiglu_error_bound(y_ref, a_ref, rel, floor)
     tol = e * (1.0 + 2.0 ** -7) + 2.0 ** -7 * np.abs(h_ref)
     return np.abs(np.atleast_2d(h) - h_ref) <= tol
 

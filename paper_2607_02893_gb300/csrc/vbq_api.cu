@@ -190,7 +190,8 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     const size_t blob_bytes = (size_t)off16 * 16 + 256;
     const size_t off_at = round_up(blob_bytes, 256);
     const size_t ctl_at = round_up(off_at + blob_off.size() * 4, 256);
-    const size_t alloc_bytes = ctl_at + (2 + (size_t)nrb) * sizeof(uint32_t);
+    // control words: call counter, zeroed-row flags, SwiGLU slab counts
+    const size_t alloc_bytes = ctl_at + (2 + 2 * (size_t)nrb) * sizeof(uint32_t);
     void* d_headers = nullptr;
     VBQ_CUDA(tmp.alloc(&d_headers, headers.size() * sizeof(vbq::UnitHeader)));
     VBQ_CUDA(cudaMemcpyAsync(d_headers, headers.data(), headers.size() * sizeof(vbq::UnitHeader),
@@ -345,6 +346,28 @@ vbq_status_t vbq_gemv_group(const vbq_layout* const* layouts, const uint16_t* co
     if (std::adjacent_find(seen_y.begin(), seen_y.end()) != seen_y.end())
         return fail(VBQ_ERR_ARG, "an output appears twice in one group");
     VBQ_CUDA(vbq::launch_gemv_group(views.data(), xs, ys, count, static_cast<cudaStream_t>(stream)));
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_gemv_swiglu(const vbq_layout* L, const uint16_t* x, float* y, uint16_t* h, void* stream) {
+    g_err[0] = 0;
+    vbq_status_t st = check_layout(L);
+    if (st) return st;
+    if (!x || !y || !h) return fail(VBQ_ERR_ARG, "x, y and h must be non-NULL");
+    if (!aligned16(x) || !aligned16(y) || !aligned16(h)) return fail(VBQ_ERR_ALIGN, "x, y and h must be 16-byte aligned");
+    if (L->view.N % 2 != 0)
+        return fail(VBQ_ERR_SHAPE, "a gate-up matrix has an even number of rows (N=%lld)", (long long)L->view.N);
+    VBQ_CUDA(vbq::launch_gemv_swiglu(L->view, x, y, h, static_cast<cudaStream_t>(stream)));
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_gemv_swiglu_in(const vbq_layout* L, const float* gu, float* y, void* stream) {
+    g_err[0] = 0;
+    vbq_status_t st = check_layout(L);
+    if (st) return st;
+    if (!gu || !y) return fail(VBQ_ERR_ARG, "gu and y must be non-NULL");
+    if (!aligned16(gu) || !aligned16(y)) return fail(VBQ_ERR_ALIGN, "gu and y must be 16-byte aligned");
+    VBQ_CUDA(vbq::launch_gemv_swiglu_in(L->view, gu, y, static_cast<cudaStream_t>(stream)));
     return VBQ_OK;
 }
 

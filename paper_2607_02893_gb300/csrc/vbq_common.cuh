@@ -21,7 +21,9 @@
 //     partials into y with atomics, and y needs no zeroing by the caller: the
 //     block that owns slab 0 of a row block zeroes those rows first and then
 //     sets that row block's flag to the current call's epoch; blocks adding
-//     other slabs wait for the flag. The epoch lives on the device (the last
+//     other slabs wait for the flag. With the SwiGLU epilogue it also resets
+//     the row block's slab count, and the block whose addition brings the
+//     count to S applies the epilogue to the finished rows. The epoch lives on the device (the last
 //     block of a call advances it), so graph replays stay correct. Calls that
 //     share a layout must not overlap on the GPU.
 //   * Within a unit the groups ("items") of one width are ordered by
@@ -62,7 +64,8 @@ static_assert(sizeof(UnitHeader) == 48, "header is 48 bytes");
 struct LayoutView {
     const uint8_t* blobs;       // blob area
     const uint32_t* blob_off;   // units + 1 offsets, in 16-byte units
-    uint32_t* ctl;              // [0..1] 64-bit call counter (see call_epoch), [2 + rb] y-zeroed flags
+    uint32_t* ctl;              // [0..1] 64-bit call counter (see call_epoch), [2 + rb] y-zeroed flags,
+                                // [2 + nrb + rb] slabs added (SwiGLU epilogue, see swiglu_row_block)
     int64_t N, K;
     int G, C, S, nrb, units;
     int max_blob16;             // largest blob, in 16-byte units

@@ -116,6 +116,19 @@ __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
     return v;
 }
 
+// Acquire-release add at GPU scope (returns the old value), and a relaxed
+// GPU-scope load of two floats (read at L2, never a stale L1 line).
+__device__ __forceinline__ uint32_t atom_add_acq_rel_gpu(uint32_t* p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+__device__ __forceinline__ float2 ld_relaxed_gpu_f32x2(const float* p) {
+    float2 v;
+    asm volatile("ld.relaxed.gpu.global.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "l"(p) : "memory");
+    return v;
+}
+
 // Split-K call counter, control words 0-1 (one 64-bit word): every call adds
 // exactly 2^CALL_SHIFT in all, split over its blocks, so (counter >>
 // CALL_SHIFT) counts the calls before this one; a block that reads it while

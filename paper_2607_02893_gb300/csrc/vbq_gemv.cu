@@ -41,11 +41,21 @@
 // 2..4 as one or two launches): the second vector's tables sit a fixed
 // distance after the first's, so each lookup address, masked code and level
 // serves both. Batches of 5..16 run on the tensor cores in vbq_gemm.cu.
+//
+// Two more instantiations fuse a SwiGLU MLP's nonlinearity into the products
+// (the paper's models use SwiGLU MLPs, §4; zero-padded intermediates are inert,
+// §6): MODE_SWIGLU_EPI, on a gate-up matrix whose rows alternate, also writes
+// h = silu(gate) * up in BF16 (the copier computes it from a row pair's sums
+// when a row has one slab, otherwise the block whose addition completes a row
+// block's slab count reads the finished rows back); MODE_SWIGLU_IN, on the
+// down projection, builds its activation tables from h_k = silu(gu[2k]) *
+// gu[2k + 1] of the gate-up product's fp32 output, so h never reaches memory.
 #include <cstddef>
 #include <mutex>
 
 #include "vbq_kernels.h"
 #include "vbq_device.cuh"
+#include <cuda_bf16.h>
 
 namespace vbq {
 namespace {
@@ -59,6 +69,13 @@ constexpr int LUT_COL_BYTES = 1280;      // 16 tables x 64 bytes (+64 for odd co
 constexpr int STAGE_BYTES = MAX_BLOB_BYTES;   // holds the largest unit blob (the packer guarantees it)
 static_assert(STAGE_BYTES % 256 == 0, "stages keep the tables 256-byte aligned");
 static_assert(LUT_COL_BYTES % 256 == 0 && 64 + 16 * 64 <= LUT_COL_BYTES, "column tables: 256-byte aligned, room for the odd shift");
+
+// What a launch does around the product (a template argument, so the plain
+// product's code carries none of the others'): MODE_PLAIN y = W x;
+// MODE_SWIGLU_EPI also writes h = silu(gate) * up in BF16 from a gate-up
+// product whose rows alternate (NX = 1); MODE_SWIGLU_IN takes as activations
+// h_k = silu(gu[2k]) * gu[2k + 1] of a gate-up output gu (NX = 1).
+enum Mode : int { MODE_PLAIN = 0, MODE_SWIGLU_EPI = 1, MODE_SWIGLU_IN = 2 };
 
 // One kernel serves NX = 1 or 2 activation vectors (batch rows) per launch.
 // With two, every table lookup address serves both: the second vector's
@@ -302,6 +319,27 @@ __device__ __forceinline__ void consumer_sync() {
     asm volatile("bar.sync 1, %0;" :: "n"(NCT) : "memory");
 }
 
+// silu(g) * u with silu(z) = z / (1 + e^-z), in fp32 with explicitly rounded
+// operations (no contraction), so every call site gives the same bits.
+// silu(0) * u = 0: zero-padded features stay inert.
+__device__ __forceinline__ float swiglu_f32(float g, float u) {
+    return __fmul_rn(__fdiv_rn(g, __fadd_rn(1.f, expf(-g))), u);
+}
+
+// The 4-bit zero-level sum of half a group's activations (32 of them), as
+// (even, odd) code slots times 2^-100, in the order dot4_half accumulates.
+__device__ __forceinline__ float2 zero_level_sum4(const float (&xh)[32]) {
+    float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
+#pragma unroll
+    for (int t4 = 0; t4 < 4; ++t4) {
+        float2& cc = (t4 & 1) ? cb : ca;
+#pragma unroll
+        for (int e = 0; e < 8; e += 2)
+            cc = __ffma2_rn(f2(xh[8 * t4 + e], xh[8 * t4 + e + 1]), f2(0x1p-100f, 0x1p-100f), cc);
+    }
+    return __fadd2_rn(ca, cb);
+}
+
 // Activations of slab s (per vector, for NX vectors stored K apart): x as fp32,
 // the pre-scaled x of the 4-bit slots, the nibble lookup tables, and the
 // per-column sums in lookup order. Consumer threads only (ct = 0 .. NCT-1):
@@ -312,20 +350,34 @@ __device__ __forceinline__ void consumer_sync() {
 // barriers. The column sum of the all-ones entries (xlut) is added over the
 // column's half-warp in the pairs tree16x2 uses.
 static_assert(NCT >= 16 * MAX_C + 2 * MAX_C, "threads for the tables and the zero-level sums");
-template <int NX>
-__device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t* __restrict__ x, int s, int ct) {
+template <int NX, int MODE>
+__device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t* __restrict__ x,
+                             const float* __restrict__ gu, int s, int ct) {
     const int cols = min(L.C, L.G - s * L.C);
     consumer_sync();                // nobody still reads the old tables
     if (ct < cols * 16) {
         const int c = ct >> 4, jn = ct & 15, jj = 4 * jn;
 #pragma unroll
         for (int v = 0; v < NX; ++v) {
-            const uint16_t* xg = x + (int64_t)v * L.K + (int64_t)s * L.C * GROUP;
             float* xs = T.xs + v * XS_FLOATS;
             float* x4s = T.x4s + v * X4S_FLOATS;
-            const uint2 four = __ldg(reinterpret_cast<const uint2*>(xg + c * GROUP + jj));
-            const float x0 = __uint_as_float(four.x << 16), x1 = __uint_as_float(four.x & 0xFFFF0000u);
-            const float x2 = __uint_as_float(four.y << 16), x3 = __uint_as_float(four.y & 0xFFFF0000u);
+            float x0, x1, x2, x3;
+            if constexpr (MODE == MODE_SWIGLU_IN) {
+                // SwiGLU input: activation k is silu(gu[2k]) * gu[2k + 1]
+                const float4* src = reinterpret_cast<const float4*>(gu + 2 * ((int64_t)s * L.C * GROUP + c * GROUP + jj));
+                const float4 a = __ldg(src), b = __ldg(src + 1);
+                x0 = swiglu_f32(a.x, a.y);
+                x1 = swiglu_f32(a.z, a.w);
+                x2 = swiglu_f32(b.x, b.y);
+                x3 = swiglu_f32(b.z, b.w);
+            } else {
+                const uint16_t* xg = x + (int64_t)v * L.K + (int64_t)s * L.C * GROUP;
+                const uint2 four = __ldg(reinterpret_cast<const uint2*>(xg + c * GROUP + jj));
+                x0 = __uint_as_float(four.x << 16);
+                x1 = __uint_as_float(four.x & 0xFFFF0000u);
+                x2 = __uint_as_float(four.y << 16);
+                x3 = __uint_as_float(four.y & 0xFFFF0000u);
+            }
             *reinterpret_cast<float4*>(&xs[(c * 4 + (jj >> 4)) * XQ + (jj & 15)]) = make_float4(x0, x1, x2, x3);
             // 4-bit slot shifts: nibble slots 0..5 of a word keep their place, 6 and 7 come down by 24
             float p4[4];
@@ -352,7 +404,7 @@ __device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t
             sv += __shfl_xor_sync(half, sv, 8);
             if (jn == 0) T.xlut[v][c] = sv;
         }
-    } else if (ct >= 16 * MAX_C && ct < 16 * MAX_C + cols * 2) {
+    } else if (MODE != MODE_SWIGLU_IN && ct >= 16 * MAX_C && ct < 16 * MAX_C + cols * 2) {
         // X for the 4-bit zero level of half hh of column c, summed as
         // dot4_half accumulates (threads the lookup tables leave idle)
         const int z = ct - 16 * MAX_C, c = z >> 1, hh = z & 1;     // c < cols, hh < 2
@@ -371,15 +423,30 @@ __device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t
                     xh[8 * q + 2 * i + 1] = __uint_as_float(ws[i] & 0xFFFF0000u);
                 }
             }
-            float2 ca = f2(0.f, 0.f), cb = f2(0.f, 0.f);
+            T.x4z[v][c][hh] = zero_level_sum4(xh);
+        }
+    }
+    if constexpr (MODE == MODE_SWIGLU_IN) {
+        // SwiGLU input: the activations exist only once the table threads have
+        // computed them, so the zero-level sums read them back from xs after a
+        // barrier (the same values the lookups and products use)
+        consumer_sync();
+        if (ct >= 16 * MAX_C && ct < 16 * MAX_C + cols * 2) {
+            const int z = ct - 16 * MAX_C, c = z >> 1, hh = z & 1;
+            float xh[32];
 #pragma unroll
-            for (int t4 = 0; t4 < 4; ++t4) {
-                float2& cc = (t4 & 1) ? cb : ca;
+            for (int q = 0; q < 2; ++q) {
+                const uint32_t a = smem_u32(T.xs) + ((c * 4 + 2 * hh + q) * XQ) * 4;
 #pragma unroll
-                for (int e = 0; e < 8; e += 2)
-                    cc = __ffma2_rn(f2(xh[8 * t4 + e], xh[8 * t4 + e + 1]), f2(0x1p-100f, 0x1p-100f), cc);
+                for (int i = 0; i < 4; ++i) {
+                    const float4 f = lds_f32x4(a + 16 * i);
+                    xh[16 * q + 4 * i] = f.x;
+                    xh[16 * q + 4 * i + 1] = f.y;
+                    xh[16 * q + 4 * i + 2] = f.z;
+                    xh[16 * q + 4 * i + 3] = f.w;
+                }
             }
-            T.x4z[v][c][hh] = __fadd2_rn(ca, cb);
+            T.x4z[0][c][hh] = zero_level_sum4(xh);
         }
     }
     consumer_sync();
@@ -575,10 +642,38 @@ __device__ __forceinline__ void consume_unit(const TablesT<NX>& T, uint32_t sblo
     if (n[0]) run_width<0, NX>(T, view(0), slots, (t0 - nt3 - nt2 - nt1) & m, tstep, lane);
 }
 
+// SwiGLU epilogue of a gate-up product whose rows alternate (row 2i the gate
+// of feature i, row 2i + 1 its up projection): h_i = silu(g_i) * u_i, rounded
+// to BF16 (to nearest even), the input format of the down projection.
+__device__ __forceinline__ uint16_t swiglu_bf16(float g, float u) {
+    return __bfloat16_as_ushort(__float2bfloat16_rn(swiglu_f32(g, u)));
+}
+
+// Several slabs per row: after adding a unit's rows into y, the copier adds 1
+// to its row block's slab count (reset by the zeroing owner of slab 0 before
+// it publishes its flag) with an acquire-release RMW by lane 0, ordered after
+// the warp's additions by the preceding __syncwarp. The RMW's reply is read one
+// unit later, so its round trip overlaps the next unit. The adder whose RMW
+// brings the count to S writes the row block's 64 outputs: its lane 0 has
+// acquired every slab's additions, and the warp barrier (which orders memory
+// among the warp's lanes) passes them on to the lanes' GPU-scope loads.
+__device__ __forceinline__ void swiglu_rows(const LayoutView& L, const float* y, uint16_t* h, int rb, int lane) {
+    const int rows = min(RB, (int)(L.N - (int64_t)rb * RB));
+    const float* yr = y + (int64_t)rb * RB;
+    uint16_t* hr = h + (int64_t)rb * (RB / 2);
+    for (int p = lane; 2 * p < rows; p += 32) {
+        const float2 gu = ld_relaxed_gpu_f32x2(yr + 2 * p);
+        hr[p] = swiglu_bf16(gu.x, gu.y);
+    }
+}
+
 // NX activation vectors x (NX x K, row-major) and outputs y (NX x N).
-template <int NX>
+template <int NX, int MODE>
 __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
-                                                              float* __restrict__ y, int dep) {
+                                                              float* __restrict__ y, int dep,
+                                                              uint16_t* __restrict__ h,
+                                                              const float* __restrict__ gu) {
+    static_assert(MODE == MODE_PLAIN || NX == 1, "the SwiGLU forms take one activation vector");
     constexpr int NSTAGE = Geo<NX>::nstage;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     // stages and tables on a 256-byte boundary: lookups merge a byte into table addresses
@@ -624,10 +719,15 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     // first slab's activations are prefetched into L2 meanwhile.
     {
         const int64_t k0 = (int64_t)s0 * L.C * GROUP;
-        const int lines = (min(L.C, L.G - s0 * L.C) * GROUP * 2 + 127) / 128;
-        if (tid >= 32 && tid - 32 < NX * lines) {
-            const int v = (tid - 32) / lines, ln = (tid - 32) - v * lines;
-            prefetch_l2(x + (int64_t)v * L.K + k0 + (int64_t)ln * 64);
+        if constexpr (MODE == MODE_SWIGLU_IN) {      // 8 bytes (a gate-up pair) per activation
+            const int lines = (min(L.C, L.G - s0 * L.C) * GROUP * 8 + 127) / 128;
+            if (tid >= 32 && tid - 32 < lines) prefetch_l2(gu + 2 * k0 + (int64_t)(tid - 32) * 32);
+        } else {
+            const int lines = (min(L.C, L.G - s0 * L.C) * GROUP * 2 + 127) / 128;
+            if (tid >= 32 && tid - 32 < NX * lines) {
+                const int v = (tid - 32) / lines, ln = (tid - 32) - v * lines;
+                prefetch_l2(x + (int64_t)v * L.K + k0 + (int64_t)ln * 64);
+            }
         }
     }
     // Ordering against the previous kernel on the stream (see Dep):
@@ -654,7 +754,10 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             __syncwarp();
             // release stores, one unit per lane in parallel: the warp's zeros
             // (ordered by __syncwarp) before each flag
-            for (int u = u_begin + lane; u < z_end; u += 32) st_release_gpu(L.ctl + 2 + u, epoch);
+            for (int u = u_begin + lane; u < z_end; u += 32) {
+                if (MODE == MODE_SWIGLU_EPI) L.ctl[2 + L.nrb + u] = 0u;     // SwiGLU slab count, before the flag's release
+                st_release_gpu(L.ctl + 2 + u, epoch);
+            }
         }
         bool dead = false;
         if (L.S > 1 && !split_k_flags_ready(L, epoch, u_begin, u_end, lane)) {
@@ -664,6 +767,8 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         }
         int st = 0, rbw = rb0, issued = n_units < NSTAGE ? n_units : NSTAGE;
         uint32_t par = 0;
+        int pend_rb = -1;               // SwiGLU: row block whose slab count's reply is pending
+        uint32_t pend_count = 0;        // (lane 0) that count before this block's addition
         for (int j = 0; j < n_units; ++j) {
             // nap between polls, except on the block's last unit, whose rows end the block
             if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, j + 1 < n_units ? 256 : 0)) {
@@ -694,15 +799,38 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                         if (L.S == 1) yr[r] = sum;
                         else red_global(yr + r, sum);
                     }
+                    if (MODE == MODE_SWIGLU_EPI && L.S == 1) {
+                        // the row is complete: gate (even row) and up (odd row) sit in
+                        // neighbouring lanes
+                        const float up = __shfl_xor_sync(0xffffffffu, sum, 1);
+                        if (!(lane & 1) && r < rows) h[((int64_t)rbw * RB + r) >> 1] = swiglu_bf16(sum, up);
+                    }
                 }
                 __syncwarp();
                 if (j + NSTAGE < n_units) {
                     if (lane == 0) issue_unit(L, u_begin + j + NSTAGE, stage0 + st * STAGE_BYTES, full0 + 8 * st);
                     ++issued;
                 }
+                if (MODE == MODE_SWIGLU_EPI && L.S > 1) {
+                    // SwiGLU: count this unit's slab, then act on the previous unit's count
+                    uint32_t count = 0;
+                    if (lane == 0) count = atom_add_acq_rel_gpu(L.ctl + 2 + L.nrb + rbw, 1u);
+                    if (pend_rb >= 0 && __shfl_sync(0xffffffffu, pend_count, 0) + 1u == (uint32_t)L.S) {
+                        __syncwarp();
+                        swiglu_rows(L, y, h, pend_rb, lane);
+                    }
+                    pend_rb = rbw;
+                    pend_count = count;
+                }
             }
             if (++st == NSTAGE) { st = 0; par ^= 1; }
             if (++rbw == L.nrb) rbw = 0;
+        }
+        if (MODE == MODE_SWIGLU_EPI && L.S > 1 && pend_rb >= 0) {
+            if (__shfl_sync(0xffffffffu, pend_count, 0) + 1u == (uint32_t)L.S) {
+                __syncwarp();
+                swiglu_rows(L, y, h, pend_rb, lane);
+            }
         }
         if (dead && lane == 0) {
             // let every copy this block started land before the block exits: the
@@ -725,11 +853,11 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         int cur = s0;
         int rbj = rb0 + team, sj = s0;                  // row block and slab of unit j
         while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
-        build_tables<NX>(T, L, x, s0, ct);
+        build_tables<NX, MODE>(T, L, x, gu, s0, ct);
         for (int j = team; j < n_units; j += teams) {
             // every consumer warp rebuilds the tables at every slab boundary of the
             // block's range, in order (the rebuild's named barrier waits for all)
-            while (cur < sj) build_tables<NX>(T, L, x, ++cur, ct);
+            while (cur < sj) build_tables<NX, MODE>(T, L, x, gu, ++cur, ct);
             const int st = j & (NSTAGE - 1);
             const uint32_t par = (uint32_t)(j / NSTAGE) & 1u;
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
@@ -744,17 +872,18 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             rbj += teams;
             while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
         }
-        while (cur < s_last) build_tables<NX>(T, L, x, ++cur, ct);   // boundaries past this team's last unit
+        while (cur < s_last) build_tables<NX, MODE>(T, L, x, gu, ++cur, ct);   // boundaries past this team's last unit
     }
 }
 
 int g_sms = 0;
 
-template <int NX>
-cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s, int dep) {
+template <int NX, int MODE = MODE_PLAIN>
+cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s, int dep,
+                         uint16_t* h = nullptr, const float* gu = nullptr) {
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemv1_kernel<NX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute(gemv1_kernel<NX, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)gemv1_smem<NX>());
         if (e != cudaSuccess) return e;
         int dev = 0;
@@ -773,7 +902,7 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, gemv1_kernel<NX>, L, x, y, dep);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, gemv1_kernel<NX, MODE>, L, x, y, dep, h, gu);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -887,6 +1016,14 @@ cudaError_t launch_gemv_group(const LayoutView* const* Ls, const uint16_t* const
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
+}
+
+cudaError_t launch_gemv_swiglu(const LayoutView& L, const uint16_t* x, float* y, uint16_t* h, cudaStream_t s) {
+    return launch_gemv1<1, MODE_SWIGLU_EPI>(L, x, y, s, DEP_BEFORE, h);
+}
+
+cudaError_t launch_gemv_swiglu_in(const LayoutView& L, const float* gu, float* y, cudaStream_t s) {
+    return launch_gemv1<1, MODE_SWIGLU_IN>(L, nullptr, y, s, DEP_BEFORE, nullptr, gu);
 }
 
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {

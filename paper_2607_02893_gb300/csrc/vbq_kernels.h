@@ -46,6 +46,17 @@ enum Dep : int { DEP_BEFORE = 0, DEP_GROUP_FIRST = 1, DEP_GROUP_NEXT = 2 };
 cudaError_t launch_gemv_group(const LayoutView* const* Ls, const uint16_t* const* xs, float* const* ys, int count,
                               cudaStream_t s);
 
+// Batch 1 on a gate-up matrix whose rows alternate (gate i, up i) with the
+// SwiGLU epilogue: y (N floats) as launch_gemv writes it, and h (N/2 BF16 bit
+// patterns) = silu(gate) * up. Uses the layout's slab counts (control words
+// 2 + nrb ..) when a row spans several slabs.
+cudaError_t launch_gemv_swiglu(const LayoutView& L, const uint16_t* x, float* y, uint16_t* h, cudaStream_t s);
+
+// Batch 1 whose activations are h_k = silu(gu[2k]) * gu[2k + 1], computed in
+// fp32 while the activation tables are built (gu: 2K floats, the y of a
+// gate-up product with alternating rows); h never reaches memory.
+cudaError_t launch_gemv_swiglu_in(const LayoutView& L, const float* gu, float* y, cudaStream_t s);
+
 // Batch 1 with the split-K control words in a fixed device array (no
 // allocation anywhere); usable for layouts with at most STATIC_CTL_WORDS - 2
 // row blocks.

@@ -36,6 +36,8 @@ SIGNATURES = {
     "vbq_gemv": (_I, [_P, _P, _P, _P]),
     "vbq_gemm_small": (_I, [_P, _P, _P, _I, _P]),
     "vbq_gemv_static": (_I, [_P, _P, _P, _P]),
+    "vbq_gemv_swiglu": (_I, [_P, _P, _P, _P, _P]),
+    "vbq_gemv_swiglu_in": (_I, [_P, _P, _P, _P]),
     "vbq_gemv_group": (_I, [ctypes.POINTER(_P), ctypes.POINTER(_P), ctypes.POINTER(_P), _I, _P]),
     "vbq_device_status": (_I, [_P]),
     "vbq_selftest_timeout": (_I, [_I, _P]),
@@ -173,6 +175,20 @@ def vbq_dequant(layout: Layout, codes_out=None, bitwidths_out=None, scales_out=N
 
 def vbq_gemv(layout: Layout, x, y, stream=None) -> None:
     _check(load().vbq_gemv(layout, _ptr(x), _ptr(y), _stream(stream, x, y)))
+
+
+def vbq_gemv_swiglu(layout: Layout, x, y, h, stream=None) -> None:
+    """Gate-up product with the SwiGLU epilogue: y = W x (N floats, rows
+    alternating gate / up) and h = silu(y[0::2]) * y[1::2] as N/2 BF16 bit
+    patterns (int16 or bfloat16 storage)."""
+    _check(load().vbq_gemv_swiglu(layout, _ptr(x), _ptr(y), _ptr(h), _stream(stream, x, y, h)))
+
+
+def vbq_gemv_swiglu_in(layout: Layout, gu, y, stream=None) -> None:
+    """Down projection of a SwiGLU MLP: y = W h with h_k = silu(gu[2k]) *
+    gu[2k + 1] computed in the kernel (gu: 2K float32, the y of a gate-up
+    product with alternating rows)."""
+    _check(load().vbq_gemv_swiglu_in(layout, _ptr(gu), _ptr(y), _stream(stream, gu, y)))
 
 
 def vbq_gemv_static(layout: Layout, x, y, stream=None) -> None:

@@ -71,6 +71,16 @@ def draw_x_bf16(batch: int, k: int, rng: np.random.Generator) -> np.ndarray:
     return f32_to_bf16_bits(rng.normal(0.0, 1.0, size=(batch, k)).astype(np.float32))
 
 
+def draw_gate_up(k: int, rng: np.random.Generator) -> np.ndarray:
+    """A gate-up product's output as the down projection reads it: 2k float32,
+    gate and up of feature i at 2i and 2i + 1, both N(0, 1.5) (about the
+    spread of the synthetic gate-up products), with one feature in eight
+    zero-padded (gate and up exactly 0)."""
+    gu = rng.normal(0.0, 1.5, size=(k, 2))
+    gu[rng.random(k) < 0.125] = 0.0
+    return gu.astype(np.float32).reshape(2 * k)
+
+
 def code_key(seed_path: Sequence[int]) -> int:
     return int(np.random.SeedSequence([0, *seed_path, 1]).generate_state(1, dtype=np.uint32)[0])
 

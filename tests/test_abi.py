@@ -83,6 +83,8 @@ def test_quantize_rejects_bad_arguments_on_host(lib):
 def test_calls_reject_null_layout(lib):
     assert lib.vbq_gemv(None, None, None, None) == -1
     assert lib.vbq_gemm_small(None, None, None, 4, None) == -1
+    assert lib.vbq_gemv_swiglu(None, None, None, None, None) == -1
+    assert lib.vbq_gemv_swiglu_in(None, None, None, None) == -1
     assert lib.vbq_dequant(None, None, None, None, None, None) == -1
     assert lib.vbq_packed_bytes(None, None, None, None) == -1
     assert lib.vbq_layout_shape(None, None, None) == -1
