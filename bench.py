@@ -17,7 +17,12 @@ epilogue in its kernel, vbq_gemv_swiglu, whose BF16 output is the down
 projection's input: the MLP as one dependent chain), `fused_swiglu_in` (the
 same chain with the SwiGLU applied by the down projection as it stages its
 activations from the gate-up product's fp32 output, vbq_gemv_swiglu_in),
-`grouped` (all of the headline's layouts as one
+`chain` (the headline's products as one vbq_chain_run: one
+persistent launch per step, every product still waiting for all earlier
+ones, weights streamed across product boundaries), `chain_fused` (the same for
+the fused workload), `chain_independent` (the headline's products as one
+chain without waits: independent products in one persistent launch, the
+kernel's streaming upper bound), `grouped` (all of the headline's layouts as one
 vbq_gemv_group per step: independent products whose launches overlap, the
 streaming upper bound) and `cublas_bf16` (dense BF16 weights of the same
 shapes through torch.mv, i.e. cuBLAS, as a reference point).
@@ -328,6 +333,21 @@ def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev
     out["grouped"] = entry(ms, step_bytes, copies, len(layouts),
                            "the headline layouts as one vbq_gemv_group per step (independent products, "
                            "overlapping launches): the streaming upper bound")
+    # the headline's chain in one persistent launch: every product still waits
+    # for all earlier ones before it touches x and y (layer-serial), but the
+    # weights stream across product boundaries
+    chain = vbq.Chain(layouts, x0, y0)
+    ms = time_graph(torch, stream, lambda: chain.run(stream=stream), steps, warm)
+    out["chain"] = entry(ms, step_bytes, copies, len(layouts),
+                         "the headline's products as one vbq_chain_run per step (one persistent launch; every "
+                         "product waits for all earlier ones, as layer-serial; weights stream across products)")
+    chain.free()
+    chain = vbq.Chain(layouts, x0, y0, [0] * len(layouts))
+    ms = time_graph(torch, stream, lambda: chain.run(stream=stream), steps, warm)
+    out["chain_independent"] = entry(ms, step_bytes, copies, len(layouts),
+                                     "the headline's products as one vbq_chain_run with no waits (independent "
+                                     "products in one persistent launch): the kernel's streaming upper bound")
+    chain.free()
     # the decode order with products that read the same input issued as one
     # group: per layer (Q, K, V) together, O, (gate, up) together, down
     names = [m.name for m in work.mats] * copies
@@ -359,6 +379,12 @@ def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev
                         steps, warm)
         out["fused"] = entry(ms, sum(fnb), fcp, len(flays),
                              "workload " + name + "-fused: QKV and gate-up as single matrices, layer-serial")
+        fchain = vbq.Chain(flays, [x[0] for x in fxs], [y[0] for y in fys])
+        ms = time_graph(torch, stream, lambda: fchain.run(stream=stream), steps, warm)
+        out["chain_fused"] = entry(ms, sum(fnb), fcp, len(flays),
+                                   "workload " + name + "-fused as one vbq_chain_run per step (every product "
+                                   "waits for all earlier ones)")
+        fchain.free()
         # the same chain with the MLP's SwiGLU fused into the products, so the
         # down projection consumes the gate-up product: (a) as the gate-up
         # kernel's epilogue (vbq_gemv_swiglu writes BF16 h, the down

@@ -243,6 +243,45 @@ vbq_status_t vbq_gemv_group(const vbq_layout* const* layouts, const uint16_t* co
                             int count, void* stream);
 
 /*
+ * vbq_chain_* — a decode chain: count batch-1 products y_i = W_i x_i run in
+ * order by one persistent kernel launch (§6 products, one per projection of
+ * a decode step). (The paper has no counterpart; this is an execution mode.)
+ *
+ * vbq_chain_create fixes the chain's layouts, inputs and outputs:
+ *   layouts, xs, ys  host arrays of count pointers: distinct layouts, device
+ *                    x_i (K_i BF16 bit patterns), device y_i (N_i floats,
+ *                    overwritten, distinct; overlap of distinct output ranges
+ *                    is not checked). The layouts must outlive the chain.
+ *   waits            host array of count flags, or NULL for all 1. waits[i] = 1:
+ *                    product i reads x_i only after every earlier product has
+ *                    completed, as when x_i derives from earlier outputs (the
+ *                    default; the results equal those of count vbq_gemv calls
+ *                    in order). waits[i] = 0: product i does not depend on
+ *                    earlier products of the chain. Since no y_i is an input of
+ *                    the chain, a product may zero its own y_i early.
+ *   count            1 .. 2^20.
+ *   out              receives the chain on VBQ_OK.
+ * It allocates a small device buffer (descriptors and completion counts) and
+ * synchronises the device.
+ *
+ * vbq_chain_run launches the chain on `stream`: one block per SM, which
+ * streams its share of every product's packed weights back to back, across
+ * product boundaries (weights never depend on activations), and waits for
+ * earlier products only before it reads x_i. Each y_i satisfies the
+ * accuracy statement of vbq_gemv. x_i must not be written by the chain's own
+ * products. Runs of one chain, and products on its layouts, must not overlap
+ * on the GPU (order them on one stream); the launch uses programmatic
+ * dependent launch like vbq_gemv. It can be captured in a CUDA graph.
+ *
+ * vbq_chain_free releases a chain (NULL is accepted).
+ */
+typedef struct vbq_chain vbq_chain;
+vbq_status_t vbq_chain_create(const vbq_layout* const* layouts, const uint16_t* const* xs, float* const* ys,
+                              const int* waits, int count, vbq_chain** out);
+vbq_status_t vbq_chain_run(const vbq_chain* chain, void* stream);
+vbq_status_t vbq_chain_free(vbq_chain* chain);
+
+/*
  * vbq_gemv_static — vbq_gemv for callers that must not allocate device memory.
  * (The paper has no counterpart; this is an operational variant.)
  *

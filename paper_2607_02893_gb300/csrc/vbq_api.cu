@@ -17,6 +17,13 @@ struct vbq_layout {
     int device = 0;
 };
 
+struct vbq_chain {
+    void* base = nullptr;             // one device allocation: the items, then the control words
+    vbq::ChainItem* items = nullptr;
+    uint32_t* cctl = nullptr;
+    int count = 0, blocks = 0, device = 0;
+};
+
 namespace {
 
 thread_local char g_err[512] = "";
@@ -382,6 +389,84 @@ vbq_status_t vbq_gemv_static(const vbq_layout* L, const uint16_t* x, float* y, v
                     "this layout has %d", vbq::STATIC_CTL_WORDS - 2, (vbq::STATIC_CTL_WORDS - 2) * vbq::RB,
                     L->view.nrb);
     VBQ_CUDA(vbq::launch_gemv1_static(L->view, x, y, static_cast<cudaStream_t>(stream)));
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_chain_create(const vbq_layout* const* layouts, const uint16_t* const* xs, float* const* ys,
+                              const int* waits, int count, vbq_chain** out) {
+    g_err[0] = 0;
+    if (!out) return fail(VBQ_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    if (count < 1 || count > (1 << 20)) return fail(VBQ_ERR_ARG, "count %d outside 1..2^20", count);
+    if (!layouts || !xs || !ys) return fail(VBQ_ERR_ARG, "layouts, xs and ys must be non-NULL arrays");
+    std::vector<vbq::ChainItem> items((size_t)count);
+    std::vector<const void*> seen_l((size_t)count), seen_y((size_t)count);
+    int sms = 0;
+    if (vbq::device_sms(&sms) != 0 || sms < 1) return fail(VBQ_ERR_CUDA, "cannot read the device's SM count");
+    int64_t units_before = 0;
+    int last_wait = 0;                // products before it are complete once it is
+    for (int i = 0; i < count; ++i) {
+        if (!layouts[i] || !layouts[i]->base) return fail(VBQ_ERR_ARG, "layout %d is NULL or empty", i);
+        if (!xs[i] || !ys[i]) return fail(VBQ_ERR_ARG, "x and y of product %d must be non-NULL", i);
+        if (!aligned16(xs[i]) || !aligned16(ys[i]))
+            return fail(VBQ_ERR_ALIGN, "x and y of product %d must be 16-byte aligned", i);
+        if (waits && waits[i] != 0 && waits[i] != 1) return fail(VBQ_ERR_ARG, "waits[%d] must be 0 or 1", i);
+        vbq::ChainItem& it = items[(size_t)i];
+        it.L = layouts[i]->view;
+        it.x = xs[i];
+        it.y = ys[i];
+        const bool w = !waits || waits[i];
+        it.wait_from = w ? last_wait : i;
+        if (w) last_wait = i;
+        it.rot = (int)(units_before % sms);
+        units_before += it.L.units;
+        seen_l[i] = layouts[i];
+        seen_y[i] = ys[i];
+    }
+    std::sort(seen_l.begin(), seen_l.end());
+    std::sort(seen_y.begin(), seen_y.end());
+    if (std::adjacent_find(seen_l.begin(), seen_l.end()) != seen_l.end())
+        return fail(VBQ_ERR_ARG, "a layout appears twice in one chain");
+    if (std::adjacent_find(seen_y.begin(), seen_y.end()) != seen_y.end())
+        return fail(VBQ_ERR_ARG, "an output appears twice in one chain");
+    const size_t items_bytes = round_up(items.size() * sizeof(vbq::ChainItem), 256);
+    // control words: call counter, a completion count per product, the zeroing count
+    const size_t bytes = items_bytes + (3 + (size_t)count) * sizeof(uint32_t);
+    vbq_chain* C = new (std::nothrow) vbq_chain();
+    if (!C) return fail(VBQ_ERR_NOMEM, "host allocation failed");
+    cudaError_t e = cudaMalloc(&C->base, bytes);
+    if (e != cudaSuccess) {
+        delete C;
+        return fail(VBQ_ERR_NOMEM, "cudaMalloc(%zu): %s", bytes, cudaGetErrorString(e));
+    }
+    C->items = static_cast<vbq::ChainItem*>(C->base);
+    C->cctl = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(C->base) + items_bytes);
+    C->count = count;
+    C->blocks = sms;
+    cudaGetDevice(&C->device);
+    if ((e = cudaMemset(C->base, 0, bytes)) == cudaSuccess)
+        e = cudaMemcpy(C->items, items.data(), items.size() * sizeof(vbq::ChainItem), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) {
+        cudaFree(C->base);
+        delete C;
+        return fail(VBQ_ERR_CUDA, "chain set-up: %s", cudaGetErrorString(e));
+    }
+    *out = C;
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_chain_run(const vbq_chain* C, void* stream) {
+    g_err[0] = 0;
+    if (!C || !C->base) return fail(VBQ_ERR_ARG, "chain is NULL or empty");
+    VBQ_CUDA(vbq::launch_chain(C->items, C->count, C->cctl, C->blocks, static_cast<cudaStream_t>(stream)));
+    return VBQ_OK;
+}
+
+vbq_status_t vbq_chain_free(vbq_chain* C) {
+    if (!C) return VBQ_OK;
+    cudaError_t e = C->base ? cudaFree(C->base) : cudaSuccess;
+    delete C;
+    if (e != cudaSuccess) return fail(VBQ_ERR_CUDA, "cudaFree: %s", cudaGetErrorString(e));
     return VBQ_OK;
 }
 

@@ -72,6 +72,20 @@ struct LayoutView {
     int64_t items[4];           // groups per width index (1, 2, 4, 8 bits): host-side launch choices
 };
 
+// One product of a chain (a sequence of batch-1 products run by one
+// persistent kernel, in order): its layout, activation vector and output.
+// Before product i touches x or y, products wait_from .. i - 1 must be
+// complete (wait_from == i: no wait). Block p takes the balanced share of
+// virtual block (p - rot) mod P, so products with fewer units than blocks
+// land on different blocks.
+struct ChainItem {
+    LayoutView L;
+    const uint16_t* x;
+    float* y;
+    int wait_from;
+    int rot;
+};
+
 __host__ __device__ inline int width_of(int w) { return 1 << w; }
 __host__ __device__ inline int unit_rb(const LayoutView& L, int u) { return u % L.nrb; }
 __host__ __device__ inline int unit_slab(const LayoutView& L, int u) { return u / L.nrb; }

@@ -129,6 +129,11 @@ __device__ __forceinline__ float2 ld_relaxed_gpu_f32x2(const float* p) {
     return v;
 }
 
+// Release reduction at GPU scope (no reply): a chain's per-product completion counts.
+__device__ __forceinline__ void red_release_gpu_add(uint32_t* p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+
 // Split-K call counter, control words 0-1 (one 64-bit word): every call adds
 // exactly 2^CALL_SHIFT in all, split over its blocks, so (counter >>
 // CALL_SHIFT) counts the calls before this one; a block that reads it while

@@ -876,6 +876,259 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     }
 }
 
+// ---------------------------------------------------------------------------
+// Chains: a sequence of batch-1 products in one persistent launch (one block
+// per SM). The chain keeps its own control words and never touches its
+// layouts' split-K words. Weights never depend on activations, so each block's copier
+// streams the unit blobs of its share of every product back to back, across
+// product boundaries, while a product that waits for earlier ones (a decode
+// chain: each input derives from earlier outputs) reads its x only once their
+// completion counts say so (the consumers wait before building the product's
+// tables). Each block adds 1 to a product's count (a release reduction) after
+// its last write of that product's y, including blocks that hold none of its
+// units; in launch e (1-based, from the chain's call counter) a product is
+// complete once its count reaches e * P. A block with units of a product adds
+// to its count only after flushing units its consumers computed after that
+// product's wait, so a count at e * P implies that every earlier product the
+// product waited for is complete too.
+// ---------------------------------------------------------------------------
+
+// Units [ub, ue) of product i that block p owns.
+__device__ __forceinline__ void chain_range(const ChainItem* items, int i, int p, int P, int& ub, int& ue) {
+    const int units = items[i].L.units;
+    int q = p - items[i].rot;
+    if (q < 0) q += P;
+    const int per = units / P, extra = units - per * P;
+    ub = q * per + min(q, extra);
+    ue = ub + per + (q < extra ? 1 : 0);
+}
+
+// A position in a block's unit sequence: unit u of product i, whose range ends at ue.
+struct ChainCursor {
+    int i, u, ue;
+};
+
+// Move to the next unit of the block's sequence (products in order, empty
+// ranges skipped); false past the end.
+__device__ __forceinline__ bool chain_next(const ChainItem* items, int count, int p, int P, ChainCursor& c) {
+    if (++c.u < c.ue) return true;
+    while (++c.i < count) {
+        chain_range(items, c.i, p, P, c.u, c.ue);
+        if (c.u < c.ue) return true;
+    }
+    c.i = count;
+    c.u = c.ue = 0;
+    return false;
+}
+
+// True once products from .. to - 1 are complete (count >= target, compared
+// modulo 2^32), within the wait limit. A whole warp: lane l watches products
+// from + l, from + l + 32, ...; the counts are read with acquire loads.
+__device__ __forceinline__ bool chain_deps_ready(const uint32_t* done, int from, int to, uint32_t target, int lane) {
+    bool seen = true;
+    const unsigned long long t0 = global_ns();
+    for (int j = from + lane; j < to && seen; j += 32) {
+        while (!(seen = (int)(ld_acquire_gpu(done + j) - target) >= 0)) {
+            if (global_ns() - t0 > WAIT_LIMIT_NS) break;
+            __nanosleep(32);            // a light backoff: two pollers per block share the count's L2 line
+        }
+    }
+    __syncwarp();
+    return __all_sync(0xffffffffu, seen);
+}
+
+// When the copier's issue position enters a new (product, slab), bring that
+// slab's activations into L2 (a prefetch reads no value, so it is safe however
+// far ahead of the product's dependencies it runs): lane l the l-th 128-byte
+// line of the slab's x.
+__device__ __forceinline__ void chain_prefetch_x(const ChainItem* items, const ChainCursor& c, int& pf_i, int& pf_s,
+                                                 int lane) {
+    const int nrb = items[c.i].L.nrb, s = c.u / nrb;
+    if (c.i == pf_i && s == pf_s) return;
+    pf_i = c.i;
+    pf_s = s;
+    const int C = items[c.i].L.C, G = items[c.i].L.G;
+    const int lines = min(C, G - s * C);                // 64 BF16 activations = one line per group column
+    if (lane < lines) prefetch_l2(items[c.i].x + ((int64_t)s * C + lane) * GROUP);
+}
+
+__global__ void __launch_bounds__(G1_THREADS, 1) gemv_chain_kernel(const ChainItem* __restrict__ items, int count,
+                                                                   uint32_t* __restrict__ cctl) {
+    constexpr int NSTAGE = Geo<1>::nstage;
+    // one team: every consumer warp works on every unit (a chain's products are
+    // serialised, so a unit's latency is what counts; with two teams a block
+    // holding one unit of a product computes it on half its warps)
+    constexpr int TW = NCW;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    unsigned char* base = smem_raw + ((256u - (smem_u32(smem_raw) & 255u)) & 255u);
+    TablesT<1>& T = *reinterpret_cast<TablesT<1>*>(base + (size_t)NSTAGE * STAGE_BYTES);
+    const uint32_t stage0 = smem_u32(base);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int P = gridDim.x, p = blockIdx.x;
+    uint32_t* done = cctl + 2;
+
+    const uint32_t full0 = smem_u32(&T.full[0]), empty0 = smem_u32(&T.empty[0]);
+    const uint32_t abort_addr = smem_u32(&T.abort);
+    if (tid == 0) {
+        for (int i = 0; i < NSTAGE; ++i) {
+            mbar_init(full0 + 8 * i, 1);
+            mbar_init(empty0 + 8 * i, TW);
+        }
+        T.abort = 0;
+        fence_barrier_init();
+    }
+    for (int i = tid; i < NSTAGE * SLOT_FLOATS; i += G1_THREADS) (&T.slots[0][0][0])[i] = 0.f;
+    __syncthreads();
+    // the copier's issue position, and the first copies (weights only: before
+    // the wait for the previous kernel)
+    ChainCursor is{-1, 0, 0};
+    int issued = 0, pf_i = -1, pf_s = -1;
+    if (warp == 0) {
+        while (issued < NSTAGE && chain_next(items, count, p, P, is)) {
+            if (lane == 0) issue_unit(items[is.i].L, is.u, stage0 + issued * STAGE_BYTES, full0 + 8 * issued);
+            chain_prefetch_x(items, is, pf_i, pf_s, lane);
+            ++issued;
+        }
+    }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const uint32_t target = call_epoch(cctl) * (uint32_t)P;
+    uint32_t* zeroed = cctl + 2 + count;
+    // Split-K for the whole chain at once: every block zeroes the rows of the
+    // slab-0 units it owns in every product whose rows span several slabs (no
+    // y is an input of the chain, so this may run ahead of any product), then
+    // counts itself in `zeroed`; a copier adds into y only once every block
+    // has (one grid-wide wait per launch instead of flags per product).
+    for (int i = warp; i < count; i += G1_THREADS / 32) {
+        const LayoutView& Li = items[i].L;
+        if (Li.S > 1) {
+            int ub, ue;
+            chain_range(items, i, p, P, ub, ue);
+            float* y = items[i].y;
+            const int z_end = min(ue, Li.nrb);
+            for (int u = ub; u < z_end; ++u) {
+                const int rows = min(RB, (int)(Li.N - (int64_t)u * RB));
+                for (int r = lane; r < rows; r += 32) y[(int64_t)u * RB + r] = 0.f;
+            }
+        }
+    }
+    __syncthreads();
+    if (tid == 0) red_release_gpu_add(zeroed, 1u);
+
+    if (warp == 0) {
+        // ---- copier: per product, split-K zeroing, then per unit rows out and
+        // the next copy of the block's sequence in; then the product's count ----
+        bool dead = false, zero_seen = false;
+        int st = 0;
+        uint32_t par = 0;
+        for (int i = 0; i < count; ++i) {
+            const LayoutView L = items[i].L;
+            float* y = items[i].y;
+            int ub, ue;
+            chain_range(items, i, p, P, ub, ue);
+            if (ub < ue) {
+                // no dependency wait here: y's values come from units the consumers
+                // compute only after the product's dependencies
+                if (!dead && L.S > 1 && !zero_seen) {
+                    if (!chain_deps_ready(zeroed, 0, 1, target, lane)) {
+                        dead = true;
+                        if (lane == 0) raise_abort(&T.abort);
+                    }
+                    zero_seen = true;
+                }
+                for (int u = ub; u < ue; ++u) {
+                    if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, 0)) {
+                        dead = true;
+                        if (lane == 0) raise_abort(&T.abort);
+                    }
+                    if (!dead) {
+                        const int rb = u % L.nrb;
+                        const int rows = min(RB, (int)(L.N - (int64_t)rb * RB));
+                        const uint32_t sl = smem_u32(T.slots[st][0]);
+                        float* yr = y + (int64_t)rb * RB;
+#pragma unroll
+                        for (int q = 0; q < RB / 32; ++q) {
+                            const int r = lane + 32 * q;
+                            const uint32_t ra = sl + (uint32_t)r * 64;
+                            float4 a[4];
+#pragma unroll
+                            for (int k = 0; k < 4; ++k) a[k] = lds_f32x4(ra + (((k + (lane >> 1)) & 3) << 4));
+#pragma unroll
+                            for (int k = 0; k < 4; ++k) sts_zero4(ra + (((k + (lane >> 1)) & 3) << 4));
+                            const float sum = (((a[0].x + a[0].y) + (a[0].z + a[0].w)) + ((a[1].x + a[1].y) + (a[1].z + a[1].w))) +
+                                              (((a[2].x + a[2].y) + (a[2].z + a[2].w)) + ((a[3].x + a[3].y) + (a[3].z + a[3].w)));
+                            if (r < rows) {
+                                if (L.S == 1) yr[r] = sum;
+                                else red_global(yr + r, sum);
+                            }
+                        }
+                        __syncwarp();
+                        if (chain_next(items, count, p, P, is)) {      // the unit NSTAGE ahead, into the freed stage
+                            if (lane == 0) issue_unit(items[is.i].L, is.u, stage0 + st * STAGE_BYTES, full0 + 8 * st);
+                            chain_prefetch_x(items, is, pf_i, pf_s, lane);
+                            ++issued;
+                        }
+                    }
+                    if (++st == NSTAGE) { st = 0; par ^= 1; }
+                }
+            }
+            // this block is done with product i (its writes of y, ordered before
+            // the release by the warp barrier); every block counts every product
+            __syncwarp();
+            if (lane == 0) red_release_gpu_add(done + i, 1u);
+        }
+        if (dead && lane == 0) {
+            for (int i = 0; i < NSTAGE && i < issued; ++i) {
+                const int jl = i + ((issued - 1 - i) / NSTAGE) * NSTAGE;   // last unit issued into stage i
+                mbar_wait_bounded(full0 + 8 * i, (uint32_t)((jl / NSTAGE) & 1));
+            }
+        }
+        if (lane == 0) call_done(cctl);
+    } else {
+        // ---- consumers: every warp takes part in every unit, rebuilding the
+        // tables at every (product, slab) boundary of the block's sequence ----
+        const int wt = warp - 1, ct = tid - 32;
+        bool dead = false;
+        ChainCursor c{-1, 0, 0};
+        int tb_i = -1, tb_s = -1;
+        LayoutView L = items[0].L;
+        const uint16_t* x = items[0].x;
+        for (int j = 0; chain_next(items, count, p, P, c); ++j) {
+            const bool new_product = c.i != tb_i;
+            if (new_product) {
+                L = items[c.i].L;
+                x = items[c.i].x;
+                const int wf = items[c.i].wait_from;
+                // the first consumer warp waits for the product's dependencies; the
+                // table build's barrier holds the others until it is through
+                if (ct < 32 && !dead && wf < c.i && !chain_deps_ready(done, wf, c.i, target, lane)) {
+                    dead = true;
+                    if (lane == 0) raise_abort(&T.abort);
+                }
+            }
+            const int sj = c.u / L.nrb;
+            if (new_product || sj != tb_s) {
+                build_tables<1, MODE_PLAIN>(T, L, x, nullptr, sj, ct);
+                tb_i = c.i;
+                tb_s = sj;
+            }
+            {
+                const int st = j & (NSTAGE - 1);
+                const uint32_t par = (uint32_t)(j / NSTAGE) & 1u;
+                if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
+                if (!dead) {
+                    // tasks rotate over the warps from unit to unit
+                    const int t0 = (wt - j) & (TW - 1);
+                    consume_unit<1>(T, stage0 + st * STAGE_BYTES, L.C, min(L.C, L.G - sj * L.C), smem_u32(T.slots[st][0]),
+                                    t0, TW, lane);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(empty0 + 8 * st);
+                }
+            }
+        }
+    }
+}
+
 int g_sms = 0;
 
 template <int NX, int MODE = MODE_PLAIN>
@@ -908,6 +1161,36 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
 }
 
 }  // namespace
+
+int device_sms(int* sms) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev);
+    return (int)e;
+}
+
+cudaError_t launch_chain(const ChainItem* items, int count, uint32_t* cctl, int blocks, cudaStream_t s) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        const cudaError_t e = cudaFuncSetAttribute(gemv_chain_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   (int)gemv1_smem<1>());
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(blocks);
+    cfg.blockDim = dim3(G1_THREADS);
+    cfg.dynamicSmemBytes = gemv1_smem<1>();
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, gemv_chain_kernel, items, count, cctl);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
 
 // ---------------------------------------------------------------------------
 // Batch 1 with the split-K control words in a fixed device array instead of

@@ -57,6 +57,14 @@ cudaError_t launch_gemv_swiglu(const LayoutView& L, const uint16_t* x, float* y,
 // gate-up product with alternating rows); h never reaches memory.
 cudaError_t launch_gemv_swiglu_in(const LayoutView& L, const float* gu, float* y, cudaStream_t s);
 
+// A chain of count batch-1 products in one persistent launch of blocks
+// blocks (every product's ChainItem::rot computed for that count). cctl:
+// 3 + count zero-initialised words owned by the chain (call counter, one
+// completion count per product, then the count of blocks that have zeroed
+// their split-K rows).
+cudaError_t launch_chain(const ChainItem* items, int count, uint32_t* cctl, int blocks, cudaStream_t s);
+int device_sms(int* sms);   // the current device's SM count (0 on success)
+
 // Batch 1 with the split-K control words in a fixed device array (no
 // allocation anywhere); usable for layouts with at most STATIC_CTL_WORDS - 2
 // row blocks.

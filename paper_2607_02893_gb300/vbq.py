@@ -38,6 +38,10 @@ SIGNATURES = {
     "vbq_gemv_static": (_I, [_P, _P, _P, _P]),
     "vbq_gemv_swiglu": (_I, [_P, _P, _P, _P, _P]),
     "vbq_gemv_swiglu_in": (_I, [_P, _P, _P, _P]),
+    "vbq_chain_create": (_I, [ctypes.POINTER(_P), ctypes.POINTER(_P), ctypes.POINTER(_P),
+                              ctypes.POINTER(_I), _I, ctypes.POINTER(_P)]),
+    "vbq_chain_run": (_I, [_P, _P]),
+    "vbq_chain_free": (_I, [_P]),
     "vbq_gemv_group": (_I, [ctypes.POINTER(_P), ctypes.POINTER(_P), ctypes.POINTER(_P), _I, _P]),
     "vbq_device_status": (_I, [_P]),
     "vbq_selftest_timeout": (_I, [_I, _P]),
@@ -208,6 +212,54 @@ def vbq_gemv_group(layouts, xs, ys, stream=None) -> None:
     xa = arr(*[_ptr(x) for x in xs])
     ya = arr(*[_ptr(y) for y in ys])
     _check(load().vbq_gemv_group(la, xa, ya, int(n), _stream(stream, *(list(xs) + list(ys)))))
+
+
+class Chain:
+    """Owns one vbq_chain*: products run in order by one persistent launch.
+    Keeps references to its layouts and buffers so they outlive it."""
+
+    def __init__(self, layouts, xs, ys, waits=None):
+        n = len(layouts)
+        if len(xs) != n or len(ys) != n or (waits is not None and len(waits) != n):
+            raise ValueError("layouts, xs, ys (and waits) must have the same length")
+        arr = _P * max(n, 1)
+        la = arr(*[lay._as_parameter_ for lay in layouts])
+        xa = arr(*[_ptr(x) for x in xs])
+        ya = arr(*[_ptr(y) for y in ys])
+        wa = None if waits is None else (_I * n)(*[int(w) for w in waits])
+        out = ctypes.c_void_p()
+        self.handle = None
+        _check(load().vbq_chain_create(la, xa, ya, wa, int(n), ctypes.byref(out)))
+        self.handle = out.value
+        self._keep = (list(layouts), list(xs), list(ys))
+
+    def run(self, stream=None) -> None:
+        if not self.handle:
+            raise ValueError("chain already freed")
+        _check(load().vbq_chain_run(self.handle, _stream(stream, *self._keep[2])))
+
+    def free(self) -> None:
+        if self.handle:
+            h, self.handle = self.handle, None
+            _check(load().vbq_chain_free(h))
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def vbq_chain_create(layouts, xs, ys, waits=None) -> Chain:
+    return Chain(layouts, xs, ys, waits)
+
+
+def vbq_chain_run(chain: Chain, stream=None) -> None:
+    chain.run(stream)
+
+
+def vbq_chain_free(chain: Chain) -> None:
+    chain.free()
 
 
 def vbq_gemm_small(layout: Layout, X, Y, B: Optional[int] = None, stream=None) -> None:

@@ -85,6 +85,20 @@ def test_calls_reject_null_layout(lib):
     assert lib.vbq_gemm_small(None, None, None, 4, None) == -1
     assert lib.vbq_gemv_swiglu(None, None, None, None, None) == -1
     assert lib.vbq_gemv_swiglu_in(None, None, None, None) == -1
+    assert lib.vbq_chain_run(None, None) == -1
+    assert lib.vbq_chain_free(None) == 0
+
+
+def test_chain_rejects_bad_arguments_on_host(lib):
+    P = ctypes.c_void_p
+    arr = (P * 2)()
+    out = P(7)
+    assert lib.vbq_chain_create(arr, arr, arr, None, 2, None) == -1         # out NULL
+    assert lib.vbq_chain_create(None, arr, arr, None, 2, ctypes.byref(out)) == -1
+    assert out.value is None                                               # cleared on error
+    assert lib.vbq_chain_create(arr, arr, arr, None, 0, ctypes.byref(out)) == -1   # empty chain
+    assert lib.vbq_chain_create(arr, arr, arr, None, -3, ctypes.byref(out)) == -1
+    assert b"count" in lib.vbq_last_error()
     assert lib.vbq_dequant(None, None, None, None, None, None) == -1
     assert lib.vbq_packed_bytes(None, None, None, None) == -1
     assert lib.vbq_layout_shape(None, None, None) == -1
