@@ -17,6 +17,9 @@ What it defines (paper: "Variable Bit-width Quantization", arXiv 2607.02893):
   boundaries"), i.e. 8*b bytes, plus its scale.
 * The inference product (§6): y = W_hat x with the weights never widened in
   memory; here simply the plain dense definition in fp64.
+* The training-time soft-quantised forward (§3.2, Alg. 1): per group, the
+  convex combination of the four candidate reconstructions under
+  pi = softmax((l + e) / tau), the expected width and the hardened width.
 * SwiGLU on a gate-up product (the models' MLP, §4; §6 relies on
   silu(0) * u = 0): h = silu(gate) * up with silu(z) = z / (1 + exp(-z)),
   gate and up rows alternating (row 2i gate i, row 2i + 1 up i), fp64.
@@ -239,6 +242,110 @@ def quantize(w: np.ndarray, widths: np.ndarray):
             codes[r, g * GROUP:(g + 1) * GROUP] = c
             scales[r, g] = s
     return codes, scales
+
+
+# ---------------------------------------------------------------------------
+# Training-time soft quantisation (§3.2 differentiable bit selection, Alg. 1)
+# ---------------------------------------------------------------------------
+
+CANDIDATES = (1, 2, 4, 8)          # the candidate widths B_k, in the order of the logits
+
+
+def reconstruct_fp32(w_group, b: int) -> np.ndarray:
+    """The reconstruction of one group at width b as a float32 training forward
+    computes it (§3.1): b >= 2, s = max|w| / (2^(b-1) - 1) and
+    s * clip(round(w / s)) (Eq. 1); b = 1, sign(w) * mean|w| (sign(0) = +1).
+    The integer decisions (the codes) are taken in float32, as the framework
+    evaluating Eq. 1 on float32 weights takes them: s and w / s are float32
+    quotients, rounded half to even. The values are returned in fp64 (s * q is
+    exact there; the 1-bit mean is the fp64 pairwise sum / 64). A group whose
+    float32 s is 0 reconstructs as 0."""
+    w32 = np.asarray(w_group, dtype=np.float32)
+    if not np.isfinite(w32).all():
+        raise ValueError("non-finite weight")
+    if b == 1:
+        mean = pairwise_sum(np.abs(w32.astype(np.float64))) / w32.size
+        return np.where(w32 >= 0, 1.0, -1.0) * mean
+    if b not in (2, 4, 8):
+        raise ValueError(f"width {b} not in {WIDTHS}")
+    qmax = np.float32((1 << (b - 1)) - 1)
+    s = np.float32(np.max(np.abs(w32)) / qmax)
+    if s == 0:
+        return np.zeros(w32.shape, dtype=np.float64)
+    t = (w32 / s).astype(np.float32)
+    q = np.clip(np.rint(t), -qmax, qmax)          # np.rint: ties to even
+    return q.astype(np.float64) * float(s)
+
+
+def soft_select(logits, gumbel, tau: float) -> np.ndarray:
+    """pi = softmax((l + e) / tau) over the last axis (the 4 candidates), fp64;
+    gumbel may be None (no noise)."""
+    z = np.asarray(logits, dtype=np.float64)
+    if gumbel is not None:
+        z = z + np.asarray(gumbel, dtype=np.float64)
+    z = z / tau
+    z = z - z.max(axis=-1, keepdims=True)
+    p = np.exp(z)
+    return p / p.sum(axis=-1, keepdims=True)
+
+
+def soft_quant_forward(w, logits, gumbel, tau: float):
+    """The soft-quantised forward of one matrix (§3.2, Alg. 1's weight step):
+    per group g, pi_g = softmax((l_g + e_g) / tau), w_soft = sum_k pi_gk *
+    w_hat^(B_k) (reconstruct_fp32), the group's expected width sum_k pi_gk B_k
+    (whose mean over groups is Alg. 1's b-bar), and the hardened width
+    B_argmax_k l_gk (the first maximum on ties; Alg. 1's return).
+    w: N x K, logits and gumbel: N x (K/64) x 4 (gumbel may be None).
+    Returns (w_soft N x K, exp_bits N x G, hard N x G uint8, pi N x G x 4)."""
+    w = np.asarray(w, dtype=np.float32)
+    n, k = w.shape
+    g = k // GROUP
+    logits = np.asarray(logits, dtype=np.float32)
+    if k % GROUP or logits.shape != (n, g, 4):
+        raise ValueError("bad shapes")
+    pi = soft_select(logits, gumbel, tau)
+    cand = np.array(CANDIDATES, dtype=np.float64)
+    exp_bits = (pi * cand).sum(axis=-1)
+    hard = np.array(CANDIDATES, dtype=np.uint8)[np.argmax(logits, axis=-1)]   # argmax: the first maximum
+    w_soft = np.empty((n, k), dtype=np.float64)
+    for r in range(n):
+        for j in range(g):
+            wg = w[r, j * GROUP:(j + 1) * GROUP]
+            acc = np.zeros(GROUP)
+            for kk, b in enumerate(CANDIDATES):
+                acc += pi[r, j, kk] * reconstruct_fp32(wg, b)
+            w_soft[r, j * GROUP:(j + 1) * GROUP] = acc
+    return w_soft, exp_bits, hard, pi
+
+
+def soft_quant_within_bound(w_soft, exp_bits, w, logits, gumbel, tau: float):
+    """Acceptance of a float32 evaluation of soft_quant_forward: per group,
+    eps = 2^-20 (1 + max_k |z_k|) with z = (l + e) / tau bounds the relative
+    error of each pi_k (z's float32 rounding moves each pi_k by at most
+    2 max|dz| relatively, plus exp and the normalisation's roundings, with a
+    factor 2 to spare). Then |dw_soft| <= (eps + 2^-20) sum_k pi_k |w_hat_k|
+    (each w_hat_k within 2^-21 relatively, the 4-term float32 sum within
+    2^-22) and |d exp_bits| <= (eps + 2^-20) sum_k pi_k B_k.
+    Returns (ok_w N x K, ok_bits N x G)."""
+    w = np.asarray(w, dtype=np.float32)
+    n, k = w.shape
+    g = k // GROUP
+    ref_w, ref_b, _, pi = soft_quant_forward(w, logits, gumbel, tau)
+    z = np.asarray(logits, dtype=np.float64)
+    if gumbel is not None:
+        z = z + np.asarray(gumbel, dtype=np.float64)
+    z = z / tau
+    eps = 2.0 ** -20 * (1.0 + np.abs(z).max(axis=-1)) + 2.0 ** -20          # N x G
+    mag = np.zeros((n, k))
+    for r in range(n):
+        for j in range(g):
+            wg = w[r, j * GROUP:(j + 1) * GROUP]
+            for kk, b in enumerate(CANDIDATES):
+                mag[r, j * GROUP:(j + 1) * GROUP] += pi[r, j, kk] * np.abs(reconstruct_fp32(wg, b))
+    tol_w = np.repeat(eps, GROUP, axis=1) * mag
+    ok_w = np.abs(np.asarray(w_soft, dtype=np.float64) - ref_w) <= tol_w
+    ok_b = np.abs(np.asarray(exp_bits, dtype=np.float64) - ref_b) <= eps * ref_b
+    return ok_w, ok_b
 
 
 # ---------------------------------------------------------------------------

@@ -254,6 +254,94 @@ def pin_payload_accounting(O, seed=6):
     _check(np.array_equal(O.unpack_lsb(buf, widths), codes), "pack/unpack roundtrip")
 
 
+def pin_soft_quant(O):
+    """The training-time soft forward (§3.2, Alg. 1) by closed forms and by the
+    export quantiser: equal logits give pi = 1/4 and an expected width of
+    (1 + 2 + 4 + 8) / 4 = 3.75; a dominant logit selects that candidate's
+    reconstruction, which is the weight itself for a group on its grid with a
+    power-of-two scale; e is added to l and tau divides both; the hardened
+    width is the first maximum's candidate; and the float32 reconstructions
+    agree with the (separately pinned) fp64 quantiser wherever no quotient
+    lies near a rounding tie."""
+    B = (1, 2, 4, 8)
+    _check(tuple(O.CANDIDATES) == B, f"candidates {O.CANDIDATES}")
+    rng = np.random.default_rng(31)
+    # equal logits: uniform selection
+    w = rng.normal(0, 0.02, (3, 128)).astype(np.float32)
+    lg = np.full((3, 2, 4), 0.7, np.float32)
+    ws, eb, hard, pi = O.soft_quant_forward(w, lg, None, 0.9)
+    _check(np.allclose(pi, 0.25, rtol=0, atol=1e-15), "equal logits -> pi = 1/4")
+    _check(np.allclose(eb, 3.75, rtol=0, atol=1e-14), f"expected width {eb}")
+    for r in range(3):
+        for j in range(2):
+            wg = w[r, 64 * j:64 * j + 64]
+            mean = sum(O.reconstruct_fp32(wg, b) for b in B) / 4.0
+            _check(np.allclose(ws[r, 64 * j:64 * j + 64], mean, rtol=1e-13, atol=0), "uniform mixture")
+    # a dominant logit selects its candidate; on-grid groups reconstruct exactly
+    for kk, b in enumerate(B[1:], start=1):
+        qmax = (1 << (b - 1)) - 1
+        q = rng.integers(-qmax, qmax + 1, size=64)
+        q[5], q[40] = qmax, -qmax
+        wg = (q * 2.0 ** -9).astype(np.float32)[None, :]
+        lg1 = np.zeros((1, 1, 4), np.float32)
+        lg1[0, 0, kk] = 60.0
+        ws1, eb1, hard1, _ = O.soft_quant_forward(wg, lg1, None, 1.0)
+        _check(np.allclose(ws1[0], wg[0].astype(np.float64), rtol=1e-20, atol=1e-24),
+               f"dominant {b}-bit logit on its grid")
+        _check(abs(eb1[0, 0] - b) < 1e-20 * 8 + 1e-22, f"dominant {b}-bit expected width {eb1}")
+        _check(int(hard1[0, 0]) == b, f"hardened {hard1}")
+    # exact ties of the float32 quotient round half to even: at 4 bits with
+    # max|w| = 7 * 2^-6 the scale is 2^-6, and w = (k + 1/2) 2^-6 lands on k + 1/2
+    halves = [0.5, 1.5, 2.5, 3.5, 4.5, 5.5, 6.5, -0.5, -1.5, -2.5, -6.5]
+    want_q = [0, 2, 2, 4, 4, 6, 6, 0, -2, -2, -6]          # by hand: the even neighbour
+    wt = np.zeros(64, np.float32)
+    wt[:len(halves)] = np.array(halves) * 2.0 ** -6
+    wt[63] = 7 * 2.0 ** -6
+    rt = O.reconstruct_fp32(wt, 4)
+    _check(np.array_equal(rt[:len(halves)], np.array(want_q, dtype=np.float64) * 2.0 ** -6),
+           f"ties to even: {rt[:len(halves)] / 2.0 ** -6}")
+    # 1 bit: a constant-magnitude group reconstructs exactly, sign(0) = +1
+    wc = np.where(rng.random(64) < 0.5, -0.03, 0.03).astype(np.float32)
+    wc[7] = 0.0
+    r1 = O.reconstruct_fp32(wc, 1)
+    m = float(np.abs(wc.astype(np.float64)).sum()) / 64
+    _check(r1[7] == m and np.allclose(np.abs(r1), m, rtol=0, atol=0), "1-bit sign * mean")
+    _check(np.array_equal(np.sign(r1[wc != 0]), np.sign(wc[wc != 0])), "1-bit signs")
+    # noise is added to the logits, tau divides both, and a shift cancels
+    l2 = rng.normal(0, 2, (2, 3, 4)).astype(np.float32)
+    e2 = rng.gumbel(size=(2, 3, 4)).astype(np.float32)
+    p_a = O.soft_select(l2, e2, 0.5)
+    p_b = O.soft_select(l2.astype(np.float64) + e2, None, 0.5)
+    p_c = O.soft_select((l2.astype(np.float64) + e2) / 0.5 + 3.0, None, 1.0)
+    _check(np.allclose(p_a, p_b, rtol=1e-14, atol=0) and np.allclose(p_a, p_c, rtol=1e-12, atol=0),
+           "softmax of (l + e) / tau")
+    _check(np.allclose(p_a.sum(-1), 1.0, atol=1e-15), "pi sums to 1")
+    z = (l2.astype(np.float64) + e2) / 0.5
+    ratio = p_a[..., 3] / p_a[..., 0]
+    _check(np.allclose(ratio, np.exp(z[..., 3] - z[..., 0]), rtol=1e-12), "pi ratio = exp(z3 - z0)")
+    # hardened widths: the first maximum
+    lh = np.array([[[1, 3, 3, 0], [5, 5, 5, 5], [0, 0, 0, 1], [-1, -2, -3, -0.5]]], np.float32)
+    _, _, hh, _ = O.soft_quant_forward(np.zeros((1, 256), np.float32), lh, None, 1.0)
+    _check(hh[0].tolist() == [2, 1, 8, 8], f"hardened widths {hh}")
+    # float32 reconstructions against the fp64 export quantiser (unrounded scale)
+    agree = 0
+    for _ in range(200):
+        wg = (rng.normal(0, 0.02, 64) * np.exp(rng.normal(0, 1))).astype(np.float32)
+        for b in (2, 4, 8):
+            qmax = (1 << (b - 1)) - 1
+            s64 = float(np.max(np.abs(wg.astype(np.float64)))) / qmax
+            frac = np.abs(wg.astype(np.float64) / s64)
+            if np.min(np.abs(frac - np.floor(frac) - 0.5)) < 1e-5:
+                continue                    # a quotient near a tie: the precisions may differ
+            codes, _ = O.quantize_group(wg.astype(np.float64), b, fp16_scale=False)
+            q_ref = codes.astype(np.int64) - (1 << (b - 1))
+            rec = O.reconstruct_fp32(wg, b)
+            s32 = float(np.float32(np.max(np.abs(wg)) / np.float32(qmax)))
+            _check(np.array_equal(np.rint(rec / s32).astype(np.int64), q_ref), f"{b}-bit codes vs the quantiser")
+            agree += 1
+    _check(agree > 400, f"only {agree} comparisons")
+
+
 ALL_PINS = [pin_eq1_golden, pin_level_grid, pin_grid_roundtrip, pin_quantizer_invariants,
             pin_one_bit_mean_order, pin_group_size_one, pin_integer_gemv, pin_exact_rational, pin_enumerated_codes,
-            pin_swiglu, pin_payload_accounting]
+            pin_swiglu, pin_soft_quant, pin_payload_accounting]

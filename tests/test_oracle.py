@@ -59,6 +59,19 @@ MUTATIONS = {
     "silu_sign": ("return z / (1.0 + np.exp(-z))", "return z / (1.0 + np.exp(z))"),
     "scale_bytes_one": ("return 2 * int(np.asarray(widths).size)",
                         "return int(np.asarray(widths).size)"),
+    "soft_tau_ignored": ("    z = z / tau\n    z = z - z.max(axis=-1, keepdims=True)",
+                         "    z = z - z.max(axis=-1, keepdims=True)"),
+    "soft_noise_subtracted": ("        z = z + np.asarray(gumbel, dtype=np.float64)\n    z = z / tau\n    z = z - z.max(",
+                              "        z = z - np.asarray(gumbel, dtype=np.float64)\n    z = z / tau\n    z = z - z.max("),
+    "soft_candidates_reversed": ("CANDIDATES = (1, 2, 4, 8)", "CANDIDATES = (8, 4, 2, 1)"),
+    "soft_not_normalised": ("    return p / p.sum(axis=-1, keepdims=True)", "    return p"),
+    "soft_round_half_away": ("q = np.clip(np.rint(t), -qmax, qmax)", "q = np.clip(np.floor(t + 0.5), -qmax, qmax)"),
+    "soft_one_bit_max": ("        mean = pairwise_sum(np.abs(w32.astype(np.float64))) / w32.size",
+                         "        mean = float(np.max(np.abs(w32)))"),
+    "soft_qmax_too_large": ("    qmax = np.float32((1 << (b - 1)) - 1)", "    qmax = np.float32(1 << (b - 1))"),
+    "soft_hard_last_max": ("[np.argmax(logits, axis=-1)]",
+                           "[3 - np.argmax(logits[..., ::-1], axis=-1)]"),
+    "soft_expected_bits_unweighted": ("    exp_bits = (pi * cand).sum(axis=-1)", "    exp_bits = pi.sum(axis=-1) * cand.mean()"),
 }
 
 
