@@ -25,7 +25,9 @@ chain without waits: independent products in one persistent launch, the
 kernel's streaming upper bound), `grouped` (all of the headline's layouts as one
 vbq_gemv_group per step: independent products whose launches overlap, the
 streaming upper bound) and `cublas_bf16` (dense BF16 weights of the same
-shapes through torch.mv, i.e. cuBLAS, as a reference point).
+shapes through torch.mv, i.e. cuBLAS, as a reference point), and, on the
+workload's largest non-head matrix, `quantize` (vbq_quantize, the export-time
+quantiser) and `soft_quant` (vbq_soft_quant, the training-time soft forward).
 
 Printed JSON line (rank 0):
   value         algorithmic HBM GB/s of the whole step: sum over GEMVs of
@@ -51,7 +53,6 @@ pass over all copies, and tokens/s counts one token per copy.
 from __future__ import annotations
 
 import argparse
-import glob
 import hashlib
 import json
 import os
@@ -99,14 +100,18 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+# the sources that define the batch-1 GEMV kernel's code (the profiled kernel)
+GEMV_SOURCES = ("vbq_common.cuh", "vbq_device.cuh", "vbq_gemv.cu")
+
+
 def kernel_source_hash() -> str:
-    """sha256 over the CUDA sources of libvbq (sorted by name)."""
+    """sha256 over the CUDA sources that define the GEMV kernel (sorted by name)."""
     h = hashlib.sha256()
-    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2607_02893_gb300", "csrc", "*"))):
-        if f.endswith((".cu", ".cuh", ".h")):
-            h.update(os.path.basename(f).encode())
-            with open(f, "rb") as fh:
-                h.update(fh.read())
+    for name in sorted(GEMV_SOURCES):
+        f = os.path.join(ROOT, "paper_2607_02893_gb300", "csrc", name)
+        h.update(name.encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
     return h.hexdigest()
 
 
@@ -481,7 +486,46 @@ def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev
                                "quantisation kernel; value counts 4 B in and 1 B out per weight"}
     del w, wd, qc, qs
     torch.cuda.empty_cache()
+    try:
+        out["soft_quant"] = soft_quant_mode(torch, vbq, big, dev)
+    except Exception as e:                      # a companion never takes the headline down
+        out["soft_quant"] = {"error": f"{type(e).__name__}: {e}"}
     return out
+
+
+def soft_quant_mode(torch, vbq, spec, dev):
+    """The training-time soft forward (vbq_soft_quant, §3.2 / Alg. 1) on the
+    workload's largest non-head matrix: median of 10 calls, each after an L2
+    flush, timed with events."""
+    from synth import gen
+    n, k = spec.n, spec.k
+    w, lg, gb = gen.draw_soft_inputs(n, k, gen.rng_for((72, n, k)))
+    W, L, E = (torch.from_numpy(a).to(dev) for a in (w, lg, gb))
+    ws = torch.empty_like(W)
+    eb = torch.empty((n, k // 64), dtype=torch.float32, device=dev)
+    hw = torch.empty((n, k // 64), dtype=torch.uint8, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        vbq.vbq_soft_quant(W, L, 0.5, gumbel=E, w_soft=ws, exp_bits=eb, hard_widths=hw)
+    times = []
+    for _ in range(10):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        vbq.vbq_soft_quant(W, L, 0.5, gumbel=E, w_soft=ws, exp_bits=eb, hard_widths=hw)
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    ms = statistics.median(times)
+    groups = n * k // 64
+    nbytes = n * k * 8 + groups * (16 + 16 + 4 + 1)
+    del W, L, E, ws, eb, hw, flush
+    torch.cuda.empty_cache()
+    return {"ms_per_call": round(ms, 4), "value": round(nbytes / (ms * 1e-3) / 1e9, 1), "unit": "GB/s",
+            "weights_per_s": round(n * k / (ms * 1e-3), 1), "shape": [n, k],
+            "note": "vbq_soft_quant (training-time soft forward: pi = softmax((l + e) / tau), the convex "
+                    "combination of the 1/2/4/8-bit reconstructions, expected and hardened widths) at tau 0.5 "
+                    "with Gumbel noise; value counts 4 B in and 4 B out per weight, 32 B in and 5 B out per group"}
 
 
 def run_ours(args, rank, world, local_rank):

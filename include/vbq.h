@@ -89,6 +89,36 @@ vbq_status_t vbq_quantize(const float* w, const uint8_t* bitwidths, int64_t N, i
                           uint8_t* codes_out, uint16_t* scales_out, void* stream);
 
 /*
+ * vbq_soft_quant — the training-time soft-quantised forward of one matrix
+ * (§3.2, differentiable bit selection; the weight step of Alg. 1). Per group g
+ * of 64 weights along K:
+ *   pi_g      = softmax((l_g + e_g) / tau) over the candidates B = {1, 2, 4, 8};
+ *   w_soft    = sum_k pi_gk * w_hat^(B_k), the candidate reconstructions of §3.1
+ *               (Eq. 1 with s = max|w| / (2^(b-1) - 1) at 2, 4 and 8 bits;
+ *               sign(w) * mean|w| at 1 bit, sign(0) = +1; a zero scale gives 0);
+ *   exp_bits  = sum_k pi_gk B_k (the mean over groups is Alg. 1's b-bar);
+ *   hard      = B_argmax_k l_gk (the first maximum; Alg. 1's hardened width).
+ * The reconstructions' integer decisions are float32 operations, as a float32
+ * training framework takes them: s and w / s are correctly rounded float32
+ * quotients, rounded half to even, then clipped. The rest is float32 with a few
+ * ulps of rounding (w_soft within (eps + 2^-20) sum_k pi_k |w_hat_k| and
+ * exp_bits within (eps + 2^-20) exp_bits, eps = 2^-20 (1 + max_k |z_k|),
+ * z = (l + e) / tau).
+ *
+ *   w            device, N x K float32, finite (not checked).
+ *   logits       device, N x (K/64) x 4 float32, finite.
+ *   gumbel       device, N x (K/64) x 4 float32 noise e, or NULL for none.
+ *   tau          the temperature, > 0 and finite (VBQ_ERR_ARG otherwise).
+ *   N, K         K % 64 == 0 (VBQ_ERR_SHAPE), N * K <= 2^40.
+ *   w_soft       device, N x K float32; overwritten.
+ *   exp_bits     device, N x (K/64) float32, or NULL.
+ *   hard_widths  device, N x (K/64) uint8, or NULL.
+ * Enqueued on `stream`; allocates nothing.
+ */
+vbq_status_t vbq_soft_quant(const float* w, const float* logits, const float* gumbel, float tau, int64_t N,
+                            int64_t K, float* w_soft, float* exp_bits, uint8_t* hard_widths, void* stream);
+
+/*
  * vbq_pack — build the packed device layout of one matrix (§6: the export
  * step that turns per-group codes into packed storage; §3.1 groups of 64).
  *

@@ -1,6 +1,7 @@
 // vbq_api.cu — the C ABI declared in include/vbq.h: argument validation,
 // layout planning and allocation, and kernel dispatch on the caller's stream.
 #include <algorithm>
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -88,6 +89,23 @@ const char* vbq_status_string(vbq_status_t st) {
 }
 
 const char* vbq_last_error(void) { return g_err; }
+
+vbq_status_t vbq_soft_quant(const float* w, const float* logits, const float* gumbel, float tau, int64_t N,
+                            int64_t K, float* w_soft, float* exp_bits, uint8_t* hard_widths, void* stream) {
+    g_err[0] = 0;
+    if (!w || !logits || !w_soft) return fail(VBQ_ERR_ARG, "w, logits and w_soft must be non-NULL");
+    if (!(tau > 0.f) || tau == INFINITY) return fail(VBQ_ERR_ARG, "tau must be positive and finite");
+    if (N < 1 || K < vbq::GROUP || K % vbq::GROUP != 0)
+        return fail(VBQ_ERR_SHAPE, "need N >= 1 and K a positive multiple of 64 (N=%lld K=%lld)",
+                    (long long)N, (long long)K);
+    if (N > (1LL << 40) / K) return fail(VBQ_ERR_UNSUPPORTED, "N x K above 2^40 weights");
+    if (!aligned16(w) || !aligned16(logits) || !aligned16(gumbel) || !aligned16(w_soft) || !aligned16(exp_bits) ||
+        !aligned16(hard_widths))
+        return fail(VBQ_ERR_ALIGN, "device arrays must be 16-byte aligned");
+    VBQ_CUDA(vbq::launch_soft_quant(w, logits, gumbel, tau, N, K, w_soft, exp_bits, hard_widths,
+                                    static_cast<cudaStream_t>(stream)));
+    return VBQ_OK;
+}
 
 vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint16_t* scales_fp16,
                       int64_t N, int64_t K, int src_on_device, void* stream, vbq_layout** out) {

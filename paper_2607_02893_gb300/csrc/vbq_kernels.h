@@ -25,6 +25,12 @@ cudaError_t launch_quant_validate(const float* w, const uint8_t* widths, int64_t
 cudaError_t launch_quantize(const float* w, const uint8_t* widths, int64_t N, int64_t K, uint8_t* codes,
                             uint16_t* scales, cudaStream_t s);
 
+// Training-time soft-quantised forward (vbq_soft.cu): w_soft (N x K), and per
+// group the expected width (exp_bits, may be null) and the hardened width
+// (hard, may be null). gumbel may be null (no noise).
+cudaError_t launch_soft_quant(const float* w, const float* logits, const float* gumbel, float tau, int64_t N,
+                              int64_t K, float* w_soft, float* exp_bits, uint8_t* hard, cudaStream_t s);
+
 // Products (vbq_gemv.cu). Y is B x N, overwritten (no zeroing needed).
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s);
 

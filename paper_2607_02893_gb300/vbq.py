@@ -29,6 +29,7 @@ _SZP = ctypes.POINTER(ctypes.c_size_t)
 _I64P = ctypes.POINTER(ctypes.c_int64)
 SIGNATURES = {
     "vbq_quantize": (_I, [_P, _P, _I64, _I64, _P, _P, _P]),
+    "vbq_soft_quant": (_I, [_P, _P, _P, ctypes.c_float, _I64, _I64, _P, _P, _P, _P]),
     "vbq_pack": (_I, [_P, _P, _P, _I64, _I64, _I, _P, ctypes.POINTER(_P)]),
     "vbq_packed_bytes": (_I, [_P, _SZP, _SZP, _SZP]),
     "vbq_layout_shape": (_I, [_P, _I64P, _I64P]),
@@ -143,6 +144,27 @@ def vbq_quantize(w, bitwidths, codes_out=None, scales_out=None, stream=None):
     _check(load().vbq_quantize(_ptr(w), _ptr(bitwidths), n, k, _ptr(codes_out), _ptr(scales_out),
                                _stream(stream, w)))
     return codes_out, scales_out
+
+
+def vbq_soft_quant(w, logits, tau: float, gumbel=None, w_soft=None, exp_bits=None, hard_widths=None,
+                   stream=None):
+    """Soft-quantised forward of w (N x K float32, device) under per-group
+    logits (N x K/64 x 4 float32) and optional Gumbel noise of the same shape;
+    returns (w_soft, exp_bits, hard_widths), allocating those not given (pass
+    exp_bits=False / hard_widths=False to skip one)."""
+    import torch
+    n, k = int(w.shape[0]), int(w.shape[1])
+    if w_soft is None:
+        w_soft = torch.empty((n, k), dtype=torch.float32, device=w.device)
+    if exp_bits is None:
+        exp_bits = torch.empty((n, k // 64), dtype=torch.float32, device=w.device)
+    if hard_widths is None:
+        hard_widths = torch.empty((n, k // 64), dtype=torch.uint8, device=w.device)
+    eb = None if exp_bits is False else exp_bits
+    hw = None if hard_widths is False else hard_widths
+    _check(load().vbq_soft_quant(_ptr(w), _ptr(logits), _ptr(gumbel), float(tau), n, k, _ptr(w_soft),
+                                 _ptr(eb), _ptr(hw), _stream(stream, w)))
+    return w_soft, eb, hw
 
 
 def vbq_pack(codes, bitwidths, scales_fp16, N: Optional[int] = None, K: Optional[int] = None,

@@ -81,6 +81,18 @@ def draw_gate_up(k: int, rng: np.random.Generator) -> np.ndarray:
     return gu.astype(np.float32).reshape(2 * k)
 
 
+def draw_soft_inputs(n: int, k: int, rng: np.random.Generator):
+    """Inputs of the training-time soft forward: weights as draw_dense_weights
+    draws them, per-group logits over the 4 candidates N(0, 2), and standard
+    Gumbel noise of the same shape (the draws the selection makes, passed in
+    as data). Returns (w N x K, logits N x K/64 x 4, gumbel N x K/64 x 4),
+    all float32."""
+    w = draw_dense_weights(n, k, rng)
+    logits = rng.normal(0.0, 2.0, size=(n, k // 64, 4)).astype(np.float32)
+    gumbel = rng.gumbel(size=(n, k // 64, 4)).astype(np.float32)
+    return w, logits, gumbel
+
+
 def code_key(seed_path: Sequence[int]) -> int:
     return int(np.random.SeedSequence([0, *seed_path, 1]).generate_state(1, dtype=np.uint32)[0])
 

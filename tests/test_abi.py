@@ -89,6 +89,20 @@ def test_calls_reject_null_layout(lib):
     assert lib.vbq_chain_free(None) == 0
 
 
+def test_soft_quant_rejects_bad_arguments_on_host(lib):
+    buf = ctypes.create_string_buffer(256)
+    p = (ctypes.addressof(buf) + 15) // 16 * 16
+    assert lib.vbq_soft_quant(None, p, None, 1.0, 1, 64, p, None, None, None) == -1      # w NULL
+    assert lib.vbq_soft_quant(p, p, None, 1.0, 1, 64, None, None, None, None) == -1      # w_soft NULL
+    for tau in (0.0, -2.0, float("inf"), float("nan")):
+        assert lib.vbq_soft_quant(p, p, None, tau, 1, 64, p, None, None, None) == -1
+    assert b"tau" in lib.vbq_last_error()
+    assert lib.vbq_soft_quant(p, p, None, 1.0, 1, 96, p, None, None, None) == -2         # K % 64
+    assert lib.vbq_soft_quant(p, p, None, 1.0, 0, 64, p, None, None, None) == -2         # N < 1
+    assert lib.vbq_soft_quant(p, p, p + 4, 1.0, 1, 64, p, None, None, None) == -5        # misaligned noise
+    assert lib.vbq_soft_quant(p, p, None, 1.0, 1, 64, p, None, p + 1, None) == -5        # misaligned widths
+
+
 def test_chain_rejects_bad_arguments_on_host(lib):
     P = ctypes.c_void_p
     arr = (P * 2)()
