@@ -108,7 +108,9 @@ vbq_status_t vbq_quantize(const float* w, const uint8_t* bitwidths, int64_t N, i
  *   w            device, N x K float32, finite (not checked).
  *   logits       device, N x (K/64) x 4 float32, finite.
  *   gumbel       device, N x (K/64) x 4 float32 noise e, or NULL for none.
- *   tau          the temperature, > 0 and finite (VBQ_ERR_ARG otherwise).
+ *   tau          the temperature, > 0 and finite (VBQ_ERR_ARG otherwise); the
+ *                quotients (l + e) / tau must stay finite in float32 (the paper
+ *                anneals tau from 5.0 to 0.5), or pi is undefined.
  *   N, K         K % 64 == 0 (VBQ_ERR_SHAPE), N * K <= 2^40.
  *   w_soft       device, N x K float32; overwritten.
  *   exp_bits     device, N x (K/64) float32, or NULL.
