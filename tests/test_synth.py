@@ -146,3 +146,28 @@ def test_scales_fp16_positive():
     rng = gen.rng_for((0, 0, 0))
     s = gen.draw_scales(100, 10, rng)
     assert s.dtype == np.float16 and (s > 0).all()
+
+
+def test_gate_up_vector():
+    # the down projection's synthetic input: 2k float32, pairs (gate, up), one
+    # feature in eight zero-padded (both exactly 0), the rest N(0, 1.5)
+    a = gen.draw_gate_up(8192, gen.rng_for((89, 8192, 0)))
+    b = gen.draw_gate_up(8192, gen.rng_for((89, 8192, 0)))
+    assert a.dtype == np.float32 and a.shape == (16384,) and np.array_equal(a, b)
+    pairs = a.reshape(-1, 2)
+    padded = (pairs == 0).all(axis=1)
+    assert abs(padded.mean() - 0.125) < 0.02
+    live = pairs[~padded]
+    assert abs(live.std() - 1.5) < 0.05 and abs(live.mean()) < 0.05
+
+
+def test_soft_inputs():
+    # weights, logits N(0, 2) and standard Gumbel noise (mean = the
+    # Euler-Mascheroni constant, variance pi^2 / 6), all float32, seeded
+    w, lg, gb = gen.draw_soft_inputs(64, 4096, gen.rng_for((70, 64, 4096)))
+    w2, lg2, gb2 = gen.draw_soft_inputs(64, 4096, gen.rng_for((70, 64, 4096)))
+    assert np.array_equal(w, w2) and np.array_equal(lg, lg2) and np.array_equal(gb, gb2)
+    assert w.shape == (64, 4096) and lg.shape == gb.shape == (64, 64, 4)
+    assert w.dtype == lg.dtype == gb.dtype == np.float32
+    assert abs(lg.std() - 2.0) < 0.05
+    assert abs(gb.mean() - 0.5772156649) < 0.02 and abs(gb.var() - np.pi ** 2 / 6) < 0.06
