@@ -342,6 +342,76 @@ def pin_soft_quant(O):
     _check(agree > 400, f"only {agree} comparisons")
 
 
+def pin_soft_bound(O):
+    """The acceptance bound of a float32 soft forward (soft_quant_within_bound,
+    §3.2 / Alg. 1's weight step) against values derived by hand.
+
+    Hand-worked group: all 64 weights equal c = 2^-4, equal logits, no noise,
+    tau = 1. Then z = (l + e) / tau = 0, so pi_k = 1/4 exactly and the bound's
+    eps = 2^-20 (1 + max|z|) + 2^-20 = 2^-19. Every reconstruction is c up to
+    float32 rounding of its scale (1 bit: mean|w| = c; 2 bits: s = c / 1, q = 1;
+    4 and 8 bits: q = 7 and 127 against s = c / 7, c / 127), so
+    sum_k pi_k |w_hat_k| = c within 2^-22 relatively and the expected width is
+    (1 + 2 + 4 + 8) / 4 = 3.75. A weight error of eps c / 2 is inside the bound
+    and one of 4 eps c outside it; the same for the expected width with 3.75
+    in place of c. The forward's own output is admitted, and a weight moved by
+    a quarter of its 4-bit step under a dominant 4-bit logit is rejected."""
+    c = 2.0 ** -4
+    w = np.full((1, 64), c, np.float32)
+    lg = np.zeros((1, 1, 4), np.float32)
+    eps = 2.0 ** -19                                    # by hand, from z = 0
+    ws, eb, _, pi = O.soft_quant_forward(w, lg, None, 1.0)
+    _check(np.array_equal(pi[0, 0], np.full(4, 0.25)), f"pi {pi[0, 0]}")
+    _check(abs(eb[0, 0] - 3.75) < 1e-15, f"expected width {eb[0, 0]}")
+    _check(np.allclose(ws, c, rtol=2.0 ** -22, atol=0), "reconstructions all c")
+    ok_w, ok_b = O.soft_quant_within_bound(ws, eb, w, lg, None, 1.0)
+    _check(ok_w.all() and ok_b.all(), "bound admits the forward's own output")
+    for j in (0, 17, 63):
+        for sgn in (1.0, -1.0):
+            near = ws.copy()
+            near[0, j] += sgn * 0.5 * eps * c
+            far = ws.copy()
+            far[0, j] += sgn * 4.0 * eps * c
+            okn, _ = O.soft_quant_within_bound(near, eb, w, lg, None, 1.0)
+            okf, _ = O.soft_quant_within_bound(far, eb, w, lg, None, 1.0)
+            _check(okn.all(), f"eps c / 2 at weight {j} admitted")
+            _check(not okf[0, j] and okf.sum() == 63, f"4 eps c at weight {j} rejected, the rest admitted")
+    _, okb = O.soft_quant_within_bound(ws, eb + 0.5 * eps * 3.75, w, lg, None, 1.0)
+    _check(okb.all(), "expected width off by eps 3.75 / 2 admitted")
+    _, okb = O.soft_quant_within_bound(ws, eb - 4.0 * eps * 3.75, w, lg, None, 1.0)
+    _check(not okb.any(), "expected width off by 4 eps 3.75 rejected")
+    # a quarter step: dominant 4-bit logit, random group; the 4-bit step is s =
+    # max|w| / 7 and pi_4 is 1 to within e^-40
+    rng = np.random.default_rng(37)
+    wr = rng.normal(0, 0.02, (1, 128)).astype(np.float32)
+    lr = np.zeros((1, 2, 4), np.float32)
+    lr[0, :, 2] = 40.0
+    ws2, eb2, _, _ = O.soft_quant_forward(wr, lr, None, 1.0)
+    ok_w, ok_b = O.soft_quant_within_bound(ws2, eb2, wr, lr, None, 1.0)
+    _check(ok_w.all() and ok_b.all(), "bound admits the forward's own output (dominant 4 bits)")
+    s4 = float(np.max(np.abs(wr[0, 64:]))) / 7.0
+    moved = ws2.copy()
+    moved[0, 64 + 9] += 0.25 * s4
+    okm, _ = O.soft_quant_within_bound(moved, eb2, wr, lr, None, 1.0)
+    _check(not okm[0, 64 + 9] and okm.sum() == 127, "a quarter 4-bit step rejected")
+    # the noise enters z: e = 1000 on the 4-bit candidate and l = 0 give z =
+    # (0, 0, 1000, 0), pi = (0, 0, 1, 0) and eps = 2^-20 (1 + 1000) + 2^-20 =
+    # 1002 2^-20 (by hand); an error of eps |w_hat_4| / 2 is admitted
+    ge = np.zeros((1, 2, 4), np.float32)
+    ge[0, :, 2] = 1000.0
+    ws3, eb3, _, _ = O.soft_quant_forward(wr, np.zeros((1, 2, 4), np.float32), ge, 1.0)
+    rec4 = O.reconstruct_fp32(wr[0, :64], 4)
+    j = int(np.argmax(np.abs(rec4)))
+    half = ws3.copy()
+    half[0, j] += 0.5 * 1002 * 2.0 ** -20 * abs(rec4[j])
+    okh, _ = O.soft_quant_within_bound(half, eb3, wr, np.zeros((1, 2, 4), np.float32), ge, 1.0)
+    _check(okh.all(), "eps from z with the noise: eps |w_hat| / 2 admitted")
+    over = ws3.copy()
+    over[0, j] += 4.0 * 1002 * 2.0 ** -20 * abs(rec4[j])
+    oko, _ = O.soft_quant_within_bound(over, eb3, wr, np.zeros((1, 2, 4), np.float32), ge, 1.0)
+    _check(not oko[0, j], "eps from z with the noise: 4 eps |w_hat| rejected")
+
+
 ALL_PINS = [pin_eq1_golden, pin_level_grid, pin_grid_roundtrip, pin_quantizer_invariants,
             pin_one_bit_mean_order, pin_group_size_one, pin_integer_gemv, pin_exact_rational, pin_enumerated_codes,
-            pin_swiglu, pin_soft_quant, pin_payload_accounting]
+            pin_swiglu, pin_soft_quant, pin_soft_bound, pin_payload_accounting]

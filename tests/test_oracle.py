@@ -71,6 +71,10 @@ MUTATIONS = {
     "soft_qmax_too_large": ("    qmax = np.float32((1 << (b - 1)) - 1)", "    qmax = np.float32(1 << (b - 1))"),
     "soft_hard_last_max": ("[np.argmax(logits, axis=-1)]",
                            "[3 - np.argmax(logits[..., ::-1], axis=-1)]"),
+    "soft_bound_eps_loosened": ("    eps = 2.0 ** -20 * (1.0 + np.abs(z).max(axis=-1)) + 2.0 ** -20",
+                                "    eps = 100.0 * (2.0 ** -20 * (1.0 + np.abs(z).max(axis=-1)) + 2.0 ** -20)"),
+    "soft_bound_no_noise": ("        z = z + np.asarray(gumbel, dtype=np.float64)\n    z = z / tau\n    eps =",
+                            "        z = z\n    z = z / tau\n    eps ="),
     "soft_expected_bits_unweighted": ("    exp_bits = (pi * cand).sum(axis=-1)", "    exp_bits = pi.sum(axis=-1) * cand.mean()"),
 }
 
