@@ -318,9 +318,10 @@ vbq_status_t vbq_chain_free(vbq_chain* chain);
  * (The paper has no counterpart; this is an operational variant.)
  *
  * Some callers cannot call cudaMalloc where they run products: a serving loop
- * with a fixed memory budget, code inside a stream capture that forbids
- * allocation calls, or a host framework whose allocator must own every
- * device byte. This entry point allocates nothing, on the device or the host.
+ * that must stay inside a memory budget fixed at start-up, or a host framework
+ * whose allocator must own every device byte (an allocation outside it would
+ * break its accounting). This entry point allocates nothing, on the device or
+ * the host.
  * It runs the same batch-1 kernel as vbq_gemv, but keeps the kernel's split-K
  * control words (a call counter and one flag per row block) in a fixed array
  * inside this library instead of in the layout.
