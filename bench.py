@@ -115,22 +115,47 @@ def kernel_source_hash() -> str:
     return h.hexdigest()
 
 
-def profiled_traffic(workload: str, batch: int):
-    """DRAM bytes per gemv1 launch from the committed ncu launch-list summary of
-    this workload, or None when there is none or the kernel changed since."""
-    path = os.path.join(ROOT, "profiles", f"gemv1_{workload.replace(':', '_')}_b{batch}_launches.txt")
+TRAFFIC_PROFILE = os.path.join(ROOT, "profiles", "gemv1_dram_traffic_by_shape.md")
+
+
+def shape_traffic_ratios():
+    """DRAM bytes over algorithmic bytes of one batch-1 GEMV launch per matrix
+    shape, from the committed per-shape ncu captures (one launch each, a small
+    replicated workload per shape): {(n, k): ratio}, or None when the file is
+    absent or the GEMV kernel's sources changed since the captures."""
     try:
-        kv = {}
-        with open(path) as f:
+        kv, ratios = {}, {}
+        with open(TRAFFIC_PROFILE) as f:
             for line in f:
-                if ":" in line and not line.startswith((" ", "#", "|", "`")):
-                    k, v = line.split(":", 1)
-                    kv[k.strip()] = v.strip()
-        if kv.get("source_sha256") != kernel_source_hash():
+                line = line.strip()
+                if line.startswith("shape:"):
+                    n, k, dram, alg = line.split(":", 1)[1].split()[:4]
+                    ratios[(int(n), int(k))] = float(dram) / float(alg)
+                elif line.startswith("source_sha256:"):
+                    kv["source_sha256"] = line.split(":", 1)[1].strip()
+        if kv.get("source_sha256") != kernel_source_hash() or not ratios:
             return None
-        return float(kv["dram_bytes_per_launch"])
+        return ratios
     except Exception:
         return None
+
+
+def profiled_traffic(mats, nbytes, batch: int):
+    """DRAM bytes per launch of the step, modelled from the per-shape captures:
+    each launch's algorithmic bytes times its shape's measured DRAM/algorithmic
+    ratio (the nearest captured shape by weight count where the exact shape
+    was not captured), averaged over the step's launches. None at batch > 1,
+    without captures, or after a kernel change."""
+    ratios = shape_traffic_ratios()
+    if batch != 1 or ratios is None:
+        return None
+    total = 0.0
+    for spec, nb in zip(mats, nbytes):
+        key = (spec.n, spec.k)
+        if key not in ratios:
+            key = min(ratios, key=lambda nk: abs(np.log(nk[0] * nk[1] / (spec.n * spec.k))))
+        total += ratios[key] * nb
+    return total / len(nbytes)
 
 
 def algorithmic_bytes(widths: np.ndarray, n: int, k: int, batch: int) -> int:
@@ -221,6 +246,77 @@ def oracle_block(spec, batch: int, rows: int, seed: int):
     t0 = time.perf_counter()
     oracle.gemv(codes, w, s, x)
     return time.perf_counter() - t0, algorithmic_bytes(w, r, spec.k, batch)
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def _oracle_worker(q, barrier, workload, batch, blocks, rounds, rank):
+    """One host process of the parallel oracle legs (spawned: no CUDA state is
+    inherited). Prepares its row blocks first (untimed: input generation is
+    not the oracle), then per round waits for every process at the barrier and
+    runs the oracle on its next block, reporting (round, start, end, bytes)."""
+    os.environ["OMP_NUM_THREADS"] = "1"
+    import oracle
+    import synth
+    from synth import gen
+    try:
+        import torch
+        torch.set_num_threads(1)
+    except Exception:
+        pass
+    work = synth.workload(workload, batch)
+    prepared = []
+    for mi, rows, seed in blocks:
+        spec = work.mats[mi]
+        rng = np.random.default_rng(seed)
+        inp = gen.matrix_inputs(spec, batch)
+        r = max(1, min(rows, spec.n))
+        row0 = int(rng.integers(0, spec.n - r + 1))
+        codes = gen.codes_torch(inp["widths"], inp["key"], spec.k, row0=row0, nrows=r, device="cpu").numpy()
+        w, sc = inp["widths"][row0:row0 + r], inp["scales"][row0:row0 + r]
+        prepared.append((codes, w, sc, gen.bf16_bits_to_f32(inp["x_bits"]),
+                         algorithmic_bytes(w, r, spec.k, batch), r))
+    for rd in range(rounds):
+        codes, w, sc, x, nb, r = prepared[rd % len(prepared)]
+        barrier.wait()
+        t0 = time.perf_counter()
+        oracle.gemv(codes, w, sc, x)
+        q.put((rd, rank, t0, time.perf_counter(), nb, r))
+
+
+def oracle_parallel(work, workload: str, batch: int, cores: int, rounds: int, block_s: float, seed: int):
+    """The oracle, unchanged, on `cores` host processes at once: in each round
+    every process runs one random row block (about block_s seconds of work),
+    the blocks cycling through the workload's matrices. Returns per round
+    (wall seconds from the first start to the last end, algorithmic bytes,
+    rows)."""
+    import multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    m = len(work.mats)
+    q, barrier = ctx.Queue(), ctx.Barrier(cores)
+    procs = []
+    for p in range(cores):
+        blocks = []
+        for rd in range(min(rounds, 8)):
+            mi = (rd * cores + p) % m
+            rows = max(1, int(block_s * ORACLE_WEIGHTS_PER_S / work.mats[mi].k))
+            blocks.append((mi, rows, seed + rd * cores + p))
+        pr = ctx.Process(target=_oracle_worker, args=(q, barrier, workload, batch, blocks, rounds, p))
+        pr.start()
+        procs.append(pr)
+    got = [q.get(timeout=600) for _ in range(rounds * cores)]
+    for pr in procs:
+        pr.join(timeout=60)
+    out = []
+    for rd in range(rounds):
+        rs = [g for g in got if g[0] == rd]
+        out.append((max(g[3] for g in rs) - min(g[2] for g in rs), sum(g[4] for g in rs), sum(g[5] for g in rs)))
+    return out
 
 
 def oracle_leg(work, batch: int, budget_s: float, seed: int = 0):
@@ -662,6 +758,7 @@ def run_ours(args, rank, world, local_rank):
     kernel_ms_per_step = ms
     kernel_gbs = step_bytes / (kernel_ms_per_step * 1e-3) / 1e9
     launches = len(layouts)
+    traffic = profiled_traffic(work.mats * copies, nbytes, B)
     result = {
         "metric": METRIC,
         "value": round(gbs, 1),
@@ -696,9 +793,11 @@ def run_ours(args, rank, world, local_rank):
             "peak_kind": peak_kind,
             "unit": "GB/s",
             "frac": round(kernel_gbs / peak, 4),
-            "traffic": profiled_traffic(args.workload, B),
-            "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum per launch, averaged over "
-                              "one step's launches (profiles/); null when absent or the kernel changed since",
+            "traffic": None if traffic is None else round(traffic),
+            "traffic_source": ("ncu dram__bytes_read.sum + dram__bytes_write.sum of one launch per matrix shape "
+                               "(profiles/gemv1_dram_traffic_by_shape.md), as a ratio to that launch's "
+                               "algorithmic bytes, applied to every launch of the step and averaged; null "
+                               "when absent or the kernel changed since"),
             "launches_timed": launches * args.steps,
             "avg_launch_us": round(kernel_ms_per_step * 1e3 / launches, 3),
             "duration_source": "CUDA events around the timed region on the launching stream, "
@@ -773,25 +872,29 @@ def run_sweep(args):
 
 
 def run_reference(args):
-    """The CPU oracle as the reference arm: step s runs the oracle on a random
-    row block of matrix s mod M, sized so that the whole run takes a few minutes."""
+    """The CPU oracle as the reference arm, on every host core: each step is
+    one round of row blocks, one per host process (spawned processes started
+    together at a barrier), the blocks cycling through the workload's
+    matrices. ms_per_step is a round's measured wall time (so steps x
+    ms_per_step is the time the run spent in the oracle) and value is the
+    algorithmic GB/s over the timed rounds. The time a whole token would take
+    at that rate is reported separately, as an extrapolation."""
     import synth
     work = synth.workload(args.workload, args.batch)
-    budget_per_step = min(2.0, 150.0 / max(1, args.steps + args.warmup))
-    t, nbytes, rows_seen = 0.0, 0, 0
-    for s in range(args.warmup + args.steps):
-        spec = work.mats[s % len(work.mats)]
-        rows = max(1, int(budget_per_step * ORACLE_WEIGHTS_PER_S / spec.k))
-        dt, nb = oracle_block(spec, args.batch, rows, seed=1000 + s)
-        if s >= args.warmup:
-            t += dt
-            nbytes += nb
-            rows_seen += min(rows, spec.n)
+    cores = host_cores()
+    block_s = min(1.0, 100.0 / max(1, args.steps + args.warmup))
+    rounds = oracle_parallel(work, args.workload, args.batch, cores, rounds=args.warmup + args.steps,
+                             block_s=block_s, seed=1000)[args.warmup:]
+    t = sum(r[0] for r in rounds)
+    nbytes = sum(r[1] for r in rounds)
+    rows_seen = sum(r[2] for r in rounds)
     gbs = nbytes / t / 1e9
-    token_bytes = sum(algorithmic_bytes_est(m, args.batch) for m in work.mats)
-    ms_per_step = token_bytes / (gbs * 1e9) * 1e3          # one full token at that rate
-    sample = (f"per step one random contiguous row block (about {budget_per_step:.2f} s of work) of one "
-              f"matrix, cycling through the {len(work.mats)} matrices; {rows_seen} rows in all")
+    ms_per_step = t / args.steps * 1e3
+    token_bytes = sum(algorithmic_bytes_est(mm, args.batch) for mm in work.mats)
+    ms_per_token = token_bytes / (gbs * 1e9) * 1e3
+    sample = (f"per step one random contiguous row block per host process ({cores} processes, about "
+              f"{block_s:.2f} s of work each), cycling through the {len(work.mats)} matrices; {rows_seen} rows "
+              f"timed; inputs prepared before the timed rounds")
     return {
         "impl": "reference",
         "metric": METRIC,
@@ -807,8 +910,10 @@ def run_reference(args):
         "dtype": "f64",
         "data": "synthetic",
         "config": {"workload": args.workload, "batch": args.batch,
-                   "tokens_per_s": round(args.batch / (ms_per_step * 1e-3), 6)},
-        "cpu_baseline": {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                   "step": "a bounded sample of the workload (see cpu_baseline.sample), not a whole token",
+                   "ms_per_token_extrapolated": round(ms_per_token, 3),
+                   "tokens_per_s_extrapolated": round(args.batch / (ms_per_token * 1e-3), 6)},
+        "cpu_baseline": {"value": round(gbs, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": round(gbs, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
@@ -830,6 +935,17 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        # no launcher: start one replica per GPU the same way the driver does
+        import socket
+        with socket.socket() as sk:
+            sk.bind(("127.0.0.1", 0))
+            port = sk.getsockname()[1]
+        cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={args.gpus}",
+               "--master-addr", "127.0.0.1", "--master-port", str(port), os.path.abspath(__file__), *sys.argv[1:]]
+        sys.exit(subprocess.call(cmd))
+    if world != args.gpus:
+        sys.exit(f"bench.py: --gpus {args.gpus} but WORLD_SIZE is {world}")
 
     if args.sweep:
         if rank == 0:
@@ -848,11 +964,20 @@ def main():
         dist.init_process_group("nccl")
     result, work = run_ours(args, rank, world, local_rank)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        t, nb, frac = oracle_leg(work, args.batch, budget_s=12.0)
+        t, nb, frac = oracle_leg(work, args.batch, budget_s=8.0)
+        cores = host_cores()
+        rounds = oracle_parallel(work, args.workload, args.batch, cores, rounds=9, block_s=1.0, seed=5000)[1:]
+        wall = sum(r[0] for r in rounds)
+        nbp = sum(r[1] for r in rounds)
         result["cpu_baseline"] = {
-            "value": round(nb / t / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sample": f"random contiguous row blocks, at least one of each of the {len(work.mats)} matrices "
-                      f"({frac * 100:.3f}% of all rows), {t:.1f} s of numpy fp64 on one host core",
+            "value": round(nbp / wall / 1e9, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
+            "sample": f"8 rounds (after one untimed) of one random contiguous row block per host process (about 1 s of work each; "
+                      f"{sum(r[2] for r in rounds)} rows) cycling through the {len(work.mats)} matrices, "
+                      f"{wall:.1f} s of wall time on {cores} processes at once (numpy fp64; inputs prepared "
+                      f"before the timed rounds)",
+            "single_core": {"value": round(nb / t / 1e9, 4), "unit": "GB/s", "cores": 1,
+                            "sample": f"random contiguous row blocks, at least one of each matrix "
+                                      f"({frac * 100:.3f}% of all rows), {t:.1f} s on one host core"},
         }
     if world > 1:
         import torch.distributed as dist

@@ -175,15 +175,15 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
         if (!last && 2 * uc < sms) continue;          // fewer units than half the SMs: narrower slabs
         if (uc > (1LL << 31) - 2) return fail(VBQ_ERR_UNSUPPORTED, "too many units");
         void* dc = nullptr;
-        VBQ_CUDA(tmp.alloc(&dc, (size_t)uc * 4 * sizeof(uint32_t)));
+        VBQ_CUDA(tmp.alloc(&dc, (size_t)uc * 5 * sizeof(uint32_t)));
         VBQ_CUDA(vbq::launch_count(d_widths, N, (int)G, cand, (int)nrb, (int)uc, static_cast<uint32_t*>(dc), s));
-        std::vector<uint32_t> cnt((size_t)uc * 4);
+        std::vector<uint32_t> cnt((size_t)uc * 5);
         VBQ_CUDA(cudaMemcpyAsync(cnt.data(), dc, cnt.size() * sizeof(uint32_t), cudaMemcpyDeviceToHost, s));
         VBQ_CUDA(cudaStreamSynchronize(s));
         std::vector<vbq::UnitHeader> hd((size_t)uc);
         uint32_t m16 = 0;
         for (int64_t u = 0; u < uc; ++u) {
-            hd[u] = vbq::make_header(&cnt[u * 4], cand);
+            hd[u] = vbq::make_header(&cnt[u * 5], cand, (int)cnt[u * 5 + 4]);
             m16 = std::max<uint32_t>(m16, hd[u].size16);
         }
         if (m16 * 16u > vbq::MAX_BLOB_BYTES && !last) continue;
@@ -200,7 +200,7 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     for (int64_t u = 0; u < units; ++u) {
         blob_off[u] = (uint32_t)off16;
         off16 += headers[u].size16;
-        for (int w = 0; w < 4; ++w) real_items[w] += counts[u * 4 + w];
+        for (int w = 0; w < 4; ++w) real_items[w] += counts[u * 5 + w];
         if (off16 > 0xffffffffull) return fail(VBQ_ERR_UNSUPPORTED, "layout too large");
     }
     blob_off[units] = (uint32_t)off16;

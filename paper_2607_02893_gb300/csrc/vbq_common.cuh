@@ -16,6 +16,8 @@
 //         row bytes of each width (row within the row block), padded to 16
 //         column ends: uint16 cend[w][c] = index (within width w) of the
 //         first item after column c
+//         task table: one 16-byte TaskDesc per warp task of the batch-1
+//         product (see TaskDesc), 8-bit tasks first, then 4, 2 and 1 bit
 //     Blob u starts at byte 16 * blob_off[u] of the layout's blob area.
 //   * When a row has several slabs, the batch-1 product adds every slab's row
 //     partials into y with atomics, and y needs no zeroing by the caller: the
@@ -57,9 +59,89 @@ struct UnitHeader {
     uint16_t row16[4];    // row-byte offsets
     uint16_t cc16;        // column-end offset (uint16 [4][C])
     uint16_t size16;      // blob size in 16-byte units
-    uint16_t pad[6];
+    uint16_t ntask;       // warp tasks of the batch-1 product
+    uint16_t task16;      // task-table offset (TaskDesc [ntask])
+    uint16_t pad[4];
 };
 static_assert(sizeof(UnitHeader) == 48, "header is 48 bytes");
+
+// One warp task of the batch-1 product, built at pack time so that a warp
+// needs nothing else to run it: up to 32 consecutive items of one width (64
+// for 1 bit, lane l holding the adjacent items 2l and 2l + 1), their byte
+// offsets within the blob, and the columns they lie in, given as masks over
+// the lanes. A width can have no items in some columns, so several column
+// ends can fall on one item.
+//   32-item tasks: lane l's item lies in column
+//     c0 + popc(M1 & lanes <= l) + 2 popc(M2 & lanes <= l),
+//     M1 and M2 holding the binary digits of the number of column ends at
+//     each item (at most 3; the packer ends a task early before an item with
+//     more).
+//   1-bit tasks: bit l of M1 marks a column end at item 2l and bit l of M2 one
+//     at item 2l + 1 (at most one each; a task ends early before an item with
+//     more). Tasks start on an even item so that a lane's pair is one 16-byte
+//     load; a task that has to begin on an odd item starts one item early
+//     with that first item switched off (skip bit), c0 being the column of
+//     its second item.
+//   x: scale byte offset of the first item (bits 0-15), c0 (16-19), count - 1
+//      (20-25), width index (26-27), skip (28)
+//   y: M1   z: M2
+//   w: payload byte offset of the first item (bits 0-15), row-byte offset (16-31)
+struct __align__(16) TaskDesc {
+    uint32_t x, y, z, w;
+};
+static_assert(sizeof(TaskDesc) == 16, "16-byte task descriptors");
+constexpr int TASK_SPAN1 = 64;   // items per 1-bit task
+constexpr int TASK_SPAN = 32;    // items per 2-, 4- and 8-bit task
+constexpr int MAX_UNIT_TASKS = 2 * MAX_UNIT_ITEMS / TASK_SPAN;   // a bound the task cuts never exceed
+
+// The tasks of one unit from its column ends ce[w][c] (w = width index, c <
+// cols): widths 8, 4, 2, 1 bit in that order, each cut into spans of at most
+// TASK_SPAN (TASK_SPAN1) items, a span ending early before an item on which
+// more column ends fall than its masks can count. Writes the descriptors when
+// out is not null (h gives the blob offsets) and returns their number.
+__host__ __device__ inline int unit_tasks(const uint16_t (*ce)[MAX_C], int cols, const UnitHeader* h,
+                                          TaskDesc* out) {
+    int nt = 0;
+    for (int w = 3; w >= 0; --w) {
+        const int span = w == 0 ? TASK_SPAN1 : TASK_SPAN, maxm = w == 0 ? 1 : 3;
+        const int n = cols > 0 ? ce[w][cols - 1] : 0;
+        int st = 0;                     // first item of the next task
+        while (st < n) {
+            const int i0 = w == 0 ? (st & ~1) : st, skip = st - i0;
+            int end = i0 + span < n ? i0 + span : n;
+            uint32_t m1 = 0, m2 = 0;
+            int c0 = 0;                 // ends are nondecreasing: c0 = the first column ending after st
+            while (c0 < cols && ce[w][c0] <= st) ++c0;
+            for (int c = c0; c < cols && ce[w][c] < end;) {
+                const int e = ce[w][c], p = e - i0;
+                int mult = 0;
+                while (c < cols && ce[w][c] == e) { ++mult; ++c; }
+                if (mult > maxm) { end = e; break; }
+                if (w == 0) {
+                    if (p & 1) m2 |= 1u << (p >> 1);
+                    else m1 |= 1u << (p >> 1);
+                } else {
+                    if (mult & 1) m1 |= 1u << p;
+                    if (mult & 2) m2 |= 1u << p;
+                }
+            }
+            if (out) {
+                const uint32_t b = 1u << w;
+                TaskDesc d;
+                d.x = (uint32_t)(h->sc16[w] * 16 + 2 * i0) | ((uint32_t)c0 << 16) |
+                      ((uint32_t)(end - i0 - 1) << 20) | ((uint32_t)w << 26) | ((uint32_t)skip << 28);
+                d.y = m1;
+                d.z = m2;
+                d.w = (uint32_t)(h->pay16[w] * 16 + 8 * b * i0) | ((uint32_t)(h->row16[w] * 16 + i0) << 16);
+                out[nt] = d;
+            }
+            ++nt;
+            st = end;
+        }
+    }
+    return nt;
+}
+
 
 struct LayoutView {
     const uint8_t* blobs;       // blob area
@@ -103,7 +185,7 @@ __host__ __device__ inline int unit_cols(const LayoutView& L, int s) {
 // Sizes of the blob parts, given the item counts of a unit.
 __host__ __device__ inline uint32_t pad16(uint32_t bytes) { return (bytes + 15u) / 16u; }
 
-__host__ __device__ inline UnitHeader make_header(const uint32_t n[4], int C) {
+__host__ __device__ inline UnitHeader make_header(const uint32_t n[4], int C, int ntask) {
     UnitHeader h{};
     uint32_t off = sizeof(UnitHeader) / 16;
     for (int w = 0; w < 4; ++w) { h.n[w] = (uint16_t)n[w]; h.pay16[w] = (uint16_t)off; off += pad16(n[w] * 8u * (1u << w)); }
@@ -111,6 +193,9 @@ __host__ __device__ inline UnitHeader make_header(const uint32_t n[4], int C) {
     for (int w = 0; w < 4; ++w) { h.row16[w] = (uint16_t)off; off += pad16(n[w]); }
     h.cc16 = (uint16_t)off;
     off += pad16(8u * (uint32_t)C);
+    h.ntask = (uint16_t)ntask;
+    h.task16 = (uint16_t)off;
+    off += (uint32_t)ntask;
     h.size16 = (uint16_t)off;
     return h;
 }

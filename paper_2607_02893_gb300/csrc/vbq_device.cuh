@@ -1,7 +1,7 @@
 // vbq_device.cuh — device helpers shared by the product kernels of this
 // library: shared-memory access by 32-bit shared address, reductions, the
 // bounded mbarrier waits and TMA bulk copies of unit blobs, the split-K flag
-// wait, and the column lookup of a unit's items.
+// wait.
 #pragma once
 
 #include <cstdint>
@@ -240,20 +240,6 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
 __device__ __forceinline__ void issue_unit(const LayoutView& L, int u, uint32_t dst, uint32_t bar) {
     const uint32_t o0 = L.blob_off[u], o1 = L.blob_off[u + 1];
     bulk_load(dst, L.blobs + (int64_t)o0 * 16, (o1 - o0) * 16, bar);
-}
-
-// Columns of a unit's items without a per-item array: lane t holds cend[t]
-// of one width (0xFFFF past the unit's last column), and item i of that width
-// lies in column #{t : cend[t] <= i}. A warp finds the columns of a task's
-// first and last items by one ballot each; only a task across column ends
-// (cf < cl) walks the few ends in between.
-__device__ __forceinline__ int col_uniform(uint32_t ce, int i) {   // i the same on every lane
-    return __popc(__ballot_sync(0xffffffffu, ce <= (uint32_t)i));
-}
-__device__ __forceinline__ int col_within(uint32_t ce, int cf, int cl, int i) {   // cf, cl the same on every lane
-    int c = cf;
-    for (int t = cf; t < cl; ++t) c += __shfl_sync(0xffffffffu, ce, t) <= (uint32_t)i;
-    return c;
 }
 
 // Split-K: true once every row block this block adds a slab s > 0 into has

@@ -10,10 +10,10 @@
 //                      into the freed stage;
 //   warps 1.. (NCW)    consumers, in 1 or 2 teams (2 from 4 units per block
 //                      on): unit j goes to team j % teams, whose warps split
-//                      its items into warp tasks and store each group's
-//                      scaled dot product in the stage's (row, column) slot;
-//                      an item's column comes from the blob's column ends (a
-//                      ballot per task, see col_uniform).
+//                      the unit's warp tasks (a table the packer stores in
+//                      the blob: each task's items, their offsets and
+//                      columns) and store each group's scaled dot product in
+//                      the stage's (row, column) slot.
 // The roles hand stages to one another through two mbarriers per stage
 // (full: blob landed; empty: the unit's team is done), so no block-wide
 // barrier sits in the steady state and up to NSTAGE units are in flight per
@@ -452,194 +452,187 @@ __device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t
     consumer_sync();
 }
 
-// Shared-memory addresses of one unit's blob and of the slab's tables, for
-// the per-width task loops.
-struct UnitView {
-    uint32_t pay, sc, row;      // this width's payload, FP16 scales, row bytes
-    uint32_t ce;                // this lane's column end for this width (0xFFFF past the slab's columns)
-    int n;                      // items of this width
+// One warp task (a TaskDesc built at pack time: items, their blob offsets and
+// columns), for the per-width bodies below. Lanes past the task's last item
+// redo its first item (always present) and store nothing, so every body is
+// branch-free.
+struct Task {
+    uint32_t pay, sc, row;      // shared addresses of the lane's (first) item: payload, scale, row byte
+    bool on, on2;               // the lane's item (1 bit: its first and second item) is stored
+    int c, c2;                  // their columns
 };
 
-// Column of item i (tasks hold items i0 .. i0 + span - 1; lanes agree on i0).
-__device__ __forceinline__ int task_column(uint32_t ce, int i0, int span, int n, int i) {
-    const int cf = col_uniform(ce, i0), cl = col_uniform(ce, min(i0 + span - 1, n - 1));
-    if (cl == cf + 1) return cf + (i >= (int)__shfl_sync(0xffffffffu, ce, cf));   // one column end inside
-    return cf == cl ? cf : col_within(ce, cf, cl, i);
+// 32-item tasks: lane l takes item l.
+__device__ __forceinline__ Task task32(uint32_t sblob, uint4 d, int lane, int bytes_per_item) {
+    Task t;
+    const int cnt = (int)((d.x >> 20) & 63u) + 1;
+    const uint32_t le = (2u << lane) - 1u;
+    t.on = lane < cnt;
+    const int ii = t.on ? lane : 0;
+    t.c = (int)((d.x >> 16) & 15u) + __popc(d.y & le) + 2 * __popc(d.z & le);
+    t.pay = sblob + (d.w & 0xFFFFu) + ii * bytes_per_item;
+    t.sc = sblob + (d.x & 0xFFFFu) + 2 * ii;
+    t.row = sblob + (d.w >> 16) + ii;
+    t.on2 = false;
+    t.c2 = t.c;
+    return t;
 }
 
-// Tasks of one width: items are taken 32 (64 for 1-bit) at a time, task
-// k = first, first + tstep, ... of this width's nt tasks. Every lane holds
-// whole groups, so a task's bookkeeping is shared by 32 groups.
-template <int W, int NX>
-__device__ __forceinline__ void run_width(const TablesT<NX>& T, const UnitView& U, uint32_t slots, int first, int tstep,
-                                          int lane) {
-    constexpr int SPAN = W == 0 ? 64 : 32;
+// 1-bit tasks: lane l takes items 2l and 2l + 1 (one 16-byte payload load, one
+// 2-byte row load, one 4-byte scale load); the first item is off in a task
+// that starts one item early (skip bit).
+__device__ __forceinline__ Task task64(uint32_t sblob, uint4 d, int lane) {
+    Task t;
+    const int cnt = (int)((d.x >> 20) & 63u) + 1;
+    const uint32_t le = (2u << lane) - 1u, lt = (1u << lane) - 1u;
+    const int j = 2 * lane;
+    t.on = j < cnt && !(lane == 0 && (d.x >> 28));
+    t.on2 = j + 1 < cnt;
+    const int ii = j < cnt ? j : 0;
+    t.c = (int)((d.x >> 16) & 15u) + __popc(d.y & le) + __popc(d.z & lt);
+    t.c2 = t.c + (int)((d.z >> lane) & 1u);
+    t.pay = sblob + (d.w & 0xFFFFu) + ii * 8;
+    t.sc = sblob + (d.x & 0xFFFFu) + 2 * ii;
+    t.row = sblob + (d.w >> 16) + ii;
+    return t;
+}
+
+// The per-width bodies: each group's scaled dot product (per activation
+// vector) into its (row, column) slot of the stage.
+template <int NX>
+__device__ __forceinline__ void body4(const TablesT<NX>& T, const Task& t, uint32_t slots, int lane) {
     constexpr uint32_t SLOT_V = SLOT_FLOATS * 4;      // bytes between the vectors' slot arrays
-    const int nt = (U.n + SPAN - 1) / SPAN;
-    for (int k = first; k < nt; k += tstep) {
-        const int i0 = k * SPAN;
-        if constexpr (W == 2) {
-            // 4-bit: one group per lane, halves in the order (lane >> 2) & 1 first,
-            // so each quarter-warp's 16-byte loads fall in 8 distinct bank groups
-            const int i = i0 + lane;
-            const int c = task_column(U.ce, i0, SPAN, U.n, i);
-            const bool on = i < U.n;
-            const int ii = on ? i : 0;                  // lanes past the end redo item 0 and store nothing
-            const int h0 = (lane >> 2) & 1;
-            const uint4 va = lds_u32x4(U.pay + ii * 32 + h0 * 16), vb = lds_u32x4(U.pay + ii * 32 + (h0 ^ 1) * 16);
-            const uint32_t xa = smem_u32(T.x4s) + (c * 2 + h0) * XH * 4, xb = smem_u32(T.x4s) + (c * 2 + (h0 ^ 1)) * XH * 4;
-            const uint32_t sa = slot_addr(slots, lds_u8(U.row + ii), c);
-            const float scl = half_bits(lds_u16(U.sc + 2 * ii)) * 0x1p100f;
-            if constexpr (NX == 1) {
-                const float2 aa = dot4_half(va, xa), ab = dot4_half(vb, xb);
-                const float4 z = lds_f32x4(smem_u32(T.x4z) + c * 16);     // (even, odd) of half 0, then of half 1
-                const float part = ((aa.x + ab.x) - 8.f * (z.x + z.z)) + ((aa.y + ab.y) - 8.f * (z.y + z.w));
-                sts_f32_if(sa, scl * part, on);
-            } else {
-                float2 aa0, aa1, ab0, ab1;
-                dot4_half2(va, xa, aa0, aa1);
-                dot4_half2(vb, xb, ab0, ab1);
-                const float4 z0 = lds_f32x4(smem_u32(T.x4z) + c * 16), z1 = lds_f32x4(smem_u32(T.x4z) + MAX_C * 16 + c * 16);
-                const float p0 = ((aa0.x + ab0.x) - 8.f * (z0.x + z0.z)) + ((aa0.y + ab0.y) - 8.f * (z0.y + z0.w));
-                const float p1 = ((aa1.x + ab1.x) - 8.f * (z1.x + z1.z)) + ((aa1.y + ab1.y) - 8.f * (z1.y + z1.w));
-                sts_f32_if(sa, scl * p0, on);
-                sts_f32_if(sa + SLOT_V, scl * p1, on);
-            }
-        } else if constexpr (W == 3) {
-            // 8-bit: one group per lane, quarter (k + (lane >> 1)) & 3 in step k
-            // (conflict-free 16-byte loads for every quarter-warp)
-            const int i = i0 + lane;
-            const int c = task_column(U.ce, i0, SPAN, U.n, i);
-            const bool on = i < U.n;
-            const int ii = on ? i : 0;
-            const int q0 = lane >> 1;
-            const uint32_t sa = slot_addr(slots, lds_u8(U.row + ii), c);
-            const float scl = half_bits(lds_u16(U.sc + 2 * ii));
-            if constexpr (NX == 1) {
-                float part = 0.f;
-#pragma unroll
-                for (int step = 0; step < 4; ++step) {
-                    const int q = (step + q0) & 3;
-                    const uint4 v = lds_u32x4(U.pay + ii * 64 + q * 16);
-                    part += dot8_quarter(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
-                }
-                sts_f32_if(sa, scl * part, on);
-            } else {
-                float p0 = 0.f, p1 = 0.f;
-#pragma unroll
-                for (int step = 0; step < 4; ++step) {
-                    const int q = (step + q0) & 3;
-                    const uint4 v = lds_u32x4(U.pay + ii * 64 + q * 16);
-                    const float2 d = dot8_quarter2(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
-                    p0 += d.x;
-                    p1 += d.y;
-                }
-                sts_f32_if(sa, scl * p0, on);
-                sts_f32_if(sa + SLOT_V, scl * p1, on);
-            }
-        } else if constexpr (W == 1) {
-            // 2-bit: one group per lane, both planes at once
-            const int i = i0 + lane;
-            const int c = task_column(U.ce, i0, SPAN, U.n, i);
-            const bool on = i < U.n;
-            const int ii = on ? i : 0;
-            const uint4 pl = lds_u32x4(U.pay + ii * 16);
-            const uint32_t tb = smem_u32(T.lut) + c * LUT_COL_BYTES;
-            const uint32_t sa = slot_addr(slots, lds_u8(U.row + ii), c);
-            const float scl = half_bits(lds_u16(U.sc + 2 * ii));
-            if constexpr (NX == 1) {
-                float va[16], vb[16];
-                plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
-                plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
-                const float2 sp = tree16x2(va, vb);
-                sts_f32_if(sa, scl * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))), on);
-            } else {
-                float2 pv[16];
-                plane_entries2(tb, col_shift4(c), pl.x, pl.y, pv);
-                const float2 s0 = tree16_pairs(pv);                       // plane 0, both vectors
-                plane_entries2(tb, col_shift4(c), pl.z, pl.w, pv);
-                const float2 s1 = tree16_pairs(pv);                       // plane 1
-                const uint32_t xl = smem_u32(T.xlut) + 4 * c;
-                sts_f32_if(sa, scl * (s0.x + 2.f * (s1.x - lds_f32r(xl))), on);
-                sts_f32_if(sa + SLOT_V, scl * (s0.y + 2.f * (s1.y - lds_f32r(xl + 4 * MAX_C))), on);
-            }
-        } else {
-            // 1-bit: two groups per lane, summed as a pair
-            const int i = i0 + 2 * lane;
-            const int cf = col_uniform(U.ce, i0), cl = col_uniform(U.ce, min(i0 + SPAN - 1, U.n - 1));
-            int ca = cf, cb = cf;
-            if (cl == cf + 1) {                         // one column end inside the task
-                const int e = (int)__shfl_sync(0xffffffffu, U.ce, cf);
-                ca = cf + (i >= e);
-                cb = cf + (i + 1 >= e);
-            } else if (cf != cl) {
-                ca = col_within(U.ce, cf, cl, i);
-                cb = col_within(U.ce, cf, cl, min(i + 1, U.n - 1));
-            }
-            // branch-free: lanes past the end redo item 0 (always present) and store nothing
-            const bool one = i < U.n, two = i + 1 < U.n;
-            const int ii = one ? i : 0;
-            const uint4 v = lds_u32x4(U.pay + ii * 8);
-            const uint32_t rows2 = lds_u16(U.row + ii);
-            const uint32_t sc2 = lds_u32(U.sc + 2 * ii);
-            const uint32_t xl = smem_u32(T.xlut);
-            const uint32_t sb = slot_addr(slots, rows2 >> 8, cb), sa = slot_addr(slots, rows2 & 0xff, ca);
-            const float scb = half_bits(sc2 >> 16), sca = half_bits(sc2);
-            if constexpr (NX == 1) {
-                float va[16], vb[16];
-                plane_entries(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
-                plane_entries(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
-                const float2 sp = tree16x2(va, vb);
-                sts_f32_if(sb, scb * (2.f * sp.y - lds_f32r(xl + 4 * cb)), two);
-                sts_f32_if(sa, sca * (2.f * sp.x - lds_f32r(xl + 4 * ca)), one);
-            } else {
-                float2 pv[16];
-                plane_entries2(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, pv);
-                const float2 sx = tree16_pairs(pv);                       // item i, both vectors
-                sts_f32_if(sa, sca * (2.f * sx.x - lds_f32r(xl + 4 * ca)), one);
-                sts_f32_if(sa + SLOT_V, sca * (2.f * sx.y - lds_f32r(xl + 4 * MAX_C + 4 * ca)), one);
-                plane_entries2(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, pv);
-                const float2 sy = tree16_pairs(pv);                       // item i + 1
-                sts_f32_if(sb, scb * (2.f * sy.x - lds_f32r(xl + 4 * cb)), two);
-                sts_f32_if(sb + SLOT_V, scb * (2.f * sy.y - lds_f32r(xl + 4 * MAX_C + 4 * cb)), two);
-            }
-        }
+    // halves in the order (lane >> 2) & 1 first, so each quarter-warp's
+    // 16-byte loads fall in 8 distinct bank groups
+    const int c = t.c;
+    const int h0 = (lane >> 2) & 1;
+    const uint4 va = lds_u32x4(t.pay + h0 * 16), vb = lds_u32x4(t.pay + (h0 ^ 1) * 16);
+    const uint32_t xa = smem_u32(T.x4s) + (c * 2 + h0) * XH * 4, xb = smem_u32(T.x4s) + (c * 2 + (h0 ^ 1)) * XH * 4;
+    const uint32_t sa = slot_addr(slots, lds_u8(t.row), c);
+    const float scl = half_bits(lds_u16(t.sc)) * 0x1p100f;
+    if constexpr (NX == 1) {
+        const float2 aa = dot4_half(va, xa), ab = dot4_half(vb, xb);
+        const float4 z = lds_f32x4(smem_u32(T.x4z) + c * 16);     // (even, odd) of half 0, then of half 1
+        const float part = ((aa.x + ab.x) - 8.f * (z.x + z.z)) + ((aa.y + ab.y) - 8.f * (z.y + z.w));
+        sts_f32_if(sa, scl * part, t.on);
+    } else {
+        float2 aa0, aa1, ab0, ab1;
+        dot4_half2(va, xa, aa0, aa1);
+        dot4_half2(vb, xb, ab0, ab1);
+        const float4 z0 = lds_f32x4(smem_u32(T.x4z) + c * 16), z1 = lds_f32x4(smem_u32(T.x4z) + MAX_C * 16 + c * 16);
+        const float p0 = ((aa0.x + ab0.x) - 8.f * (z0.x + z0.z)) + ((aa0.y + ab0.y) - 8.f * (z0.y + z0.w));
+        const float p1 = ((aa1.x + ab1.x) - 8.f * (z1.x + z1.z)) + ((aa1.y + ab1.y) - 8.f * (z1.y + z1.w));
+        sts_f32_if(sa, scl * p0, t.on);
+        sts_f32_if(sa + SLOT_V, scl * p1, t.on);
     }
 }
 
-// One consumer warp's share of a unit (blob at shared address sblob, cols
-// group columns). The unit's tasks are numbered 8-bit, 4-bit, 2-bit, 1-bit
-// (costliest first); this warp takes tasks t0, t0 + tstep, ... of that
-// sequence (tstep a power of two). Each group's result goes to its slot in
-// the stage's slot array at shared address slots.
 template <int NX>
-__device__ __forceinline__ void consume_unit(const TablesT<NX>& T, uint32_t sblob, int C, int cols, uint32_t slots,
-                                             int t0, int tstep, int lane) {
-    // UnitHeader fields, read as three 16-byte words
-    const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
-    const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
-    const int n[4] = {(int)(h0.x & 0xFFFF), (int)(h0.x >> 16), (int)(h0.y & 0xFFFF), (int)(h0.y >> 16)};
-    const uint32_t pay16[4] = {h0.z & 0xFFFF, h0.z >> 16, h0.w & 0xFFFF, h0.w >> 16};
-    const uint32_t sc16[4] = {h1.x & 0xFFFF, h1.x >> 16, h1.y & 0xFFFF, h1.y >> 16};
-    const uint32_t row16[4] = {h1.z & 0xFFFF, h1.z >> 16, h1.w & 0xFFFF, h1.w >> 16};
-    auto view = [&](int w) {
-        UnitView U;
-        U.pay = sblob + pay16[w] * 16;
-        U.sc = sblob + sc16[w] * 16;
-        U.row = sblob + row16[w] * 16;
-        U.ce = lane < cols ? lds_u16(cc + 2 * (w * C + lane)) : 0xFFFFu;
-        U.n = n[w];
-        return U;
-    };
-    // first task of each width for this warp: the width's tasks start at base b
-    // in the unit's sequence; this warp's next index at or after b is
-    // b + ((t0 - b) mod tstep), tstep a power of two
-    const int nt3 = (n[3] + 31) >> 5, nt2 = (n[2] + 31) >> 5, nt1 = (n[1] + 31) >> 5;
-    const int m = tstep - 1;
-    if (n[3]) run_width<3, NX>(T, view(3), slots, t0 & m, tstep, lane);
-    if (n[2]) run_width<2, NX>(T, view(2), slots, (t0 - nt3) & m, tstep, lane);
-    if (n[1]) run_width<1, NX>(T, view(1), slots, (t0 - nt3 - nt2) & m, tstep, lane);
-    if (n[0]) run_width<0, NX>(T, view(0), slots, (t0 - nt3 - nt2 - nt1) & m, tstep, lane);
+__device__ __forceinline__ void body8(const TablesT<NX>& T, const Task& t, uint32_t slots, int lane) {
+    constexpr uint32_t SLOT_V = SLOT_FLOATS * 4;
+    // quarter (k + (lane >> 1)) & 3 in step k: conflict-free 16-byte loads
+    const int c = t.c;
+    const int q0 = lane >> 1;
+    const uint32_t sa = slot_addr(slots, lds_u8(t.row), c);
+    const float scl = half_bits(lds_u16(t.sc));
+    if constexpr (NX == 1) {
+        float part = 0.f;
+#pragma unroll
+        for (int step = 0; step < 4; ++step) {
+            const int q = (step + q0) & 3;
+            const uint4 v = lds_u32x4(t.pay + q * 16);
+            part += dot8_quarter(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
+        }
+        sts_f32_if(sa, scl * part, t.on);
+    } else {
+        float p0 = 0.f, p1 = 0.f;
+#pragma unroll
+        for (int step = 0; step < 4; ++step) {
+            const int q = (step + q0) & 3;
+            const uint4 v = lds_u32x4(t.pay + q * 16);
+            const float2 dd = dot8_quarter2(v, smem_u32(T.xs) + (c * 4 + q) * XQ * 4);
+            p0 += dd.x;
+            p1 += dd.y;
+        }
+        sts_f32_if(sa, scl * p0, t.on);
+        sts_f32_if(sa + SLOT_V, scl * p1, t.on);
+    }
+}
+
+template <int NX>
+__device__ __forceinline__ void body2(const TablesT<NX>& T, const Task& t, uint32_t slots) {
+    constexpr uint32_t SLOT_V = SLOT_FLOATS * 4;
+    const int c = t.c;
+    const uint4 pl = lds_u32x4(t.pay);
+    const uint32_t tb = smem_u32(T.lut) + c * LUT_COL_BYTES;
+    const uint32_t sa = slot_addr(slots, lds_u8(t.row), c);
+    const float scl = half_bits(lds_u16(t.sc));
+    if constexpr (NX == 1) {
+        float va[16], vb[16];
+        plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
+        plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
+        const float2 sp = tree16x2(va, vb);
+        sts_f32_if(sa, scl * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))), t.on);
+    } else {
+        float2 pv[16];
+        plane_entries2(tb, col_shift4(c), pl.x, pl.y, pv);
+        const float2 s0 = tree16_pairs(pv);                       // plane 0, both vectors
+        plane_entries2(tb, col_shift4(c), pl.z, pl.w, pv);
+        const float2 s1 = tree16_pairs(pv);                       // plane 1
+        const uint32_t xl = smem_u32(T.xlut) + 4 * c;
+        sts_f32_if(sa, scl * (s0.x + 2.f * (s1.x - lds_f32r(xl))), t.on);
+        sts_f32_if(sa + SLOT_V, scl * (s0.y + 2.f * (s1.y - lds_f32r(xl + 4 * MAX_C))), t.on);
+    }
+}
+
+template <int NX>
+__device__ __forceinline__ void body1(const TablesT<NX>& T, const Task& t, uint32_t slots) {
+    constexpr uint32_t SLOT_V = SLOT_FLOATS * 4;
+    const int ca = t.c, cb = t.c2;
+    const uint4 v = lds_u32x4(t.pay);
+    const uint32_t rows2 = lds_u16(t.row);
+    const uint32_t sc2 = lds_u32(t.sc);
+    const uint32_t xl = smem_u32(T.xlut);
+    const uint32_t sb = slot_addr(slots, rows2 >> 8, cb), sa = slot_addr(slots, rows2 & 0xff, ca);
+    const float scb = half_bits(sc2 >> 16), sca = half_bits(sc2);
+    if constexpr (NX == 1) {
+        float va[16], vb[16];
+        plane_entries(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
+        plane_entries(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
+        const float2 sp = tree16x2(va, vb);
+        sts_f32_if(sb, scb * (2.f * sp.y - lds_f32r(xl + 4 * cb)), t.on2);
+        sts_f32_if(sa, sca * (2.f * sp.x - lds_f32r(xl + 4 * ca)), t.on);
+    } else {
+        float2 pv[16];
+        plane_entries2(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, pv);
+        const float2 sx = tree16_pairs(pv);                       // first item, both vectors
+        sts_f32_if(sa, sca * (2.f * sx.x - lds_f32r(xl + 4 * ca)), t.on);
+        sts_f32_if(sa + SLOT_V, sca * (2.f * sx.y - lds_f32r(xl + 4 * MAX_C + 4 * ca)), t.on);
+        plane_entries2(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, pv);
+        const float2 sy = tree16_pairs(pv);                       // second item
+        sts_f32_if(sb, scb * (2.f * sy.x - lds_f32r(xl + 4 * cb)), t.on2);
+        sts_f32_if(sb + SLOT_V, scb * (2.f * sy.y - lds_f32r(xl + 4 * MAX_C + 4 * cb)), t.on2);
+    }
+}
+
+// One consumer warp's share of a unit (blob at shared address sblob): tasks
+// t0, t0 + tstep, ... of the unit's task table (8-bit tasks first, costliest
+// first). Each group's result goes to its slot in the stage's slot array at
+// shared address slots.
+template <int NX>
+__device__ __forceinline__ void consume_unit(const TablesT<NX>& T, uint32_t sblob, uint32_t slots, int t0, int tstep,
+                                             int lane) {
+    const uint32_t hw = lds_u32(sblob + offsetof(UnitHeader, ntask));     // ntask | task16 << 16
+    const int ntask = (int)(hw & 0xFFFFu);
+    const uint32_t tasks = sblob + (hw >> 16) * 16;
+    for (int k = t0; k < ntask; k += tstep) {
+        const uint4 d = lds_u32x4(tasks + k * 16);
+        const uint32_t w = (d.x >> 26) & 3u;
+        if (w == 0) body1<NX>(T, task64(sblob, d, lane), slots);
+        else if (w == 1) body2<NX>(T, task32(sblob, d, lane, 16), slots);
+        else if (w == 2) body4<NX>(T, task32(sblob, d, lane, 32), slots, lane);
+        else body8<NX>(T, task32(sblob, d, lane, 64), slots, lane);
+    }
 }
 
 // SwiGLU epilogue of a gate-up product whose rows alternate (row 2i the gate
@@ -864,8 +857,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             if (!dead) {
                 // tasks rotate over the team's warps from unit to unit, so no warp always draws the costly ones
                 const int t0 = (wt - (j >> lg_teams)) & (tw - 1);
-                consume_unit<NX>(T, stage0 + st * STAGE_BYTES, L.C, min(L.C, L.G - sj * L.C), smem_u32(T.slots[st][0]),
-                                 t0, tw, lane);
+                consume_unit<NX>(T, stage0 + st * STAGE_BYTES, smem_u32(T.slots[st][0]), t0, tw, lane);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty0 + 8 * st);
             }
@@ -1119,8 +1111,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv_chain_kernel(const ChainIt
                 if (!dead) {
                     // tasks rotate over the warps from unit to unit
                     const int t0 = (wt - j) & (TW - 1);
-                    consume_unit<1>(T, stage0 + st * STAGE_BYTES, L.C, min(L.C, L.G - sj * L.C), smem_u32(T.slots[st][0]),
-                                    t0, TW, lane);
+                    consume_unit<1>(T, stage0 + st * STAGE_BYTES, smem_u32(T.slots[st][0]), t0, TW, lane);
                     __syncwarp();
                     if (lane == 0) mbar_arrive(empty0 + 8 * st);
                 }

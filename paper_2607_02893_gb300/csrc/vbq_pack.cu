@@ -32,23 +32,38 @@ __global__ void validate_kernel(const uint8_t* __restrict__ codes, const uint8_t
     if (flags) atomicOr(err, flags);
 }
 
-// One block per unit (slab-major numbering), one thread per row: item counts per width.
-__global__ void count_kernel(const uint8_t* __restrict__ widths, int64_t N, int G, int C, int nrb,
-                             uint32_t* __restrict__ counts) {
-    __shared__ uint32_t cnt[4];
+// One block per unit (slab-major numbering), one thread per row: item counts
+// per width and the number of warp tasks the unit's column ends give
+// (unit_tasks), as counts[5u .. 5u + 4].
+__global__ void __launch_bounds__(RB) count_kernel(const uint8_t* __restrict__ widths, int64_t N, int G, int C,
+                                                   int nrb, uint32_t* __restrict__ counts) {
+    __shared__ uint32_t wcnt[RB / 32][4];
+    __shared__ uint16_t ce[4][MAX_C];
     const int u = blockIdx.x, rb = u % nrb, s = u / nrb;
-    if (threadIdx.x < 4) cnt[threadIdx.x] = 0;
-    __syncthreads();
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t row = (int64_t)rb * RB + threadIdx.x;
+    const bool valid = row < N;
     const int c0 = s * C, cols = min(C, G - c0);
-    uint32_t local[4] = {0, 0, 0, 0};
-    if (row < N) {
-        for (int c = 0; c < cols; ++c) local[width_index(widths[row * G + c0 + c]) & 3] += 1;
+    uint32_t run[4] = {0, 0, 0, 0};
+    for (int c = 0; c < cols; ++c) {
+        const int w = valid ? width_index(widths[row * G + c0 + c]) & 3 : 0;
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const uint32_t m = __ballot_sync(0xffffffffu, valid && w == v);
+            if (lane == 0) wcnt[warp][v] = __popc(m);
+        }
+        __syncthreads();
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            for (int pw = 0; pw < RB / 32; ++pw) run[v] += wcnt[pw][v];
+            if (threadIdx.x == 0) ce[v][c] = (uint16_t)run[v];
+        }
+        __syncthreads();
     }
-    for (int w = 0; w < 4; ++w)
-        if (local[w]) atomicAdd(&cnt[w], local[w]);
-    __syncthreads();
-    if (threadIdx.x < 4) counts[(int64_t)u * 4 + threadIdx.x] = cnt[threadIdx.x];
+    if (threadIdx.x == 0) {
+        for (int v = 0; v < 4; ++v) counts[(int64_t)u * 5 + v] = run[v];
+        counts[(int64_t)u * 5 + 4] = (uint32_t)unit_tasks(ce, cols, nullptr, nullptr);
+    }
 }
 
 // One block per unit, one thread per row (RB threads). Walks the unit's columns
@@ -74,6 +89,7 @@ __global__ void __launch_bounds__(RB) scatter_kernel(const uint8_t* __restrict__
     if (threadIdx.x < sizeof(UnitHeader) / 4)
         reinterpret_cast<uint32_t*>(blob)[threadIdx.x] = reinterpret_cast<const uint32_t*>(&headers[u])[threadIdx.x];
     uint16_t* cend = reinterpret_cast<uint16_t*>(blob + h.cc16 * 16);
+    __shared__ uint16_t ce_s[4][MAX_C];
     uint32_t run[4] = {0, 0, 0, 0};
     const uint32_t lt = (1u << lane) - 1u;
     for (int c = 0; c < cols; ++c) {
@@ -107,10 +123,16 @@ __global__ void __launch_bounds__(RB) scatter_kernel(const uint8_t* __restrict__
             uint32_t tot = 0;
             for (int pw = 0; pw < RB / 32; ++pw) tot += wcnt[pw][v];
             run[v] += tot;
-            if (threadIdx.x == 0) cend[v * L.C + c] = (uint16_t)run[v];
+            if (threadIdx.x == 0) {
+                cend[v * L.C + c] = (uint16_t)run[v];
+                ce_s[v][c] = (uint16_t)run[v];
+            }
         }
         __syncthreads();
     }
+    // the batch-1 product's warp tasks (the count was planned on the host from
+    // the same column ends)
+    if (threadIdx.x == 0) unit_tasks(ce_s, cols, &h, reinterpret_cast<TaskDesc*>(blob + h.task16 * 16));
 }
 
 // Unpack one item of width B into codes_out (64 bytes) and/or w_out
