@@ -169,7 +169,7 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     int64_t S = 0, units = 0;
     uint32_t max16 = 0;
     for (int cand : {16, 8, 4, 2, 1}) {
-        if (cand > G && cand != 1) continue;
+        if (cand > vbq::MAX_C || (cand > G && cand != 1)) continue;
         const int64_t Sc = (G + cand - 1) / cand, uc = nrb * Sc;
         const bool last = (cand == 1);
         if (!last && 2 * uc < sms) continue;          // fewer units than half the SMs: narrower slabs

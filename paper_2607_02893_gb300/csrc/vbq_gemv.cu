@@ -21,18 +21,21 @@
 // slab-major order, so consecutive units share their activations; on a slab
 // change the consumer warps rebuild, under a named barrier of their own, the
 // per-slab activation tables: x as fp32 and, for every 4 consecutive weights of
-// a group column, the 16 subset sums of their activations (a lookup table
-// indexed by 4 code bits). Per width:
-//   b = 1  one table lookup per 4 weights: S = sum of x over set bits, and
-//          the group's dot product is 2S - X (L_1(u) = 2u - 1, X = sum of x);
-//          two groups per lane, their sums added as f32x2 pairs;
-//   b = 2  the two bit planes use the same tables: S0 + 2 S1 - 2X;
+// a group column, the 16 signed sums of their activations (a lookup table
+// indexed by 4 code bits: bit i set adds x_i, clear subtracts it). Per width:
+//   b = 1  one table lookup per 4 weights; L_1(u) = 2u - 1 is the sign the
+//          table applies, so the group's dot product is the sum T of its 16
+//          lookups; two groups per lane, their sums added as f32x2 pairs;
+//   b = 2  the two bit planes use the same tables: with u = b0 + 2 b1,
+//          L_2(u) = b0 + 2 b1 - 2 = (2 b0 - 1) / 2 + (2 b1 - 1) - 1/2, so the
+//          dot product is T0 / 2 + T1 - X / 2 (X = sum of x);
 //   b = 4  codes are masked in place and read as exact denormal floats
 //          against activations pre-scaled per code slot (packed f32x2 FMAs);
 //          8X (summed in the same order) is subtracted for the zero level;
 //   b = 8  same with a byte permute and 2^23 + 128.
-// X is summed from the tables in the same order as the lookups, so a group
-// whose codes are all at the zero level contributes exactly 0. Each group's
+// X is summed from the tables in the same order as the lookups (and entry
+// 15 - m is exactly -entry m), so a group whose codes are all at the zero
+// level contributes exactly 0. Each group's
 // fp32 dot product is scaled once by its FP16 scale and stored in its
 // (row, column) slot; the copier sums a row's slots in a fixed order and
 // writes y directly (one slab per row) or through atomics (several slabs).
@@ -62,7 +65,9 @@ namespace {
 
 constexpr int NCW = 16;                  // consumer warps of the batch-1 kernel
 constexpr int NCT = 32 * NCW;            // consumer threads
-constexpr int G1_THREADS = 32 * (NCW + 1);
+constexpr int NCOPY = 2;                 // copier warps of the batch-1 kernel (unit j: copier j % 2)
+constexpr int G1_THREADS = 32 * (NCW + NCOPY);
+constexpr int CH_THREADS = 32 * (NCW + 1);    // the chain kernel: one copier warp
 constexpr int XQ = 20;                   // floats per 16-code quarter of x (16 + 4 pad: quarters use other banks)
 constexpr int XH = 36;                   // floats per 32-code half of the pre-scaled x (32 + 4 pad)
 constexpr int LUT_COL_BYTES = 1280;      // 16 tables x 64 bytes (+64 for odd columns), columns on 256-byte boundaries
@@ -388,16 +393,18 @@ __device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t
                 p4[i] = xv4[i] * __uint_as_float((uint32_t)(127 + 49 - e) << 23);
             }
             *reinterpret_cast<float4*>(&x4s[(c * 2 + (jj >> 5)) * XH + (jj & 31)]) = make_float4(p4[0], p4[1], p4[2], p4[3]);
-            const float t3 = x0 + x1, t12 = x3 + x2;
+            // entry m = sum_i (2 m_i - 1) x_i (code bit i of the nibble picks +x_i or
+            // -x_i), as p[m & 3] + q[m >> 2]; entry 15 - m is exactly -entry m
+            const float a = x0 + x1, b = x0 - x1, cc = x2 + x3, d = x2 - x3;
             float4* dst = reinterpret_cast<float4*>(T.lut + v * LUT_BYTES + c * LUT_COL_BYTES + (c & 1) * 64 + jn * 64);
-            dst[0] = make_float4(0.f, x0, x1, t3);
-            dst[1] = make_float4(x2, x2 + x0, x2 + x1, x2 + t3);
-            dst[2] = make_float4(x3, x3 + x0, x3 + x1, x3 + t3);
-            dst[3] = make_float4(t12, t12 + x0, t12 + x1, t12 + t3);
+            dst[0] = make_float4(-a + -cc, b + -cc, -b + -cc, a + -cc);
+            dst[1] = make_float4(-a + d, b + d, -b + d, a + d);
+            dst[2] = make_float4(-a + -d, b + -d, -b + -d, a + -d);
+            dst[3] = make_float4(-a + cc, b + cc, -b + cc, a + cc);
             // xlut: balanced tree over the column's 16 all-ones entries (xor 1, 2, 4, 8
             // pair them as tree16x2 pairs the lookups)
             const unsigned half = (ct & 16) ? 0xFFFF0000u : 0x0000FFFFu;
-            float sv = t12 + t3;
+            float sv = a + cc;
             sv += __shfl_xor_sync(half, sv, 1);
             sv += __shfl_xor_sync(half, sv, 2);
             sv += __shfl_xor_sync(half, sv, 4);
@@ -567,12 +574,14 @@ __device__ __forceinline__ void body2(const TablesT<NX>& T, const Task& t, uint3
     const uint32_t tb = smem_u32(T.lut) + c * LUT_COL_BYTES;
     const uint32_t sa = slot_addr(slots, lds_u8(t.row), c);
     const float scl = half_bits(lds_u16(t.sc));
+    // T0 / 2 + T1 - X / 2: for an all-zero-level group (b0 = 0, b1 = 1) T0 = -X
+    // and T1 = X exactly, and X - X / 2 is exact, so the result is exactly 0
     if constexpr (NX == 1) {
         float va[16], vb[16];
         plane_entries(tb, col_shift4(c), pl.x, pl.y, va);
         plane_entries(tb, col_shift4(c), pl.z, pl.w, vb);
         const float2 sp = tree16x2(va, vb);
-        sts_f32_if(sa, scl * (sp.x + 2.f * (sp.y - lds_f32r(smem_u32(T.xlut) + 4 * c))), t.on);
+        sts_f32_if(sa, scl * ((0.5f * sp.x + sp.y) - 0.5f * lds_f32r(smem_u32(T.xlut) + 4 * c)), t.on);
     } else {
         float2 pv[16];
         plane_entries2(tb, col_shift4(c), pl.x, pl.y, pv);
@@ -580,8 +589,8 @@ __device__ __forceinline__ void body2(const TablesT<NX>& T, const Task& t, uint3
         plane_entries2(tb, col_shift4(c), pl.z, pl.w, pv);
         const float2 s1 = tree16_pairs(pv);                       // plane 1
         const uint32_t xl = smem_u32(T.xlut) + 4 * c;
-        sts_f32_if(sa, scl * (s0.x + 2.f * (s1.x - lds_f32r(xl))), t.on);
-        sts_f32_if(sa + SLOT_V, scl * (s0.y + 2.f * (s1.y - lds_f32r(xl + 4 * MAX_C))), t.on);
+        sts_f32_if(sa, scl * ((0.5f * s0.x + s1.x) - 0.5f * lds_f32r(xl)), t.on);
+        sts_f32_if(sa + SLOT_V, scl * ((0.5f * s0.y + s1.y) - 0.5f * lds_f32r(xl + 4 * MAX_C)), t.on);
     }
 }
 
@@ -592,7 +601,6 @@ __device__ __forceinline__ void body1(const TablesT<NX>& T, const Task& t, uint3
     const uint4 v = lds_u32x4(t.pay);
     const uint32_t rows2 = lds_u16(t.row);
     const uint32_t sc2 = lds_u32(t.sc);
-    const uint32_t xl = smem_u32(T.xlut);
     const uint32_t sb = slot_addr(slots, rows2 >> 8, cb), sa = slot_addr(slots, rows2 & 0xff, ca);
     const float scb = half_bits(sc2 >> 16), sca = half_bits(sc2);
     if constexpr (NX == 1) {
@@ -600,18 +608,18 @@ __device__ __forceinline__ void body1(const TablesT<NX>& T, const Task& t, uint3
         plane_entries(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, va);
         plane_entries(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, vb);
         const float2 sp = tree16x2(va, vb);
-        sts_f32_if(sb, scb * (2.f * sp.y - lds_f32r(xl + 4 * cb)), t.on2);
-        sts_f32_if(sa, sca * (2.f * sp.x - lds_f32r(xl + 4 * ca)), t.on);
+        sts_f32_if(sb, scb * sp.y, t.on2);
+        sts_f32_if(sa, sca * sp.x, t.on);
     } else {
         float2 pv[16];
         plane_entries2(smem_u32(T.lut) + ca * LUT_COL_BYTES, col_shift4(ca), v.x, v.y, pv);
         const float2 sx = tree16_pairs(pv);                       // first item, both vectors
-        sts_f32_if(sa, sca * (2.f * sx.x - lds_f32r(xl + 4 * ca)), t.on);
-        sts_f32_if(sa + SLOT_V, sca * (2.f * sx.y - lds_f32r(xl + 4 * MAX_C + 4 * ca)), t.on);
+        sts_f32_if(sa, sca * sx.x, t.on);
+        sts_f32_if(sa + SLOT_V, sca * sx.y, t.on);
         plane_entries2(smem_u32(T.lut) + cb * LUT_COL_BYTES, col_shift4(cb), v.z, v.w, pv);
         const float2 sy = tree16_pairs(pv);                       // second item
-        sts_f32_if(sb, scb * (2.f * sy.x - lds_f32r(xl + 4 * cb)), t.on2);
-        sts_f32_if(sb + SLOT_V, scb * (2.f * sy.y - lds_f32r(xl + 4 * MAX_C + 4 * cb)), t.on2);
+        sts_f32_if(sb, scb * sy.x, t.on2);
+        sts_f32_if(sb + SLOT_V, scb * sy.y, t.on2);
     }
 }
 
@@ -660,6 +668,27 @@ __device__ __forceinline__ void swiglu_rows(const LayoutView& L, const float* y,
     }
 }
 
+// Split-K for one copier: true once every row block it adds into (units
+// u_begin + j for j = cp, cp + step, ... below n) has been zeroed in this call
+// (flag == epoch), within the wait limit. Copier 0 zeroes this block's own
+// slab-0 rows, so it skips those; the others wait for them like any other.
+// Lane i watches the copier's units i, i + 32, ...; acquire loads.
+__device__ __forceinline__ bool copier_flags_ready(const LayoutView& L, uint32_t epoch, int u_begin, int n, int cp,
+                                                   int step, int lane) {
+    bool seen = true;
+    const unsigned long long t0 = global_ns();
+    for (int j = cp + step * lane; j < n && seen; j += 32 * step) {
+        const int u = u_begin + j;
+        if (u >= L.nrb || cp != 0) {
+            const uint32_t* f = L.ctl + 2 + (u % L.nrb);
+            while (!(seen = ld_acquire_gpu(f) == epoch))
+                if (global_ns() - t0 > WAIT_LIMIT_NS) break;
+        }
+    }
+    __syncwarp();                       // every lane's later additions after every acquire
+    return __all_sync(0xffffffffu, seen);
+}
+
 // NX activation vectors x (NX x K, row-major) and outputs y (NX x N).
 template <int NX, int MODE>
 __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
@@ -668,6 +697,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                                                               const float* __restrict__ gu) {
     static_assert(MODE == MODE_PLAIN || NX == 1, "the SwiGLU forms take one activation vector");
     constexpr int NSTAGE = Geo<NX>::nstage;
+    static_assert(NSTAGE % NCOPY == 0, "each stage belongs to one copier");
     extern __shared__ __align__(16) unsigned char smem_raw[];
     // stages and tables on a 256-byte boundary: lookups merge a byte into table addresses
     unsigned char* base = smem_raw + ((256u - (smem_u32(smem_raw) & 255u)) & 255u);
@@ -714,11 +744,11 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         const int64_t k0 = (int64_t)s0 * L.C * GROUP;
         if constexpr (MODE == MODE_SWIGLU_IN) {      // 8 bytes (a gate-up pair) per activation
             const int lines = (min(L.C, L.G - s0 * L.C) * GROUP * 8 + 127) / 128;
-            if (tid >= 32 && tid - 32 < lines) prefetch_l2(gu + 2 * k0 + (int64_t)(tid - 32) * 32);
+            if (tid >= 32 * NCOPY && tid - 32 * NCOPY < lines) prefetch_l2(gu + 2 * k0 + (int64_t)(tid - 32 * NCOPY) * 32);
         } else {
             const int lines = (min(L.C, L.G - s0 * L.C) * GROUP * 2 + 127) / 128;
-            if (tid >= 32 && tid - 32 < NX * lines) {
-                const int v = (tid - 32) / lines, ln = (tid - 32) - v * lines;
+            if (tid >= 32 * NCOPY && tid - 32 * NCOPY < NX * lines) {
+                const int v = (tid - 32 * NCOPY) / lines, ln = (tid - 32 * NCOPY) - v * lines;
                 prefetch_l2(x + (int64_t)v * L.K + k0 + (int64_t)ln * 64);
             }
         }
@@ -728,48 +758,60 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     if (dep != DEP_GROUP_NEXT) asm volatile("griddepcontrol.wait;" ::: "memory");
     if (dep == DEP_GROUP_FIRST) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-    if (warp == 0) {
-        // ---- copier: split-K zeroing, then per unit: rows out, next copy in ----
+    if (warp < NCOPY) {
+        // ---- copiers: split-K zeroing, then per unit j = cp, cp + NCOPY, ...:
+        // rows out, next copy in (copier cp owns the stages s = cp mod NCOPY) ----
+        const int cp = warp;
         uint32_t epoch = 0;
         if (L.S > 1) {
-            // this call's epoch; zero y for the row blocks whose slab 0 this block
-            // owns (units u < nrb) and publish them
             epoch = call_epoch(L.ctl);
-            const int z_end = min(u_end, L.nrb);
-            for (int u = u_begin; u < z_end; ++u) {
-                const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
+            if (cp == 0) {
+                // zero y for the row blocks whose slab 0 this block owns (units
+                // u < nrb) and publish them
+                const int z_end = min(u_end, L.nrb);
+                for (int u = u_begin; u < z_end; ++u) {
+                    const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
 #pragma unroll
-                for (int v = 0; v < NX; ++v) {
-                    float* dst = y + (int64_t)v * L.N + (int64_t)u * RB;
-                    for (int r = lane; r < rows; r += 32) dst[r] = 0.f;
+                    for (int v = 0; v < NX; ++v) {
+                        float* dst = y + (int64_t)v * L.N + (int64_t)u * RB;
+                        for (int r = lane; r < rows; r += 32) dst[r] = 0.f;
+                    }
                 }
-            }
-            __syncwarp();
-            // release stores, one unit per lane in parallel: the warp's zeros
-            // (ordered by __syncwarp) before each flag
-            for (int u = u_begin + lane; u < z_end; u += 32) {
-                if (MODE == MODE_SWIGLU_EPI) L.ctl[2 + L.nrb + u] = 0u;     // SwiGLU slab count, before the flag's release
-                st_release_gpu(L.ctl + 2 + u, epoch);
+                __syncwarp();
+                // release stores, one unit per lane in parallel: the warp's zeros
+                // (ordered by __syncwarp) before each flag
+                for (int u = u_begin + lane; u < z_end; u += 32) {
+                    if (MODE == MODE_SWIGLU_EPI) L.ctl[2 + L.nrb + u] = 0u;     // SwiGLU slab count, before the flag's release
+                    st_release_gpu(L.ctl + 2 + u, epoch);
+                }
             }
         }
         bool dead = false;
-        if (L.S > 1 && !split_k_flags_ready(L, epoch, u_begin, u_end, lane)) {
-            // a row block this block adds into was never zeroed in time
+        // a row block this copier adds into that was never zeroed in time (the
+        // other copiers also wait for copier 0's zeroing of this block's own rows)
+        if (L.S > 1 && !copier_flags_ready(L, epoch, u_begin, n_units, cp, NCOPY, lane)) {
             dead = true;
             if (lane == 0) raise_abort(&T.abort);
         }
-        int st = 0, rbw = rb0, issued = n_units < NSTAGE ? n_units : NSTAGE;
-        uint32_t par = 0;
+        int jdone = -1;                 // the last unit this copier flushed (and refilled after)
         int pend_rb = -1;               // SwiGLU: row block whose slab count's reply is pending
-        uint32_t pend_count = 0;        // (lane 0) that count before this block's addition
-        for (int j = 0; j < n_units; ++j) {
-            // nap between polls, except on the block's last unit, whose rows end the block
-            if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, j + 1 < n_units ? 256 : 0)) {
+        uint32_t pend_count = 0;        // (lane 0) that count before this copier's addition
+        for (int j = cp; j < n_units; j += NCOPY) {
+            const int st = j & (NSTAGE - 1);
+            const uint32_t par = (uint32_t)(j / NSTAGE) & 1u;
+            const int u = u_begin + j, rbw = u % L.nrb, sw = u / L.nrb;
+            // nap between polls, except on the block's last units, whose rows end the block
+            if (!dead && !warp_wait(empty0 + 8 * st, par, abort_addr, j + NCOPY < n_units ? 256 : 0)) {
                 dead = true;
                 if (lane == 0) raise_abort(&T.abort);
             }
             if (!dead) {
                 const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
+                // the stage's next unit rewrites every slot this one wrote unless it
+                // has fewer columns (the last, partial slab): zero only then
+                const int cols = min(L.C, L.G - sw * L.C);
+                const int un = u + NSTAGE;
+                const bool rezero = j + NSTAGE < n_units && min(L.C, L.G - (un / L.nrb) * L.C) < cols;
 #pragma unroll
                 for (int v = 0; v < NX; ++v)            // per vector: its slots into its row of y
 #pragma unroll
@@ -778,16 +820,18 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                     float* yr = y + (int64_t)v * L.N + (int64_t)rbw * RB;
                     // row r's 16 slots as four 16-byte chunks, chunk (k + (lane >> 1)) & 3
                     // at step k (each quarter-warp touches 8 distinct bank groups);
-                    // summed as a tree, then zeroed for the stage's next unit
+                    // summed as a tree
                     const int r = lane + 32 * q;
                     const uint32_t ra = sl + (uint32_t)r * 64;
-                    float4 a[4];
+                    float4 a4[4];
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) a[k] = lds_f32x4(ra + (((k + (lane >> 1)) & 3) << 4));
+                    for (int k = 0; k < 4; ++k) a4[k] = lds_f32x4(ra + (((k + (lane >> 1)) & 3) << 4));
+                    if (rezero) {
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) sts_zero4(ra + (((k + (lane >> 1)) & 3) << 4));
-                    const float sum = (((a[0].x + a[0].y) + (a[0].z + a[0].w)) + ((a[1].x + a[1].y) + (a[1].z + a[1].w))) +
-                                      (((a[2].x + a[2].y) + (a[2].z + a[2].w)) + ((a[3].x + a[3].y) + (a[3].z + a[3].w)));
+                        for (int k = 0; k < 4; ++k) sts_zero4(ra + (((k + (lane >> 1)) & 3) << 4));
+                    }
+                    const float sum = (((a4[0].x + a4[0].y) + (a4[0].z + a4[0].w)) + ((a4[1].x + a4[1].y) + (a4[1].z + a4[1].w))) +
+                                      (((a4[2].x + a4[2].y) + (a4[2].z + a4[2].w)) + ((a4[3].x + a4[3].y) + (a4[3].z + a4[3].w)));
                     if (r < rows) {
                         if (L.S == 1) yr[r] = sum;
                         else red_global(yr + r, sum);
@@ -800,10 +844,9 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                     }
                 }
                 __syncwarp();
-                if (j + NSTAGE < n_units) {
-                    if (lane == 0) issue_unit(L, u_begin + j + NSTAGE, stage0 + st * STAGE_BYTES, full0 + 8 * st);
-                    ++issued;
-                }
+                if (j + NSTAGE < n_units && lane == 0)
+                    issue_unit(L, u_begin + j + NSTAGE, stage0 + st * STAGE_BYTES, full0 + 8 * st);
+                jdone = j;
                 if (MODE == MODE_SWIGLU_EPI && L.S > 1) {
                     // SwiGLU: count this unit's slab, then act on the previous unit's count
                     uint32_t count = 0;
@@ -816,8 +859,6 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                     pend_count = count;
                 }
             }
-            if (++st == NSTAGE) { st = 0; par ^= 1; }
-            if (++rbw == L.nrb) rbw = 0;
         }
         if (MODE == MODE_SWIGLU_EPI && L.S > 1 && pend_rb >= 0) {
             if (__shfl_sync(0xffffffffu, pend_count, 0) + 1u == (uint32_t)L.S) {
@@ -826,21 +867,25 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             }
         }
         if (dead && lane == 0) {
-            // let every copy this block started land before the block exits: the
-            // last unit issued into each stage, with that unit's parity (a phase
-            // that already completed returns at once)
-            for (int i = 0; i < NSTAGE && i < issued; ++i) {
-                const int jl = i + ((issued - 1 - i) / NSTAGE) * NSTAGE;   // last unit issued into stage i
-                mbar_wait_bounded(full0 + 8 * i, (uint32_t)((jl / NSTAGE) & 1));
+            // let every copy this copier's stages received land before the block
+            // exits: units below NSTAGE were issued at the start, and each flushed
+            // unit j issued j + NSTAGE, so the last unit issued into stage i is the
+            // largest k = i mod NSTAGE below both n_units and jdone + NSTAGE + 1;
+            // wait for it with its parity (a completed phase returns at once)
+            const int kmax = min(n_units - 1, max(jdone + NSTAGE, NSTAGE - 1));
+            for (int i = cp; i < NSTAGE; i += NCOPY) {
+                if (i > kmax) continue;
+                const int k = kmax - ((kmax - i) % NSTAGE);
+                mbar_wait_bounded(full0 + 8 * i, (uint32_t)((k / NSTAGE) & 1));
             }
         }
-        if (L.S > 1 && lane == 0) call_done(L.ctl);      // this block's share of the call count
+        if (cp == 0 && L.S > 1 && lane == 0) call_done(L.ctl);      // this block's share of the call count
         // a grouped product that started without waiting completes only after
         // its predecessor, so completion stays in stream order
-        if (dep == DEP_GROUP_NEXT && lane == 0) asm volatile("griddepcontrol.wait;" ::: "memory");
+        if (cp == 0 && dep == DEP_GROUP_NEXT && lane == 0) asm volatile("griddepcontrol.wait;" ::: "memory");
     } else {
         // ---- consumers: team `team` takes units j = team, team + teams, ... ----
-        const int cw = warp - 1, ct = tid - 32, team = cw / tw, wt = cw - team * tw;
+        const int cw = warp - NCOPY, ct = tid - 32 * NCOPY, team = cw / tw, wt = cw - team * tw;
         const int s_last = (u_end - 1) / L.nrb;
         bool dead = false;
         int cur = s0;
@@ -944,7 +989,7 @@ __device__ __forceinline__ void chain_prefetch_x(const ChainItem* items, const C
     if (lane < lines) prefetch_l2(items[c.i].x + ((int64_t)s * C + lane) * GROUP);
 }
 
-__global__ void __launch_bounds__(G1_THREADS, 1) gemv_chain_kernel(const ChainItem* __restrict__ items, int count,
+__global__ void __launch_bounds__(CH_THREADS, 1) gemv_chain_kernel(const ChainItem* __restrict__ items, int count,
                                                                    uint32_t* __restrict__ cctl) {
     constexpr int NSTAGE = Geo<1>::nstage;
     // one team: every consumer warp works on every unit (a chain's products are
@@ -969,7 +1014,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv_chain_kernel(const ChainIt
         T.abort = 0;
         fence_barrier_init();
     }
-    for (int i = tid; i < NSTAGE * SLOT_FLOATS; i += G1_THREADS) (&T.slots[0][0][0])[i] = 0.f;
+    for (int i = tid; i < NSTAGE * SLOT_FLOATS; i += CH_THREADS) (&T.slots[0][0][0])[i] = 0.f;
     __syncthreads();
     // the copier's issue position, and the first copies (weights only: before
     // the wait for the previous kernel)
@@ -991,7 +1036,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv_chain_kernel(const ChainIt
     // y is an input of the chain, so this may run ahead of any product), then
     // counts itself in `zeroed`; a copier adds into y only once every block
     // has (one grid-wide wait per launch instead of flags per product).
-    for (int i = warp; i < count; i += G1_THREADS / 32) {
+    for (int i = warp; i < count; i += CH_THREADS / 32) {
         const LayoutView& Li = items[i].L;
         if (Li.S > 1) {
             int ub, ue;
@@ -1170,7 +1215,7 @@ cudaError_t launch_chain(const ChainItem* items, int count, uint32_t* cctl, int 
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(blocks);
-    cfg.blockDim = dim3(G1_THREADS);
+    cfg.blockDim = dim3(CH_THREADS);
     cfg.dynamicSmemBytes = gemv1_smem<1>();
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
