@@ -129,6 +129,17 @@ __device__ __forceinline__ float2 ld_relaxed_gpu_f32x2(const float* p) {
     return v;
 }
 
+// Shared-memory words at CTA scope: a release addition (no reply) and an
+// acquire load.
+__device__ __forceinline__ void red_release_cta_shared_add(uint32_t addr, uint32_t v) {
+    asm volatile("red.release.cta.shared::cta.add.u32 [%0], %1;" :: "r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_acquire_cta_shared(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+
 // Release reduction at GPU scope (no reply): a chain's per-product completion counts.
 __device__ __forceinline__ void red_release_gpu_add(uint32_t* p, uint32_t v) {
     asm volatile("red.release.gpu.global.add.u32 [%0], %1;" :: "l"(p), "r"(v) : "memory");

@@ -116,6 +116,7 @@ struct __align__(16) TablesT {
     float slots[Geo<NX>::nstage][NX][SLOT_FLOATS];   // per stage and vector: one value per (row, column) (see slot_addr)
     unsigned long long full[Geo<NX>::nstage];        // blob landed (TMA transaction count)
     unsigned long long empty[Geo<NX>::nstage];       // the unit's team is done (one arrival per team warp)
+    uint32_t sk_ok;                      // split-K: copiers whose flag checks passed (+1 each; 0x10000 on failure)
     int abort;                           // set by any role whose wait ran out
 };
 template <int NX> struct TablesCheck {
@@ -623,17 +624,20 @@ __device__ __forceinline__ void body1(const TablesT<NX>& T, const Task& t, uint3
     }
 }
 
-// One consumer warp's share of a unit (blob at shared address sblob): tasks
-// t0, t0 + tstep, ... of the unit's task table (8-bit tasks first, costliest
-// first). Each group's result goes to its slot in the stage's slot array at
-// shared address slots.
+// One consumer warp's share of a unit (blob at shared address sblob): of the
+// unit's task table (8-bit tasks first, so costliest first), warp t0 of
+// tstep takes task t0 in round 0, tstep - 1 - t0 of the next tstep in round
+// 1, and so on alternately (snake order: a warp that drew a costly task early
+// draws a cheap one next). Each group's result goes to its slot in the
+// stage's slot array at shared address slots.
 template <int NX>
 __device__ __forceinline__ void consume_unit(const TablesT<NX>& T, uint32_t sblob, uint32_t slots, int t0, int tstep,
                                              int lane) {
     const uint32_t hw = lds_u32(sblob + offsetof(UnitHeader, ntask));     // ntask | task16 << 16
     const int ntask = (int)(hw & 0xFFFFu);
     const uint32_t tasks = sblob + (hw >> 16) * 16;
-    for (int k = t0; k < ntask; k += tstep) {
+    const int back = tstep - 1 - t0;
+    for (int k = t0, r = 0; k < ntask; k += ((r ^= 1) ? 2 * back + 1 : 2 * t0 + 1)) {
         const uint4 d = lds_u32x4(tasks + k * 16);
         const uint32_t w = (d.x >> 26) & 3u;
         if (w == 0) body1<NX>(T, task64(sblob, d, lane), slots);
@@ -689,6 +693,41 @@ __device__ __forceinline__ bool copier_flags_ready(const LayoutView& L, uint32_t
     return __all_sync(0xffffffffu, seen);
 }
 
+// Consumer warps of one team (named barrier 2 + team; tw warps).
+__device__ __forceinline__ void team_sync(int team, int tw) {
+    asm volatile("bar.sync %0, %1;" :: "r"(2 + team), "r"(32 * tw) : "memory");
+}
+
+// A team's cooperative flush of a finished unit: warp wt of tw takes rows
+// [wt * 128 / tw, (wt + 1) * 128 / tw), tw / 4 lanes per row, each lane
+// summing 64 / tw of the row's 16 slots (16-byte chunks; absent columns hold
+// 0), then the row's lanes added by xor shuffles in a fixed order. Rows are
+// stored when the matrix has one slab and added otherwise.
+template <int NX>
+__device__ __forceinline__ void team_flush(const TablesT<NX>& T, const LayoutView& L, float* __restrict__ y, int st,
+                                           int rb, int wt, int tw, int lane) {
+    const int lpr = tw >> 2;                    // lanes per row: 4 (16 warps) or 2 (8 warps)
+    const int rpw = 32 / lpr;                   // rows per warp
+    const int r = wt * rpw + lane / lpr, part = lane % lpr;
+    const int rows = min(RB, (int)(L.N - (int64_t)rb * RB));
+    const int chunks = 4 / lpr;                 // 16-byte chunks per lane
+#pragma unroll
+    for (int v = 0; v < NX; ++v) {
+        const uint32_t ra = smem_u32(T.slots[st][v]) + (uint32_t)r * 64;
+        float sum = 0.f;
+        for (int k = 0; k < chunks; ++k) {
+            const float4 a = lds_f32x4(ra + ((part * chunks + k) << 4));
+            sum += (a.x + a.y) + (a.z + a.w);
+        }
+        for (int o = 1; o < lpr; o <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+        if (part == 0 && r < rows) {
+            float* yr = y + (int64_t)v * L.N + (int64_t)rb * RB + r;
+            if (L.S == 1) *yr = sum;
+            else red_global(yr, sum);
+        }
+    }
+}
+
 // NX activation vectors x (NX x K, row-major) and outputs y (NX x N).
 template <int NX, int MODE>
 __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
@@ -698,6 +737,9 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     static_assert(MODE == MODE_PLAIN || NX == 1, "the SwiGLU forms take one activation vector");
     constexpr int NSTAGE = Geo<NX>::nstage;
     static_assert(NSTAGE % NCOPY == 0, "each stage belongs to one copier");
+    // each team flushes its own last unit (the copiers would add a hand-off
+    // at the very end of the block); the SwiGLU epilogue stays with the copiers
+    constexpr bool COOP = MODE != MODE_SWIGLU_EPI;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     // stages and tables on a 256-byte boundary: lookups merge a byte into table addresses
     unsigned char* base = smem_raw + ((256u - (smem_u32(smem_raw) & 255u)) & 255u);
@@ -726,6 +768,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             mbar_init(empty0 + 8 * i, tw);
         }
         T.abort = 0;
+        T.sk_ok = 0;
         fence_barrier_init();
     }
     // slots no group of a unit writes (rows past N, columns past the last
@@ -793,10 +836,13 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             dead = true;
             if (lane == 0) raise_abort(&T.abort);
         }
+        // the flags this warp acquired, passed on to the consumers' final flush
+        if (L.S > 1 && lane == 0) red_release_cta_shared_add(smem_u32(&T.sk_ok), dead ? 0x10000u : 1u);
         int jdone = -1;                 // the last unit this copier flushed (and refilled after)
         int pend_rb = -1;               // SwiGLU: row block whose slab count's reply is pending
         uint32_t pend_count = 0;        // (lane 0) that count before this copier's addition
         for (int j = cp; j < n_units; j += NCOPY) {
+            if (COOP && j >= n_units - teams) break;          // each team flushes its last unit itself
             const int st = j & (NSTAGE - 1);
             const uint32_t par = (uint32_t)(j / NSTAGE) & 1u;
             const int u = u_begin + j, rbw = u % L.nrb, sw = u / L.nrb;
@@ -904,7 +950,24 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                 const int t0 = (wt - (j >> lg_teams)) & (tw - 1);
                 consume_unit<NX>(T, stage0 + st * STAGE_BYTES, smem_u32(T.slots[st][0]), t0, tw, lane);
                 __syncwarp();
-                if (lane == 0) mbar_arrive(empty0 + 8 * st);
+                if (!(COOP && j >= n_units - teams) && lane == 0) mbar_arrive(empty0 + 8 * st);
+            }
+            if (COOP && j >= n_units - teams) {
+                // the team's last unit: every warp of the team flushes 128 / tw of its rows
+                team_sync(team, tw);
+                if (L.S > 1) {
+                    // split-K: after the copiers' flag checks (bounded wait)
+                    uint32_t g = 0;
+                    const unsigned long long w0 = global_ns();
+                    while ((g = ld_acquire_cta_shared(smem_u32(&T.sk_ok))) < (uint32_t)NCOPY &&
+                           !lds_volatile(abort_addr) && global_ns() - w0 < WAIT_LIMIT_NS)
+                        __nanosleep(32);
+                    if (g != (uint32_t)NCOPY) {
+                        dead = true;
+                        if (lane == 0) raise_abort(&T.abort);
+                    }
+                }
+                if (!dead) team_flush<NX>(T, L, y, st, rbj, wt, tw, lane);
             }
             rbj += teams;
             while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
