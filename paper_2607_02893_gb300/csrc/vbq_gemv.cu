@@ -624,20 +624,17 @@ __device__ __forceinline__ void body1(const TablesT<NX>& T, const Task& t, uint3
     }
 }
 
-// One consumer warp's share of a unit (blob at shared address sblob): of the
-// unit's task table (8-bit tasks first, so costliest first), warp t0 of
-// tstep takes task t0 in round 0, tstep - 1 - t0 of the next tstep in round
-// 1, and so on alternately (snake order: a warp that drew a costly task early
-// draws a cheap one next). Each group's result goes to its slot in the
-// stage's slot array at shared address slots.
+// One consumer warp's share of a unit (blob at shared address sblob): tasks
+// t0, t0 + tstep, ... of the unit's task table (8-bit tasks first, costliest
+// first). Each group's result goes to its slot in the stage's slot array at
+// shared address slots.
 template <int NX>
 __device__ __forceinline__ void consume_unit(const TablesT<NX>& T, uint32_t sblob, uint32_t slots, int t0, int tstep,
                                              int lane) {
     const uint32_t hw = lds_u32(sblob + offsetof(UnitHeader, ntask));     // ntask | task16 << 16
     const int ntask = (int)(hw & 0xFFFFu);
     const uint32_t tasks = sblob + (hw >> 16) * 16;
-    const int back = tstep - 1 - t0;
-    for (int k = t0, r = 0; k < ntask; k += ((r ^= 1) ? 2 * back + 1 : 2 * t0 + 1)) {
+    for (int k = t0; k < ntask; k += tstep) {
         const uint4 d = lds_u32x4(tasks + k * 16);
         const uint32_t w = (d.x >> 26) & 3u;
         if (w == 0) body1<NX>(T, task64(sblob, d, lane), slots);
