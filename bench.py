@@ -449,6 +449,17 @@ def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev
                                      "the headline's products as one vbq_chain_run with no waits (independent "
                                      "products in one persistent launch): the kernel's streaming upper bound")
     chain.free()
+    # the decode step's own dependencies: K and V read Q's input, up reads
+    # gate's, so they share their predecessor's dependencies (waits 2)
+    by_input = [2 if m.name.rpartition(".")[2] in ("k", "v", "up") else 1 for m in work.mats] * copies
+    if 2 in by_input:
+        chain = vbq.Chain(layouts, x0, y0, by_input)
+        ms = time_graph(torch, stream, lambda: chain.run(stream=stream), steps, warm)
+        out["chain_by_input"] = entry(ms, step_bytes, copies, len(layouts),
+                                      "the headline's products as one vbq_chain_run with the decode step's "
+                                      "dependencies: Q, K, V wait for the previous layer, O for Q, K and V, gate "
+                                      "and up for O, down for gate and up")
+        chain.free()
     # the decode order with products that read the same input issued as one
     # group: per layer (Q, K, V) together, O, (gate, up) together, down
     names = [m.name for m in work.mats] * copies

@@ -288,9 +288,14 @@ vbq_status_t vbq_gemv_group(const vbq_layout* const* layouts, const uint16_t* co
  *                    product i reads x_i only after every earlier product has
  *                    completed, as when x_i derives from earlier outputs (the
  *                    default; the results equal those of count vbq_gemv calls
- *                    in order). waits[i] = 0: product i does not depend on
- *                    earlier products of the chain. Since no y_i is an input of
- *                    the chain, a product may zero its own y_i early.
+ *                    in order). waits[i] = 2: product i has the dependencies
+ *                    of product i - 1 and does not depend on it, as when
+ *                    products read the same input (a decode step's Q, K and V,
+ *                    or gate and up): it may run alongside product i - 1, and a
+ *                    later product with waits = 1 waits for both. waits[i] = 0:
+ *                    product i does not depend on earlier products of the
+ *                    chain. Since no y_i is an input of the chain, a product
+ *                    may zero its own y_i early.
  *   count            1 .. 2^20.
  *   out              receives the chain on VBQ_OK.
  * It allocates a small device buffer (descriptors and completion counts) and

@@ -428,14 +428,22 @@ vbq_status_t vbq_chain_create(const vbq_layout* const* layouts, const uint16_t* 
         if (!xs[i] || !ys[i]) return fail(VBQ_ERR_ARG, "x and y of product %d must be non-NULL", i);
         if (!aligned16(xs[i]) || !aligned16(ys[i]))
             return fail(VBQ_ERR_ALIGN, "x and y of product %d must be 16-byte aligned", i);
-        if (waits && waits[i] != 0 && waits[i] != 1) return fail(VBQ_ERR_ARG, "waits[%d] must be 0 or 1", i);
+        if (waits && (waits[i] < 0 || waits[i] > 2)) return fail(VBQ_ERR_ARG, "waits[%d] must be 0, 1 or 2", i);
         vbq::ChainItem& it = items[(size_t)i];
         it.L = layouts[i]->view;
         it.x = xs[i];
         it.y = ys[i];
-        const bool w = !waits || waits[i];
-        it.wait_from = w ? last_wait : i;
-        if (w) last_wait = i;
+        const int w = waits ? waits[i] : 1;
+        if (w == 2 && i > 0) {          // the same dependencies as the product before
+            it.wait_from = items[(size_t)i - 1].wait_from;
+            it.wait_hi = items[(size_t)i - 1].wait_hi;
+        } else if (w != 0) {            // every product since the last waiting one (itself after the rest)
+            it.wait_from = last_wait;
+            it.wait_hi = i;
+            last_wait = i;
+        } else {
+            it.wait_from = it.wait_hi = i;
+        }
         it.rot = (int)(units_before % sms);
         units_before += it.L.units;
         seen_l[i] = layouts[i];

@@ -156,15 +156,16 @@ struct LayoutView {
 
 // One product of a chain (a sequence of batch-1 products run by one
 // persistent kernel, in order): its layout, activation vector and output.
-// Before product i touches x or y, products wait_from .. i - 1 must be
-// complete (wait_from == i: no wait). Block p takes the balanced share of
-// virtual block (p - rot) mod P, so products with fewer units than blocks
-// land on different blocks.
+// Before product i touches x or y, products wait_from .. wait_hi - 1 must be
+// complete (wait_from == wait_hi: no wait; wait_hi <= i). Block p takes the
+// balanced share of virtual block (p - rot) mod P, so products with fewer
+// units than blocks land on different blocks.
 struct ChainItem {
     LayoutView L;
     const uint16_t* x;
     float* y;
     int wait_from;
+    int wait_hi;
     int rot;
 };
 

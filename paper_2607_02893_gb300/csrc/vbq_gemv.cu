@@ -1195,10 +1195,10 @@ __global__ void __launch_bounds__(CH_THREADS, 1) gemv_chain_kernel(const ChainIt
             if (new_product) {
                 L = items[c.i].L;
                 x = items[c.i].x;
-                const int wf = items[c.i].wait_from;
+                const int wf = items[c.i].wait_from, wh = items[c.i].wait_hi;
                 // the first consumer warp waits for the product's dependencies; the
                 // table build's barrier holds the others until it is through
-                if (ct < 32 && !dead && wf < c.i && !chain_deps_ready(done, wf, c.i, target, lane)) {
+                if (ct < 32 && !dead && wf < wh && !chain_deps_ready(done, wf, wh, target, lane)) {
                     dead = true;
                     if (lane == 0) raise_abort(&T.abort);
                 }

@@ -4,8 +4,8 @@ the C ABI) with the CPU oracle.
 A chain runs its products in order in one launch, streaming weights across
 product boundaries. Every y_i must satisfy the product bound of vbq_gemv.
 Covered: products of one and several slabs, ragged row blocks, products with
-fewer units than blocks, every product waiting (the default) and mixed
-waits, repeated runs (the completion counts and split-K epochs carry over),
+fewer units than blocks, every product waiting (the default), mixed waits
+and products sharing their predecessor's dependencies, repeated runs (the completion counts and split-K epochs carry over),
 plain products on the same layouts between runs, graph capture, and the
 full-size stacks as bench.py runs them (sampled rows)."""
 
@@ -47,13 +47,19 @@ def _check(ms, ys):
         assert ok.all(), f"{m.n}x{m.k}: {int((~ok).sum())} outputs outside the bound"
 
 
-@pytest.mark.parametrize("waits", ["all", "mixed", "none"])
+WAITS = {"all": None, "mixed": [i % 2 for i in range(len(SHAPES))], "none": [0] * len(SHAPES),
+         # decode-step style: products that read the same input share their
+         # dependencies (waits 2), the next one waits for all of them
+         "grouped": [1, 2, 2, 1, 2, 1, 0, 2, 1]}
+
+
+@pytest.mark.parametrize("waits", sorted(WAITS))
 def test_chain_parity(waits):
     ms = _mats(0)
     lays = [vbq.vbq_pack(*m.device_args(DEV)) for m in ms]
     xs = [bits_to_i16(m.x_bits[0]).to(DEV) for m in ms]
     ys = [torch.full((m.n,), float("nan"), dtype=torch.float32, device=DEV) for m in ms]
-    w = None if waits == "all" else [i % 2 for i in range(len(ms))] if waits == "mixed" else [0] * len(ms)
+    w = WAITS[waits]
     chain = vbq.Chain(lays, xs, ys, w)
     for _ in range(3):
         for y in ys:
@@ -92,7 +98,7 @@ def test_chain_rejects_bad_arguments():
     ys = [torch.empty(m.n, dtype=torch.float32, device=DEV) for m in ms]
     for args, name in [((lays[:1] * 2, xs, ys), "VBQ_ERR_ARG"),          # a layout twice
                        ((lays, xs, [ys[0], ys[0]]), "VBQ_ERR_ARG"),       # an output twice
-                       ((lays, xs, ys, [1, 2]), "VBQ_ERR_ARG"),           # a bad wait flag
+                       ((lays, xs, ys, [1, 3]), "VBQ_ERR_ARG"),           # a bad wait flag
                        ((lays, [xs[0][1:], xs[1]], ys), "VBQ_ERR_ALIGN")]:
         with pytest.raises(vbq.VbqError) as e:
             vbq.Chain(*args)
