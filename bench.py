@@ -547,6 +547,33 @@ def companion_modes(args, work, layouts, xs, ys, step_bytes, copies, stream, dev
                               "layer-serial, same shapes as the headline")
         del rlays, rxs, rys
         torch.cuda.empty_cache()
+    # the ~1B layer stack, layer-serial as the headline, and a batch of 16 on
+    # the ~9B stack's 14336x4096 MLP shape
+    if name == "stack9b":
+        peak, _ = measured_peak()
+        w1 = synth.workload("stack1b", 1)
+        l1, x1, y1, nb1, _, cp1 = setup_stack(w1, 1, dev, min_bytes=3 * l2)
+        ms = time_graph(torch, stream,
+                        lambda: [vbq.vbq_gemv(l, x[0], y[0], stream=stream) for l, x, y in zip(l1, x1, y1)],
+                        steps, warm)
+        e1 = entry(ms, sum(nb1), cp1, len(l1), "workload stack1b (~1B stack, 155 GEMVs per token), layer-serial "
+                   "as the headline" + (f"; packed {cp1} times to exceed 3x L2" if cp1 > 1 else ""))
+        e1["frac"] = round(e1["value"] / peak, 4)
+        out["stack1b"] = e1
+        del l1, x1, y1
+        torch.cuda.empty_cache()
+        wb = synth.workload("matrix:14336:4096:main", 16)
+        lb, xb, yb, nbb, _, cpb = setup_stack(wb, 16, dev, min_bytes=3 * l2)
+        ms = time_graph(torch, stream,
+                        lambda: [vbq.vbq_gemm_small(l, x, y, 16, stream=stream) for l, x, y in zip(lb, xb, yb)],
+                        steps, warm)
+        eb = entry(ms, sum(nbb), cpb * 16, len(lb), "vbq_gemm_small, batch 16, on 14336x4096 (main width mix), "
+                   f"{cpb} packed copies cycled; value counts payload + scales + 16 x and 16 y per product")
+        eb["frac"] = round(eb["value"] / peak, 4)
+        eb["us_per_product"] = round(ms * 1e3 / len(lb), 2)
+        out["batch16_mlp"] = eb
+        del lb, xb, yb
+        torch.cuda.empty_cache()
     # dense BF16 reference: the same shapes, one copy per packed copy so the
     # weights stream from HBM too
     g = torch.Generator(device=dev)

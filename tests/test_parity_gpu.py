@@ -11,6 +11,7 @@ import torch
 import oracle
 import paper_2607_02893_gb300 as vbq
 import synth
+from synth import gen
 from vbq_cases import Matrix, bits_to_i16, scales_to_i16
 
 pytestmark = pytest.mark.gpu
@@ -276,3 +277,46 @@ def test_empty_output_dequant_is_noop():
     layout = _pack(m)
     vbq.vbq_dequant(layout)
     torch.cuda.synchronize()
+
+
+def _row_width_matrix(n, k, row_widths, seed):
+    """A matrix whose every row has one width (row_widths[r]); codes uniform,
+    scales and x as the generators draw them."""
+    spec = synth.MatrixSpec("rows", n, k, synth.DIST_MAIN, (95, n, k, seed))
+    inp = gen.matrix_inputs(spec, 3)
+    widths = np.repeat(np.asarray(row_widths, np.uint8)[:, None], k // 64, axis=1)
+    m = Matrix.__new__(Matrix)
+    m.n, m.k = n, k
+    m.widths, m.scales, m.x_bits, m.key = widths, inp["scales"], inp["x_bits"], inp["key"]
+    m.codes = gen.codes_torch(widths, inp["key"], k, device="cpu")
+    return m
+
+
+@pytest.mark.parametrize("case", ["tiers", "tiny_tiers", "interleaved", "one_row"])
+def test_row_uniform_units(case):
+    # rows of one width each: the fixed recipe's layout (§3.4), contiguous
+    # tiers (units whose rows all share one width, and units that straddle a
+    # tier boundary) and interleaved widths; all must match the oracle, at
+    # several slabs and with a ragged last row block
+    rng = np.random.default_rng(3)
+    if case == "tiers":
+        n, k = 1000, 64 * 37
+        rw = np.repeat(np.array([8, 4, 2, 1], np.uint8), [5, 15, 100, 880])
+    elif case == "tiny_tiers":          # tiers of 1-3 rows inside units
+        n, k = 777, 64 * 20
+        rw = np.repeat(np.array([8, 4, 2, 1, 2, 8], np.uint8), [1, 3, 2, 700, 70, 1])
+    elif case == "interleaved":
+        n, k = 900, 64 * 33
+        rw = rng.choice(np.array([1, 2, 4, 8], np.uint8), size=n)
+    else:
+        n, k = 1, 64 * 50
+        rw = np.array([4], np.uint8)
+    m = _row_width_matrix(n, k, rw, ["tiers", "tiny_tiers", "interleaved", "one_row"].index(case))
+    layout = _pack(m)
+    _assert_bound(_gemv(layout, m), m)
+    _assert_bound(_gemv(layout, m, 3), m, 3)
+    # the packed codes read back unchanged
+    codes = torch.empty((n, k), dtype=torch.uint8, device=DEV)
+    vbq.vbq_dequant(layout, codes, None, None, None)
+    torch.cuda.synchronize()
+    assert torch.equal(codes.cpu(), m.codes.cpu())
