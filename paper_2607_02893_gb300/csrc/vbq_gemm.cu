@@ -57,7 +57,9 @@ static_assert(STAGE_BYTES_B % 256 == 0, "stage alignment");
 template <int NB>
 struct __align__(16) TablesB {
     uint32_t afr[MAX_C][32][NB];         // A fragments (fp16x2) per column and lane: NB/4 per k-step
+    uint16_t xb[NB][MAX_C * GROUP];      // the slab's activations (BF16 bits), rows >= B zero
     float e2[MAX_C][16];                 // per column and batch row: 2^E (0 for absent rows)
+    float fx[MAX_C][16];                 // per column and batch row: 2^(24 - E), the A prescale
     float ys[Pipe<NB>::stages][NB][YS_STRIDE];     // row partials of each stage, per batch row
     unsigned long long full[Pipe<NB>::stages];     // blob landed
     unsigned long long empty[Pipe<NB>::stages];    // the unit's team is done
@@ -73,44 +75,81 @@ __device__ __forceinline__ void consumer_sync_b() {
 }
 
 __device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
                  : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
                  : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
 // The same with a zero accumulator (the first k-step of a tile).
 __device__ __forceinline__ void mma16816_z(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%10,%10};"
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%10,%10};"
                  : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
                  : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
 }
 
 __device__ __forceinline__ float bf16_bits(uint32_t b) { return __uint_as_float(b << 16); }
 
+// red_shared at a constant offset of OFF floats from addr.
+template <int OFF>
+__device__ __forceinline__ void red_shared_off(uint32_t addr, float v) {
+    asm volatile("red.shared.add.f32 [%0+%2], %1;" :: "r"(addr), "f"(v), "n"(OFF * 4) : "memory");
+}
+
 // Per slab: E and the A fragments of every column.
 // Consumer threads only (ct = 0 .. NCTB-1); starts and ends with a consumer barrier.
+// Kept out of line: inlined, it changed the register allocation of the tile
+// loops (measured up to 20% slower on all-4-bit matrices).
+// The slab's activations are first staged in shared memory with every thread's
+// 16-byte loads in flight at once (the table build is on the path of every
+// unit of the slab, so its latency counts, not its instructions).
 template <int NB>
-__device__ void build_tables_b(TablesB<NB>& T, const LayoutView& L, const uint16_t* __restrict__ X, int B, int s,
+__device__ __noinline__ void build_tables_b(TablesB<NB>& T, const LayoutView& L, const uint16_t* __restrict__ X, int B, int s,
                                int ct) {
+    constexpr int ROW_CHUNKS = MAX_C * GROUP / 8;                 // 16-byte chunks of one staged row
+    constexpr int PER = NB * ROW_CHUNKS / NCTB;
+    static_assert(PER * NCTB == NB * ROW_CHUNKS, "whole chunks per consumer thread");
     const int cols = min(L.C, L.G - s * L.C);
     const int64_t k0 = (int64_t)s * L.C * GROUP;
-    const int lane = ct & 31, cwarp = ct >> 5;
-    consumer_sync_b();                   // nobody still reads the old fragments
-    // one warp per (batch row, column): max |x| over the column's 64 values
-    for (int p = cwarp; p < 16 * cols; p += NCWB) {
-        const int b = p / cols, c = p - b * cols;
-        float m = 0.f;
-        if (b < B) {
-            const uint32_t two = __ldg(reinterpret_cast<const uint32_t*>(X + (int64_t)b * L.K + k0 + c * GROUP) + lane);
-            m = fmaxf(fabsf(__uint_as_float(two << 16)), fabsf(__uint_as_float(two & 0xFFFF0000u)));
+    consumer_sync_b();                   // nobody still reads the old tables
+    {
+        uint4 v[PER];
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const int q = ct + i * NCTB, b = q / ROW_CHUNKS, o = q - b * ROW_CHUNKS;
+            v[i] = make_uint4(0u, 0u, 0u, 0u);
+            if (b < B && o < cols * (GROUP / 8))
+                v[i] = __ldg(reinterpret_cast<const uint4*>(X + (int64_t)b * L.K + k0) + o);
         }
 #pragma unroll
-        for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-        if (lane == 0) {
-            // |x| < 2^(ex+1) with ex the exponent of m: x * 2^(24 - E) < 2^14 for E = ex + 11
-            const int ex = m > 0.f ? (int)((__float_as_uint(m) >> 23) & 0xFF) - 127 : -11;
-            const int E = ex + 11;
-            T.e2[c][b] = b < B ? ldexpf(1.f, E) : 0.f;
+        for (int i = 0; i < PER; ++i) *reinterpret_cast<uint4*>(&T.xb[0][0] + (size_t)(ct + i * NCTB) * 8) = v[i];
+    }
+    consumer_sync_b();
+    // two threads per (column, batch row < NB): the largest |x| of the column's 64
+    // values, as BF16 magnitude bits (ordered like the magnitudes), and from
+    // its exponent ex: E = ex + 11, so |x| * 2^(24 - E) < 2^14 fits fp16.
+    // E is held in [-100, 127] so that 2^E and 2^(24 - E) stay normal floats
+    // (a column of values below 2^-111 then keeps fewer fp16 bits, far below
+    // the accuracy bound's absolute term; values of 2^116 and more overflow).
+    {
+        const int pr = ct >> 1, c = pr / NB, b = pr % NB;         // c < 256 / NB, every column of the slab
+        uint32_t m = 0;
+        if (c < cols) {
+            const uint4* src = reinterpret_cast<const uint4*>(&T.xb[b][c * GROUP + 32 * (ct & 1)]);
+            uint32_t m2 = 0;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint4 w = src[q];
+                m2 = __vmaxu2(m2, __vmaxu2(w.x & 0x7FFF7FFFu, w.y & 0x7FFF7FFFu));
+                m2 = __vmaxu2(m2, __vmaxu2(w.z & 0x7FFF7FFFu, w.w & 0x7FFF7FFFu));
+            }
+            m = max(m2 & 0xFFFFu, m2 >> 16);
+        }
+        m = max(m, __shfl_xor_sync(0xffffffffu, m, 1));
+        const int ef = (int)(m >> 7);                             // biased exponent of max |x| (0: zero or subnormal)
+        const int E = min(max(ef - 127 + 11, -100), 127);
+        if (c < cols && (ct & 1) == 0) {
+            T.e2[c][b] = b < B ? __uint_as_float((uint32_t)(127 + E) << 23) : 0.f;
+            T.fx[c][b] = __uint_as_float((uint32_t)(127 + 24 - E) << 23);
         }
     }
     consumer_sync_b();
@@ -125,16 +164,10 @@ __device__ void build_tables_b(TablesB<NB>& T, const LayoutView& L, const uint16
         if (NB == 16) { s2 = r >> 2; h = (r >> 1) & 1; row = g + 8 * (r & 1); }
         else { s2 = r >> 1; h = r & 1; row = g; }
         const int rho = 2 * s2 + h;
-        uint32_t v = 0;
-        if (row < B) {
-            const float f = ldexpf(1.f, 24) / T.e2[c][row];
-            const uint16_t* xr = X + (int64_t)row * L.K + k0 + c * GROUP;
-            const float lo = bf16_bits(__ldg(xr + 16 * t + rho)) * f;
-            const float hi = bf16_bits(__ldg(xr + 16 * t + 8 + rho)) * f;
-            const __half2 hv = __floats2half2_rn(lo, hi);
-            v = *reinterpret_cast<const uint32_t*>(&hv);
-        }
-        T.afr[c][l][r] = v;
+        const float f = T.fx[c][row];
+        const uint16_t* xr = &T.xb[row][c * GROUP + 16 * t + rho];
+        const __half2 hv = __floats2half2_rn(bf16_bits(xr[0]) * f, bf16_bits(xr[8]) * f);
+        T.afr[c][l][r] = *reinterpret_cast<const uint32_t*>(&hv);
     }
     consumer_sync_b();
 }
@@ -196,36 +229,81 @@ __device__ __forceinline__ void to_levels(uint32_t (&b)[8]) {
 
 // Tiles k0 .. k1-1 of one (column, width W) bucket: items bs + 8k .. of the
 // bucket [bs, be); pay / scb / rwb: the width's payload, scales and row bytes.
+// One tile's operands: the lane's B fragments (levels, fp16) and where its
+// two output items go.
+struct TileIn {
+    uint32_t b[8];
+    float2 sab;                  // FP16 scales of items 2t, 2t+1
+    uint32_t aa, ab;             // their row partials (batch row g)
+    bool oa, ob;                 // the items exist
+};
+
+template <int W>
+__device__ __forceinline__ void tile_in(TileIn& ti, uint32_t pay, uint32_t scb, uint32_t rwb, int i0, int nv,
+                                        uint32_t ysg, int g, int t) {
+    const int ig = i0 + min(g, nv - 1);                              // lane's item (a valid one past the end)
+    if (W == 0) bfrag_1(lds_u32x2(pay + ig * 8), t, ti.b);
+    else if (W == 1) bfrag_2(lds_u32x4(pay + ig * 16), t, ti.b);
+    else if (W == 2) bfrag_4(lds_u32x2(pay + ig * 32 + 8 * t), ti.b);
+    else bfrag_8(lds_u32x4(pay + ig * 64 + 16 * t), ti.b);
+    // scales and rows of the lane's output items 2t, 2t+1; batch rows >= B add
+    // the zeros their A rows give
+    const int ia = i0 + min(2 * t, nv - 1), ib = i0 + min(2 * t + 1, nv - 1);
+    ti.sab = f2(half_bits(lds_u16(scb + 2 * ia)), half_bits(lds_u16(scb + 2 * ib)));
+    ti.aa = ysg + 4 * lds_u8(rwb + ia);
+    ti.ab = ysg + 4 * lds_u8(rwb + ib);
+    ti.oa = 2 * t < nv;
+    ti.ob = 2 * t + 1 < nv;
+    to_levels<W>(ti.b);
+}
+
+template <int NB>
+__device__ __forceinline__ void tile_mma(const uint32_t (&A4)[4][4], const TileIn& ti, float (&d)[4]) {
+    mma16816_z(d, A4[0], ti.b[0], ti.b[1]);
+#pragma unroll
+    for (int s2 = 1; s2 < 4; ++s2) mma16816(d, A4[s2], ti.b[2 * s2], ti.b[2 * s2 + 1]);
+}
+
+// D times the items' scales and the batch rows' 2^E (a power of two: the order
+// of the two products does not change the result), into the row partials.
+template <int NB>
+__device__ __forceinline__ void tile_out(const TileIn& ti, const float (&d)[4], float e2g, float e2g8) {
+    const float2 v01 = __fmul2_rn(__fmul2_rn(f2(d[0], d[1]), ti.sab), f2(e2g, e2g));
+    if (ti.oa) red_shared(ti.aa, v01.x);
+    if (ti.ob) red_shared(ti.ab, v01.y);
+    if (NB == 16) {
+        const float2 v23 = __fmul2_rn(__fmul2_rn(f2(d[2], d[3]), ti.sab), f2(e2g8, e2g8));
+        if (ti.oa) red_shared_off<8 * YS_STRIDE>(ti.aa, v23.x);
+        if (ti.ob) red_shared_off<8 * YS_STRIDE>(ti.ab, v23.y);
+    }
+}
+
+// Tiles k0 .. k1-1 of one (column, width W) bucket: items bs + 8k .. of the
+// bucket [bs, be); pay / scb / rwb: the width's payload, scales and row bytes.
+// Two tiles at a time, their loads, MMAs and stores interleaved (the MMA
+// chain of one tile alone leaves the warp waiting).
 template <int NB, int W>
 __device__ __forceinline__ void run_tiles(const uint32_t (&A4)[4][4], float e2g, float e2g8, uint32_t pay, uint32_t scb,
-                                          uint32_t rwb, int bs, int be, int k0, int k1, uint32_t ys, int B, int g,
-                                          int t) {
-    for (int k = k0; k < k1; ++k) {
-        const int i0 = bs + 8 * k, nv = min(8, be - i0);              // this tile's items: i0 .. i0 + nv - 1
-        const int ig = i0 + min(g, nv - 1);                          // lane's item (a valid one past the end)
-        uint32_t b[8];
-        if (W == 0) bfrag_1(lds_u32x2(pay + ig * 8), t, b);
-        else if (W == 1) bfrag_2(lds_u32x4(pay + ig * 16), t, b);
-        else if (W == 2) bfrag_4(lds_u32x2(pay + ig * 32 + 8 * t), b);
-        else bfrag_8(lds_u32x4(pay + ig * 64 + 16 * t), b);
-        // scales and rows of the lane's output items 2t, 2t+1 (loaded early)
-        const int ia = i0 + min(2 * t, nv - 1), ib = i0 + min(2 * t + 1, nv - 1);
-        const float sa = half_bits(lds_u16(scb + 2 * ia)), sb = half_bits(lds_u16(scb + 2 * ib));
-        const int ra = lds_u8(rwb + ia), rb = lds_u8(rwb + ib);
-        to_levels<W>(b);
-        float d[4];
-        mma16816_z(d, A4[0], b[0], b[1]);
-#pragma unroll
-        for (int s2 = 1; s2 < 4; ++s2) mma16816(d, A4[s2], b[2 * s2], b[2 * s2 + 1]);
-        // items 2t and 2t+1: scaled, added to the row partials of batch rows g and g + 8
-        if (g < B) {
-            if (2 * t < nv) red_shared(ys + 4 * (g * YS_STRIDE + ra), d[0] * (sa * e2g));
-            if (2 * t + 1 < nv) red_shared(ys + 4 * (g * YS_STRIDE + rb), d[1] * (sb * e2g));
-        }
-        if (NB == 16 && g + 8 < B) {
-            if (2 * t < nv) red_shared(ys + 4 * ((g + 8) * YS_STRIDE + ra), d[2] * (sa * e2g8));
-            if (2 * t + 1 < nv) red_shared(ys + 4 * ((g + 8) * YS_STRIDE + rb), d[3] * (sb * e2g8));
-        }
+                                          uint32_t rwb, int bs, int be, int k0, int k1, uint32_t ysg, int g, int t) {
+    int k = k0;
+    for (; k + 1 < k1; k += 2) {
+        const int i0 = bs + 8 * k, i1 = i0 + 8;                      // the first tile is whole
+        TileIn p, q;
+        tile_in<W>(p, pay, scb, rwb, i0, 8, ysg, g, t);
+        tile_in<W>(q, pay, scb, rwb, i1, min(8, be - i1), ysg, g, t);
+        float dp[4], dq[4];
+        tile_mma<NB>(A4, p, dp);
+        tile_mma<NB>(A4, q, dq);
+        tile_out<NB>(p, dp, e2g, e2g8);
+        tile_out<NB>(q, dq, e2g, e2g8);
+    }
+    if (k < k1) {
+        const int i0 = bs + 8 * k;
+        TileIn p;
+        tile_in<W>(p, pay, scb, rwb, i0, min(8, be - i0), ysg, g, t);
+        float dp[4];
+        tile_mma<NB>(A4, p, dp);
+        tile_out<NB>(p, dp, e2g, e2g8);
     }
 }
 
@@ -234,8 +312,9 @@ __device__ __forceinline__ void run_tiles(const uint32_t (&A4)[4][4], float e2g,
 // contiguous run of them, so its A fragments change only with the column.
 template <int NB>
 __device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sblob, int C, int cols, uint32_t ys,
-                                               int B, int wt, int tw, int lane) {
+                                               int wt, int tw, int lane) {
     const int g = lane >> 2, t = lane & 3;
+    const uint32_t ysg = ys + 4u * (uint32_t)(g * YS_STRIDE);     // the lane's batch row g
     const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
     const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
     // lane c (< cols) holds, per width, its bucket's first item and end, and tile counts
@@ -295,10 +374,10 @@ __device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sb
             const int k0 = max(ta - tile0, 0), k1 = min(tb - tile0, nt);
             if (k0 < k1) {
                 const int bs = __shfl_sync(0xffffffffu, start[w], c), be = __shfl_sync(0xffffffffu, end[w], c);
-                if (w == 0) run_tiles<NB, 0>(A4, e2g, e2g8, pay[0], scb[0], rwb[0], bs, be, k0, k1, ys, B, g, t);
-                else if (w == 1) run_tiles<NB, 1>(A4, e2g, e2g8, pay[1], scb[1], rwb[1], bs, be, k0, k1, ys, B, g, t);
-                else if (w == 2) run_tiles<NB, 2>(A4, e2g, e2g8, pay[2], scb[2], rwb[2], bs, be, k0, k1, ys, B, g, t);
-                else run_tiles<NB, 3>(A4, e2g, e2g8, pay[3], scb[3], rwb[3], bs, be, k0, k1, ys, B, g, t);
+                if (w == 0) run_tiles<NB, 0>(A4, e2g, e2g8, pay[0], scb[0], rwb[0], bs, be, k0, k1, ysg, g, t);
+                else if (w == 1) run_tiles<NB, 1>(A4, e2g, e2g8, pay[1], scb[1], rwb[1], bs, be, k0, k1, ysg, g, t);
+                else if (w == 2) run_tiles<NB, 2>(A4, e2g, e2g8, pay[2], scb[2], rwb[2], bs, be, k0, k1, ysg, g, t);
+                else run_tiles<NB, 3>(A4, e2g, e2g8, pay[3], scb[3], rwb[3], bs, be, k0, k1, ysg, g, t);
             }
             tile0 += nt;
         }
@@ -432,7 +511,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
                 consume_unit_b<NB>(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
-                                   smem_u32(&T.ys[st][0][0]), B, wt, tw, lane);
+                                   smem_u32(&T.ys[st][0][0]), wt, tw, lane);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty0 + 8 * st);
             }

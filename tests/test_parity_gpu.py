@@ -320,3 +320,22 @@ def test_row_uniform_units(case):
     vbq.vbq_dequant(layout, codes, None, None, None)
     torch.cuda.synchronize()
     assert torch.equal(codes.cpu(), m.codes.cpu())
+
+
+@pytest.mark.parametrize("batch", [1, 2, 5, 16])
+def test_activation_magnitudes(batch):
+    # group columns whose activations sit far from N(0, 1): 2^60, 2^-120
+    # (normal BF16), 2^-130 (BF16 subnormals), all zero, and mixed with
+    # ordinary ones; the bound of §6's product holds at every magnitude the
+    # kernels document (batch 1 and the tensor-core path scale per column)
+    m = Matrix(300, 64 * 24, seed_path=(94, batch, 0), batch=batch)
+    x = m.x().astype(np.float64)
+    col_scale = np.ones(24)
+    col_scale[[1, 7]] = 2.0 ** 60
+    col_scale[[2, 9, 15]] = 2.0 ** -120
+    col_scale[[3, 20]] = 2.0 ** -130
+    col_scale[[4]] = 0.0
+    x = x * np.repeat(col_scale, 64)[None, :]
+    m.x_bits = gen.f32_to_bf16_bits(x.astype(np.float32))
+    layout = _pack(m)
+    _assert_bound(_gemv(layout, m, batch), m, batch)
