@@ -56,7 +56,8 @@ static_assert(STAGE_BYTES_B % 256 == 0, "stage alignment");
 // Shared-memory tables of the batched kernel; NB = 8 or 16 A rows.
 template <int NB>
 struct __align__(16) TablesB {
-    uint32_t afr[MAX_C][32][NB];         // A fragments (fp16x2) per column and lane: NB/4 per k-step
+    uint32_t afr[MAX_C][NB / 4][32][4];  // A fragments (fp16x2) per column, register quad and lane: a warp's
+                                         // 16-byte loads of one quad read 512 contiguous bytes
     uint16_t xb[NB][MAX_C * GROUP];      // the slab's activations (BF16 bits), rows >= B zero
     float e2[MAX_C][16];                 // per column and batch row: 2^E (0 for absent rows)
     float fx[MAX_C][16];                 // per column and batch row: 2^(24 - E), the A prescale
@@ -167,7 +168,7 @@ __device__ __noinline__ void build_tables_b(TablesB<NB>& T, const LayoutView& L,
         const float f = T.fx[c][row];
         const uint16_t* xr = &T.xb[row][c * GROUP + 16 * t + rho];
         const __half2 hv = __floats2half2_rn(bf16_bits(xr[0]) * f, bf16_bits(xr[8]) * f);
-        T.afr[c][l][r] = *reinterpret_cast<const uint32_t*>(&hv);
+        T.afr[c][r >> 2][l][r & 3] = *reinterpret_cast<const uint32_t*>(&hv);
     }
     consumer_sync_b();
 }
@@ -351,10 +352,9 @@ __device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sb
         if (c_begin >= tb) break;
         uint32_t a[NB];
         {
-            const uint32_t* src = &T.afr[c][lane][0];
 #pragma unroll
             for (int r = 0; r < NB; r += 4) {
-                const uint4 v = *reinterpret_cast<const uint4*>(src + r);
+                const uint4 v = *reinterpret_cast<const uint4*>(&T.afr[c][r >> 2][lane][0]);
                 a[r] = v.x; a[r + 1] = v.y; a[r + 2] = v.z; a[r + 3] = v.w;
             }
         }
