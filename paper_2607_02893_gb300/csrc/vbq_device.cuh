@@ -153,11 +153,13 @@ __device__ __forceinline__ void red_release_gpu_add(uint32_t* p, uint32_t v) {
 // flags carry) is that count + 1. The additions need no reply, so no block
 // waits on them before it exits.
 constexpr int CALL_SHIFT = 20;
-__device__ __forceinline__ uint32_t call_epoch(const uint32_t* ctl) {
+__device__ __forceinline__ unsigned long long call_count_raw(const uint32_t* ctl) {
     unsigned long long c;
     asm volatile("ld.volatile.global.u64 %0, [%1];" : "=l"(c) : "l"(ctl) : "memory");
-    return (uint32_t)(c >> CALL_SHIFT) + 1u;
+    return c;
 }
+__device__ __forceinline__ uint32_t epoch_of(unsigned long long c) { return (uint32_t)(c >> CALL_SHIFT) + 1u; }
+__device__ __forceinline__ uint32_t call_epoch(const uint32_t* ctl) { return epoch_of(call_count_raw(ctl)); }
 __device__ __forceinline__ void call_done(uint32_t* ctl) {     // one thread per block, once per call
     const unsigned long long q = (1ull << CALL_SHIFT) / gridDim.x;
     const unsigned long long share = blockIdx.x == 0 ? (1ull << CALL_SHIFT) - q * (gridDim.x - 1) : q;

@@ -435,7 +435,9 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
         // ---- copier: split-K zeroing, then per unit: rows out, next copy in ----
         uint32_t epoch = 0;
         if (L.S > 1) {
-            epoch = call_epoch(L.ctl);
+            // the call count's load is in flight while the warp zeroes (the zeros
+            // do not depend on it; the flags do)
+            const unsigned long long count = call_count_raw(L.ctl);
             const int z_end = min(u_end, L.nrb);
             for (int u = u_begin; u < z_end; ++u) {
                 const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
@@ -445,6 +447,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
                 }
             }
             __syncwarp();
+            epoch = epoch_of(count);
             // release stores, one unit per lane in parallel: the warp's zeros
             // (ordered by __syncwarp) before each flag
             for (int u = u_begin + lane; u < z_end; u += 32) st_release_gpu(L.ctl + 2 + u, epoch);

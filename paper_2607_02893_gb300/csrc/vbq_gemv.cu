@@ -804,7 +804,9 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
         const int cp = warp;
         uint32_t epoch = 0;
         if (L.S > 1) {
-            epoch = call_epoch(L.ctl);
+            // the call count's load is in flight while copier 0 zeroes (the
+            // zeros do not depend on it; the flags it publishes do)
+            const unsigned long long count = call_count_raw(L.ctl);
             if (cp == 0) {
                 // zero y for the row blocks whose slab 0 this block owns (units
                 // u < nrb) and publish them
@@ -818,6 +820,10 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                     }
                 }
                 __syncwarp();
+            }
+            epoch = epoch_of(count);
+            if (cp == 0) {
+                const int z_end = min(u_end, L.nrb);
                 // release stores, one unit per lane in parallel: the warp's zeros
                 // (ordered by __syncwarp) before each flag
                 for (int u = u_begin + lane; u < z_end; u += 32) {
