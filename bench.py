@@ -19,13 +19,19 @@ same chain with the SwiGLU applied by the down projection as it stages its
 activations from the gate-up product's fp32 output, vbq_gemv_swiglu_in),
 `chain` (the headline's products as one vbq_chain_run: one
 persistent launch per step, every product still waiting for all earlier
-ones, weights streamed across product boundaries), `chain_fused` (the same for
+ones, weights streamed across product boundaries), `chain_by_input` (the same
+chain where a product that reads the same input as its predecessor, K and V
+after Q, up after gate, waits only for what that predecessor waits for),
+`chain_fused` (the same for
 the fused workload), `chain_independent` (the headline's products as one
 chain without waits: independent products in one persistent launch, the
 kernel's streaming upper bound), `grouped` (all of the headline's layouts as one
 vbq_gemv_group per step: independent products whose launches overlap, the
 streaming upper bound) and `cublas_bf16` (dense BF16 weights of the same
-shapes through torch.mv, i.e. cuBLAS, as a reference point), and, on the
+shapes through torch.mv, i.e. cuBLAS, as a reference point), `recipe` (the
+fixed recipe's widths on the same shapes, layer-serial), and for the ~9B stack
+`stack1b` (the ~1B stack, layer-serial as the headline) and `batch16_mlp`
+(vbq_gemm_small at batch 16 on the 14336x4096 MLP shape); and, on the
 workload's largest non-head matrix, `quantize` (vbq_quantize, the export-time
 quantiser) and `soft_quant` (vbq_soft_quant, the training-time soft forward).
 
@@ -35,13 +41,15 @@ Printed JSON line (rank 0):
   roofline      the GEMV kernel (the only kernel of the step): per-launch
                 algorithmic bytes / CUDA-event launch duration, against the
                 measured copy bandwidth; `traffic` is the DRAM bytes per launch
-                from the committed ncu launch list of this workload, reported
-                only while the kernel sources still hash to the captured ones.
+                modelled from committed one-launch ncu captures per matrix
+                shape (each launch's algorithmic bytes times its shape's
+                DRAM/algorithmic ratio), reported only while the kernel
+                sources still hash to the captured ones.
   e2e           the same metric with the step's activations copied in from
                 pinned host memory and the head's logits copied back, inside
                 the timed region.
   cpu_baseline  the CPU oracle (numpy fp64) on a bounded row sample of the
-                same stack.
+                same stack, one process per host core (and on one core).
 
 Workloads smaller than three times L2 are replicated (every copy packed
 separately) so that each step streams its weights from HBM; a step is then one
