@@ -28,6 +28,14 @@
  *     untouched. Nothing aborts or throws across the ABI. vbq_last_error()
  *     gives a human-readable detail of the calling thread's last error.
  *   - Device arrays must be 16-byte aligned (VBQ_ERR_ALIGN otherwise).
+ *   - The library keeps per-device state for the life of the process (each
+ *     kernel's shared-memory limit, set once per device; the device address
+ *     of vbq_gemv_static's array). A device reset (cudaDeviceReset), or
+ *     anything else that destroys and recreates the device's primary
+ *     context, invalidates that state: do not call the library on that
+ *     device afterwards in the same process.
+ *   - Activations (BF16) must be finite with magnitude below 2^64; larger
+ *     values may overflow inside the kernels' scaled arithmetic.
  */
 #ifndef VBQ_H
 #define VBQ_H
@@ -337,8 +345,7 @@ vbq_status_t vbq_chain_free(vbq_chain* chain);
  *
  * The array (32 KB) is a static device variable: every GPU that loads the
  * library holds it until the process exits. The first call on a device looks
- * up the array's address with that device current, so make the first call
- * on each device before any stream capture. Every call on a device shares the
+ * up the array's address with that device current. Every call on a device shares the
  * array and leaves its contents for the next call: each call adds the same
  * amount to the counter, whatever its grid, so the epoch its flags carry only
  * grows and flags left behind never match a later call. Calls that overlap on

@@ -5,6 +5,7 @@
 #pragma once
 
 #include <cstdint>
+#include <mutex>
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
 
@@ -12,6 +13,35 @@
 
 namespace vbq {
 namespace {
+
+// Host side, per kernel: its dynamic shared-memory limit is a per-device
+// property of the function, set once on every device it is launched on, and
+// the device's SM count sizes the persistent grids. Host threads may launch
+// concurrently, so this state is read and written under a lock.
+struct LaunchPrep {
+    static constexpr int MAX_DEVICES = 64;
+    std::mutex mu;
+    bool ready[MAX_DEVICES] = {};
+    int sms[MAX_DEVICES] = {};
+
+    template <class Kernel>
+    cudaError_t get(Kernel kernel, size_t smem, int* sms_out) {
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e != cudaSuccess) return e;
+        if (dev < 0 || dev >= MAX_DEVICES) return cudaErrorInvalidDevice;
+        std::lock_guard<std::mutex> lock(mu);
+        if (!ready[dev]) {
+            if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
+                cudaSuccess)
+                return e;
+            if ((e = cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+            ready[dev] = true;
+        }
+        *sms_out = sms[dev];
+        return cudaSuccess;
+    }
+};
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));

@@ -525,21 +525,13 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
     }
 }
 
-int g_sms_b = 0;
-
 template <int NB>
 cudaError_t launch_gemmb(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemmb_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)gemmb_smem<NB>());
-        if (e != cudaSuccess) return e;
-        int dev = 0;
-        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-        if ((e = cudaDeviceGetAttribute(&g_sms_b, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        attr_set = true;
-    }
-    const int grid = L.units < g_sms_b ? L.units : g_sms_b;
+    static LaunchPrep prep;
+    int sms = 0;
+    cudaError_t e = prep.get(gemmb_kernel<NB>, gemmb_smem<NB>(), &sms);
+    if (e != cudaSuccess) return e;
+    const int grid = L.units < sms ? L.units : sms;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(GB_THREADS);
@@ -550,7 +542,7 @@ cudaError_t launch_gemmb(const LayoutView& L, const uint16_t* X, float* Y, int B
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, gemmb_kernel<NB>, L, X, Y, B);
+    e = cudaLaunchKernelEx(&cfg, gemmb_kernel<NB>, L, X, Y, B);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

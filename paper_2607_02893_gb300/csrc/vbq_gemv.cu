@@ -1231,22 +1231,14 @@ __global__ void __launch_bounds__(CH_THREADS, 1) gemv_chain_kernel(const ChainIt
     }
 }
 
-int g_sms = 0;
-
 template <int NX, int MODE = MODE_PLAIN>
 cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s, int dep,
                          uint16_t* h = nullptr, const float* gu = nullptr) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemv1_kernel<NX, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)gemv1_smem<NX>());
-        if (e != cudaSuccess) return e;
-        int dev = 0;
-        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-        if ((e = cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        attr_set = true;
-    }
-    const int grid = L.units < g_sms ? L.units : g_sms;
+    static LaunchPrep prep;
+    int sms = 0;
+    cudaError_t e = prep.get(gemv1_kernel<NX, MODE>, gemv1_smem<NX>(), &sms);
+    if (e != cudaSuccess) return e;
+    const int grid = L.units < sms ? L.units : sms;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(G1_THREADS);
@@ -1257,7 +1249,7 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, gemv1_kernel<NX, MODE>, L, x, y, dep, h, gu);
+    e = cudaLaunchKernelEx(&cfg, gemv1_kernel<NX, MODE>, L, x, y, dep, h, gu);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -1272,13 +1264,10 @@ int device_sms(int* sms) {
 }
 
 cudaError_t launch_chain(const ChainItem* items, int count, uint32_t* cctl, int blocks, cudaStream_t s) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        const cudaError_t e = cudaFuncSetAttribute(gemv_chain_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                   (int)gemv1_smem<1>());
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static LaunchPrep prep;
+    int sms = 0;
+    const cudaError_t pe = prep.get(gemv_chain_kernel, gemv1_smem<1>(), &sms);
+    if (pe != cudaSuccess) return pe;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(blocks);
     cfg.blockDim = dim3(CH_THREADS);

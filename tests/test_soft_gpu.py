@@ -114,3 +114,39 @@ def test_soft_fullsize_sampled():
     ws, eb, hw = _run(w, lg, gb, 0.5)
     rows = sorted({0, n - 1, *(int(r) for r in np.random.default_rng(4).integers(0, n, size=6))})
     _check(w, lg, gb, 0.5, ws, eb, hw, rows)
+
+
+def test_soft_extreme_scales_and_near_ties():
+    # The codes come from |w| * fl(1/s) unless that product is within 2^-15 of
+    # a half-integer or s lies outside [2^-125, 2^125]; then from the IEEE
+    # quotient. Groups here: max|w| near 1e-37, so the 8-bit scale is a float32
+    # subnormal and the 4-bit one below 2^-125 (the weights themselves stay
+    # mostly normal: the bound is relative, and subnormal weights would lose
+    # relative precision in any float32 evaluation); scales so large that
+    # fl(1/s) would be subnormal; zeros of both signs; and quotients placed a
+    # few ulps and about 2^-14 from half-integers at each width (either
+    # decision there moves a weight by a whole step).
+    rng = gen.rng_for((70, 3, 0))
+    n, k = 6, 64 * 8
+    w = np.zeros((n, k), dtype=np.float32)
+    w[0] = (rng.standard_normal(k) * 3e-38).astype(np.float32)          # 8-bit scale subnormal
+    w[1] = (rng.standard_normal(k) * 1e35).astype(np.float32)          # sum|w| stays finite in float32
+    w[1, ::64] = np.float32(3.0e38)                                       # s = max|w| above 2^125
+    w[2, 1::2] = -0.0
+    w[2, ::2] = rng.standard_normal(k // 2).astype(np.float32)
+    for r, qmax in ((3, 1), (4, 7), (5, 127)):
+        s = np.float32(np.float32(1.0) / np.float32(qmax))                # max|w| = 1 in every group
+        j = (np.arange(k) % (2 * qmax)) - qmax
+        half = ((j + 0.5) * s).astype(np.float32)
+        ulps = rng.integers(-3, 4, size=k)
+        near = np.nextafter(half, np.where(ulps >= 0, np.float32(np.inf), np.float32(-np.inf)))
+        for _ in range(2):
+            near = np.where(np.abs(ulps) > 1, np.nextafter(near, np.where(ulps >= 0, np.inf, -np.inf)).astype(np.float32), near)
+        off = (half + np.float32(2.0 ** -14) * s * np.where(np.arange(k) % 3 == 0, 1, -1)).astype(np.float32)
+        row = np.where(np.arange(k) % 2 == 0, near, off).astype(np.float32)
+        row[::64] = np.float32(1.0)
+        w[r] = np.clip(row, -1.0, 1.0)
+    lg = rng.standard_normal((n, k // 64, 4)).astype(np.float32)
+    ws, eb, hw = _run(w, lg, None, 0.8)
+    _check(w, lg, None, 0.8, ws, eb, hw)
+    assert np.isfinite(ws).all()
