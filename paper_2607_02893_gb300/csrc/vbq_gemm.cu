@@ -42,9 +42,12 @@ constexpr int NCWB = 16;                 // consumer warps
 constexpr int NCTB = 32 * NCWB;
 constexpr int GB_THREADS = 32 * (NCWB + 1);
 constexpr int STAGE_BYTES_B = MAX_BLOB_BYTES;
-// Row partials of one batch row take RB + 1 floats, so the same row of eight
-// batch rows (the eight lane groups of an epilogue store) falls in eight banks.
-constexpr int YS_STRIDE = RB + 1;
+// Row partials of one batch row take RB + 4 floats: each batch row starts on
+// a 16-byte boundary (the flush moves 4 rows per lane), and the same row of
+// eight batch rows (the eight lane groups of an epilogue store) falls in
+// banks 4 apart.
+constexpr int YS_STRIDE = RB + 4;
+static_assert(YS_STRIDE % 4 == 0 && RB == 32 * 4, "a warp flushes a batch row's 128 partials 4 per lane");
 // Stages and consumer teams: with NB = 8 A rows the tables leave room for four
 // stages, so up to two teams of two stages each (a team's next blob lands
 // while it works on the current one); NB = 16 fits three stages and one team.
@@ -89,6 +92,12 @@ __device__ __forceinline__ void mma16816_z(float (&d)[4], const uint32_t (&a)[4]
 }
 
 __device__ __forceinline__ float bf16_bits(uint32_t b) { return __uint_as_float(b << 16); }
+
+// y[0..3] += v as one vector reduction (16-byte aligned address).
+__device__ __forceinline__ void red_global_v4(float* p, float4 v) {
+    asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" :: "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+                 : "memory");
+}
 
 // red_shared at a constant offset of OFF floats from addr.
 template <int OFF>
@@ -433,6 +442,9 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
 
     if (warp == 0) {
         // ---- copier: split-K zeroing, then per unit: rows out, next copy in ----
+        // (whole row blocks move 4 rows per lane when every batch row of Y
+        // starts on a 16-byte boundary)
+        const bool vec = (L.N & 3) == 0;
         uint32_t epoch = 0;
         if (L.S > 1) {
             // the call count's load is in flight while the warp zeroes (the zeros
@@ -441,9 +453,11 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             const int z_end = min(u_end, L.nrb);
             for (int u = u_begin; u < z_end; ++u) {
                 const int rows = min(RB, (int)(L.N - (int64_t)u * RB));
-                for (int q = lane; q < B * rows; q += 32) {
-                    const int b = q / rows, r = q - b * rows;
-                    Y[(int64_t)b * L.N + (int64_t)u * RB + r] = 0.f;
+                for (int b = 0; b < B; ++b) {
+                    float* yr = Y + (int64_t)b * L.N + (int64_t)u * RB;
+                    if (vec && rows == RB) reinterpret_cast<float4*>(yr)[lane] = make_float4(0.f, 0.f, 0.f, 0.f);
+                    else
+                        for (int r = lane; r < rows; r += 32) yr[r] = 0.f;
                 }
             }
             __syncwarp();
@@ -470,16 +484,21 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             if (!dead) {
                 const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
                 for (int b = 0; b < B; ++b) {
-                    float* ys = T.ys[st][b];
-                    float* yr = Y + (int64_t)b * L.N + (int64_t)rbw * RB;
+                    const uint32_t ysb = smem_u32(&T.ys[st][b][0]) + 16u * lane;
+                    float* yr = Y + (int64_t)b * L.N + (int64_t)rbw * RB + 4 * lane;
+                    const float4 v = lds_f32x4(ysb);
+                    sts_zero4(ysb);
+                    if (vec && rows == RB) {
+                        if (L.S == 1) *reinterpret_cast<float4*>(yr) = v;
+                        else red_global_v4(yr, v);
+                    } else {
+                        const float vv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-                    for (int q = 0; q < RB / 32; ++q) {
-                        const int r = lane + 32 * q;
-                        const float v = ys[r];
-                        ys[r] = 0.f;
-                        if (r < rows) {
-                            if (L.S == 1) yr[r] = v;
-                            else red_global(yr + r, v);
+                        for (int i = 0; i < 4; ++i) {
+                            if (4 * lane + i < rows) {
+                                if (L.S == 1) yr[i] = vv[i];
+                                else red_global(yr + i, vv[i]);
+                            }
                         }
                     }
                 }
