@@ -1371,7 +1371,7 @@ cudaError_t launch_selftest_timeout(unsigned long long limit_ns, cudaStream_t s)
 constexpr int GEMV1_MAX_B = 4;
 constexpr double COST_ONE[4] = {5.33, 7.02, 9.98, 14.0};
 constexpr double COST_PAIR[4] = {8.62, 11.8, 16.3, 27.5};
-constexpr double COST_MMA[4] = {23.9, 26.2, 26.7, 34.2};
+constexpr double COST_MMA[4] = {18.7, 20.3, 20.3, 27.0};
 
 bool tables_for_batch(const LayoutView& L, int B) {
     double tab = 0.0, mma = 0.0;
