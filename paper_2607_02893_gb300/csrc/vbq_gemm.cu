@@ -241,6 +241,16 @@ __device__ __forceinline__ void to_levels(uint32_t (&b)[8]) {
 // bucket [bs, be); pay / scb / rwb: the width's payload, scales and row bytes.
 // One tile's operands: the lane's B fragments (levels, fp16) and where its
 // two output items go.
+// The lane's 16 weights of item ig (positions 16t .. 16t + 15) as 8 fp16x2
+// registers of u * 2^-24 (register rho: weights 16t + rho and 16t + 8 + rho).
+template <int W>
+__device__ __forceinline__ void item_frag(uint32_t pay, int ig, int t, uint32_t (&b)[8]) {
+    if (W == 0) bfrag_1(lds_u32x2(pay + ig * 8), t, b);
+    else if (W == 1) bfrag_2(lds_u32x4(pay + ig * 16), t, b);
+    else if (W == 2) bfrag_4(lds_u32x2(pay + ig * 32 + 8 * t), b);
+    else bfrag_8(lds_u32x4(pay + ig * 64 + 16 * t), b);
+}
+
 struct TileIn {
     uint32_t b[8];
     float2 sab;                  // FP16 scales of items 2t, 2t+1
@@ -252,10 +262,7 @@ template <int W>
 __device__ __forceinline__ void tile_in(TileIn& ti, uint32_t pay, uint32_t scb, uint32_t rwb, int i0, int nv,
                                         uint32_t ysg, int g, int t) {
     const int ig = i0 + min(g, nv - 1);                              // lane's item (a valid one past the end)
-    if (W == 0) bfrag_1(lds_u32x2(pay + ig * 8), t, ti.b);
-    else if (W == 1) bfrag_2(lds_u32x4(pay + ig * 16), t, ti.b);
-    else if (W == 2) bfrag_4(lds_u32x2(pay + ig * 32 + 8 * t), ti.b);
-    else bfrag_8(lds_u32x4(pay + ig * 64 + 16 * t), ti.b);
+    item_frag<W>(pay, ig, t, ti.b);
     // scales and rows of the lane's output items 2t, 2t+1; batch rows >= B add
     // the zeros their A rows give
     const int ia = i0 + min(2 * t, nv - 1), ib = i0 + min(2 * t + 1, nv - 1);
@@ -314,6 +321,145 @@ __device__ __forceinline__ void run_tiles(const uint32_t (&A4)[4][4], float e2g,
         float dp[4];
         tile_mma<NB>(A4, p, dp);
         tile_out<NB>(p, dp, e2g, e2g8);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Up to 8 batch rows: the weights are the MMA's A operand (16 items of one
+// (column, width) bucket as its 16 rows) and the activations its B operand
+// (batch rows as its 8 columns). Lane (g, t) decodes items g and g + 8 of a
+// tile, and D gives it batch rows 2t and 2t + 1 of both, so a tile covers 16
+// items with 4 MMAs and 4 shared-memory additions per lane. The k order is the
+// one above: in k-step s, A register (row, h) holds weights 16t + 2s + h and
+// 16t + 8 + 2s + h, which is the activations' fragment register 2s + h of
+// the NB = 8 table, read here as B's two registers.
+// ---------------------------------------------------------------------------
+struct Tile16In {
+    uint32_t bg[8], bh[8];       // levels of the lane's items g and g + 8 (fp16x2, u * 2^-24)
+    float sg, sh;                // their FP16 scales
+    uint32_t ag, ah;             // their row partials of batch row 2t (2t + 1 is YS_STRIDE floats on)
+    bool og, oh;                 // the items exist
+};
+
+template <int W>
+__device__ __forceinline__ void tile16_in(Tile16In& ti, uint32_t pay, uint32_t scb, uint32_t rwb, int i0, int nv,
+                                          uint32_t yst, int g, int t) {
+    const int ig = i0 + min(g, nv - 1), ih = i0 + min(g + 8, nv - 1);    // valid items past the end
+    item_frag<W>(pay, ig, t, ti.bg);
+    item_frag<W>(pay, ih, t, ti.bh);
+    ti.sg = half_bits(lds_u16(scb + 2 * ig));
+    ti.sh = half_bits(lds_u16(scb + 2 * ih));
+    ti.ag = yst + 4 * lds_u8(rwb + ig);
+    ti.ah = yst + 4 * lds_u8(rwb + ih);
+    ti.og = g < nv;
+    ti.oh = g + 8 < nv;
+    to_levels<W>(ti.bg);
+    to_levels<W>(ti.bh);
+}
+
+__device__ __forceinline__ void tile16_mma(const uint32_t (&xb)[8], const Tile16In& ti, float (&d)[4]) {
+    {
+        const uint32_t a[4] = {ti.bg[0], ti.bh[0], ti.bg[1], ti.bh[1]};
+        mma16816_z(d, a, xb[0], xb[1]);
+    }
+#pragma unroll
+    for (int s2 = 1; s2 < 4; ++s2) {
+        const uint32_t a[4] = {ti.bg[2 * s2], ti.bh[2 * s2], ti.bg[2 * s2 + 1], ti.bh[2 * s2 + 1]};
+        mma16816(d, a, xb[2 * s2], xb[2 * s2 + 1]);
+    }
+}
+
+// D (items g, g + 8 x batch rows 2t, 2t + 1) times the items' scales and the
+// batch rows' 2^E, into the row partials.
+__device__ __forceinline__ void tile16_out(const Tile16In& ti, const float (&d)[4], float2 e2) {
+    const float2 vg = __fmul2_rn(__fmul2_rn(f2(d[0], d[1]), f2(ti.sg, ti.sg)), e2);
+    const float2 vh = __fmul2_rn(__fmul2_rn(f2(d[2], d[3]), f2(ti.sh, ti.sh)), e2);
+    if (ti.og) {
+        red_shared(ti.ag, vg.x);
+        red_shared_off<YS_STRIDE>(ti.ag, vg.y);
+    }
+    if (ti.oh) {
+        red_shared(ti.ah, vh.x);
+        red_shared_off<YS_STRIDE>(ti.ah, vh.y);
+    }
+}
+
+// Tiles k0 .. k1-1 (16 items each) of one (column, width W) bucket [bs, be).
+template <int W>
+__device__ __forceinline__ void run_tiles16(const uint32_t (&xb)[8], float2 e2, uint32_t pay, uint32_t scb, uint32_t rwb,
+                                            int bs, int be, int k0, int k1, uint32_t yst, int g, int t) {
+    for (int k = k0; k < k1; ++k) {
+        const int i0 = bs + 16 * k;
+        Tile16In ti;
+        tile16_in<W>(ti, pay, scb, rwb, i0, min(16, be - i0), yst, g, t);
+        float d[4];
+        tile16_mma(xb, ti, d);
+        tile16_out(ti, d, e2);
+    }
+}
+
+// One consumer warp's share of a unit at up to 8 batch rows: tiles of 16 items
+// of one (column, width) bucket, in (column, width) order; warp wt of a team
+// of tw warps takes a contiguous run of them.
+__device__ __forceinline__ void consume_unit_b16(const TablesB<8>& T, uint32_t sblob, int C, int cols, uint32_t ys,
+                                                 int wt, int tw, int lane) {
+    const int g = lane >> 2, t = lane & 3;
+    const uint32_t yst = ys + 4u * (uint32_t)(2 * t * YS_STRIDE);   // the lane's batch row 2t
+    const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
+    const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
+    int start[4], end[4], ntile[4], nt_col = 0;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        const int e = lane < cols ? (int)lds_u16(cc + 2 * (w * C + lane)) : 0;
+        int a = __shfl_up_sync(0xffffffffu, e, 1);
+        if (lane == 0) a = 0;
+        start[w] = a;
+        end[w] = e;
+        ntile[w] = lane < cols ? (e - a + 15) >> 4 : 0;
+        nt_col += ntile[w];
+    }
+    int incl = nt_col;                   // tiles of columns 0..lane
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+    }
+    const int total = __shfl_sync(0xffffffffu, incl, 31);
+    const int lg_tw = __popc(tw - 1);                  // tw is a power of two
+    const int ta = (total * wt) >> lg_tw, tb = (total * (wt + 1)) >> lg_tw;
+    if (ta >= tb) return;
+    const uint32_t pay[4] = {sblob + (h0.z & 0xFFFF) * 16, sblob + (h0.z >> 16) * 16, sblob + (h0.w & 0xFFFF) * 16,
+                             sblob + (h0.w >> 16) * 16};
+    const uint32_t scb[4] = {sblob + (h1.x & 0xFFFF) * 16, sblob + (h1.x >> 16) * 16, sblob + (h1.y & 0xFFFF) * 16,
+                             sblob + (h1.y >> 16) * 16};
+    const uint32_t rwb[4] = {sblob + (h1.z & 0xFFFF) * 16, sblob + (h1.z >> 16) * 16, sblob + (h1.w & 0xFFFF) * 16,
+                             sblob + (h1.w >> 16) * 16};
+    for (int c = __popc(__ballot_sync(0xffffffffu, incl <= ta)); c < cols; ++c) {
+        const int c_end = __shfl_sync(0xffffffffu, incl, c), c_begin = c_end - __shfl_sync(0xffffffffu, nt_col, c);
+        if (c_begin >= tb) break;
+        // the column's activation fragments (the NB = 8 table's 8 registers per lane)
+        uint32_t xb[8];
+        {
+            const uint4 v0 = *reinterpret_cast<const uint4*>(&T.afr[c][0][lane][0]);
+            const uint4 v1 = *reinterpret_cast<const uint4*>(&T.afr[c][1][lane][0]);
+            xb[0] = v0.x; xb[1] = v0.y; xb[2] = v0.z; xb[3] = v0.w;
+            xb[4] = v1.x; xb[5] = v1.y; xb[6] = v1.z; xb[7] = v1.w;
+        }
+        const float2 e2 = f2(T.e2[c][2 * t], T.e2[c][2 * t + 1]);
+        int tile0 = c_begin;
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            const int nt = __shfl_sync(0xffffffffu, ntile[w], c);
+            const int k0 = max(ta - tile0, 0), k1 = min(tb - tile0, nt);
+            if (k0 < k1) {
+                const int bs = __shfl_sync(0xffffffffu, start[w], c), be = __shfl_sync(0xffffffffu, end[w], c);
+                if (w == 0) run_tiles16<0>(xb, e2, pay[0], scb[0], rwb[0], bs, be, k0, k1, yst, g, t);
+                else if (w == 1) run_tiles16<1>(xb, e2, pay[1], scb[1], rwb[1], bs, be, k0, k1, yst, g, t);
+                else if (w == 2) run_tiles16<2>(xb, e2, pay[2], scb[2], rwb[2], bs, be, k0, k1, yst, g, t);
+                else run_tiles16<3>(xb, e2, pay[3], scb[3], rwb[3], bs, be, k0, k1, yst, g, t);
+            }
+            tile0 += nt;
+        }
     }
 }
 
@@ -532,8 +678,12 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             const uint32_t par = (uint32_t)(j / NST) & 1u;
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
-                consume_unit_b<NB>(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
-                                   smem_u32(&T.ys[st][0][0]), wt, tw, lane);
+                if constexpr (NB == 8)
+                    consume_unit_b16(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
+                                     smem_u32(&T.ys[st][0][0]), wt, tw, lane);
+                else
+                    consume_unit_b<NB>(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
+                                       smem_u32(&T.ys[st][0][0]), wt, tw, lane);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty0 + 8 * st);
             }
