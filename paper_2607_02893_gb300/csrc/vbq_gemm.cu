@@ -4,23 +4,24 @@
 // With B activation rows every decoded weight is used B times, so the product
 // is a dense contraction over dequantised tiles: here mma.sync m16n8k16 with
 // fp16 operands and fp32 accumulators. The operands are arranged so that the
-// packed bits go into B fragments with masks and byte permutes only:
+// packed bits go into A fragments with masks and byte permutes only:
 //
-//   A (16 x 16 per k-step) = activations: row b = batch row b (rows >= B are
-//       zero), pre-scaled per (batch row, group column) by 2^(24 - E), E set
-//       from the largest |x| of that column so every value stays in fp16
-//       range; built once per slab into shared memory, one fragment set per
-//       column and lane.
-//   B (16 x 8) = eight items (groups) of one width and one column: lane (g, t)
-//       holds item g's weights 16t + rho (low half) and 16t + 8 + rho (high
-//       half) of register rho. Any fixed assignment of the 64 weights of a
-//       group to the MMA's k positions gives the same sum, as long as A uses
-//       the same one; this one lets every width expand with one or two
-//       instructions per register into exact fp16 denormals u * 2^-24.
-//       One more packed fp16 subtraction (a fused 2u - 1 for one bit) turns
-//       u * 2^-24 into L(u) * 2^-24, exactly (every value is an integer times
-//       the smallest fp16 denormal, and fp16 arithmetic keeps denormals).
-//   D (16 x 8) = batch row x item: sum over the group of L(u) * x * 2^-E.
+//   A (16 x 16 per k-step) = sixteen items (groups) of one width and one
+//       column: lane (g, t) decodes items g and g + 8, holding each item's
+//       weights 16t + rho (low half) and 16t + 8 + rho (high half) in register
+//       rho. Any fixed assignment of the 64 weights of a group to the MMA's k
+//       positions gives the same sum, as long as B uses the same one; this
+//       one lets every width expand with one or two instructions per register
+//       into exact fp16 denormals u * 2^-24. One more packed fp16 subtraction
+//       (a fused 2u - 1 for one bit) turns u * 2^-24 into L(u) * 2^-24,
+//       exactly (every value is an integer times the smallest fp16 denormal,
+//       and fp16 arithmetic keeps denormals).
+//   B (16 x 8 per k-step) = activations: column n = batch row n (8 per MMA;
+//       two MMAs per k-step for more than 8 rows; rows >= B are zero),
+//       pre-scaled per (batch row, group column) by 2^(24 - E), E set from the
+//       largest |x| of that column so every value stays in fp16 range; built
+//       once per slab into shared memory, one fragment set per column and lane.
+//   D (16 x 8) = item x batch row: sum over the group of L(u) * x * 2^-E.
 //       Every product is exact, so a group whose codes all sit at the zero
 //       level gives exactly 0.
 //
@@ -59,11 +60,11 @@ static_assert(STAGE_BYTES_B % 256 == 0, "stage alignment");
 // Shared-memory tables of the batched kernel; NB = 8 or 16 A rows.
 template <int NB>
 struct __align__(16) TablesB {
-    uint32_t afr[MAX_C][NB / 4][32][4];  // A fragments (fp16x2) per column, register quad and lane: a warp's
+    uint32_t xfr[MAX_C][NB / 4][32][4];  // activation (B) fragments (fp16x2) per column, register quad and lane: a warp's
                                          // 16-byte loads of one quad read 512 contiguous bytes
     uint16_t xb[NB][MAX_C * GROUP];      // the slab's activations (BF16 bits), rows >= B zero
     float e2[MAX_C][16];                 // per column and batch row: 2^E (0 for absent rows)
-    float fx[MAX_C][16];                 // per column and batch row: 2^(24 - E), the A prescale
+    float fx[MAX_C][16];                 // per column and batch row: 2^(24 - E), the activations' prescale
     float ys[Pipe<NB>::stages][NB][YS_STRIDE];     // row partials of each stage, per batch row
     unsigned long long full[Pipe<NB>::stages];     // blob landed
     unsigned long long empty[Pipe<NB>::stages];    // the unit's team is done
@@ -105,7 +106,7 @@ __device__ __forceinline__ void red_shared_off(uint32_t addr, float v) {
     asm volatile("red.shared.add.f32 [%0+%2], %1;" :: "r"(addr), "f"(v), "n"(OFF * 4) : "memory");
 }
 
-// Per slab: E and the A fragments of every column.
+// Per slab: E and the activation fragments of every column.
 // Consumer threads only (ct = 0 .. NCTB-1); starts and ends with a consumer barrier.
 // Kept out of line: inlined, it changed the register allocation of the tile
 // loops (measured up to 20% slower on all-4-bit matrices).
@@ -163,10 +164,11 @@ __device__ __noinline__ void build_tables_b(TablesB<NB>& T, const LayoutView& L,
         }
     }
     consumer_sync_b();
-    // A fragments: register r of lane (g, t) for column c. NB = 16: k-step
-    // s = r / 4, q = r % 4 -> (row g + 8 (q & 1), half h = q >> 1); NB = 8:
-    // s = r / 2, h = r % 2, row g. Register pair (rho = 2s + h): weights
-    // 16t + rho (low) and 16t + 8 + rho (high) of the column.
+    // Activation fragments: register r of lane (g, t) for column c. NB = 16:
+    // k-step s = r / 4, q = r % 4 -> (batch row g + 8 (q & 1), half h = q >> 1);
+    // NB = 8: s = r / 2, h = r % 2, batch row g. Register pair (rho = 2s + h):
+    // the row's activations at weights 16t + rho (low) and 16t + 8 + rho (high)
+    // of the column.
     for (int p = ct; p < cols * 32 * NB; p += NCTB) {
         const int r = p % NB, l = (p / NB) & 31, c = p / (NB * 32);
         const int g = l >> 2, t = l & 3;
@@ -177,7 +179,7 @@ __device__ __noinline__ void build_tables_b(TablesB<NB>& T, const LayoutView& L,
         const float f = T.fx[c][row];
         const uint16_t* xr = &T.xb[row][c * GROUP + 16 * t + rho];
         const __half2 hv = __floats2half2_rn(bf16_bits(xr[0]) * f, bf16_bits(xr[8]) * f);
-        T.afr[c][r >> 2][l][r & 3] = *reinterpret_cast<const uint32_t*>(&hv);
+        T.xfr[c][r >> 2][l][r & 3] = *reinterpret_cast<const uint32_t*>(&hv);
     }
     consumer_sync_b();
 }
@@ -251,88 +253,17 @@ __device__ __forceinline__ void item_frag(uint32_t pay, int ig, int t, uint32_t 
     else bfrag_8(lds_u32x4(pay + ig * 64 + 16 * t), b);
 }
 
-struct TileIn {
-    uint32_t b[8];
-    float2 sab;                  // FP16 scales of items 2t, 2t+1
-    uint32_t aa, ab;             // their row partials (batch row g)
-    bool oa, ob;                 // the items exist
-};
-
-template <int W>
-__device__ __forceinline__ void tile_in(TileIn& ti, uint32_t pay, uint32_t scb, uint32_t rwb, int i0, int nv,
-                                        uint32_t ysg, int g, int t) {
-    const int ig = i0 + min(g, nv - 1);                              // lane's item (a valid one past the end)
-    item_frag<W>(pay, ig, t, ti.b);
-    // scales and rows of the lane's output items 2t, 2t+1; batch rows >= B add
-    // the zeros their A rows give
-    const int ia = i0 + min(2 * t, nv - 1), ib = i0 + min(2 * t + 1, nv - 1);
-    ti.sab = f2(half_bits(lds_u16(scb + 2 * ia)), half_bits(lds_u16(scb + 2 * ib)));
-    ti.aa = ysg + 4 * lds_u8(rwb + ia);
-    ti.ab = ysg + 4 * lds_u8(rwb + ib);
-    ti.oa = 2 * t < nv;
-    ti.ob = 2 * t + 1 < nv;
-    to_levels<W>(ti.b);
-}
-
-template <int NB>
-__device__ __forceinline__ void tile_mma(const uint32_t (&A4)[4][4], const TileIn& ti, float (&d)[4]) {
-    mma16816_z(d, A4[0], ti.b[0], ti.b[1]);
-#pragma unroll
-    for (int s2 = 1; s2 < 4; ++s2) mma16816(d, A4[s2], ti.b[2 * s2], ti.b[2 * s2 + 1]);
-}
-
-// D times the items' scales and the batch rows' 2^E (a power of two: the order
-// of the two products does not change the result), into the row partials.
-template <int NB>
-__device__ __forceinline__ void tile_out(const TileIn& ti, const float (&d)[4], float e2g, float e2g8) {
-    const float2 v01 = __fmul2_rn(__fmul2_rn(f2(d[0], d[1]), ti.sab), f2(e2g, e2g));
-    if (ti.oa) red_shared(ti.aa, v01.x);
-    if (ti.ob) red_shared(ti.ab, v01.y);
-    if (NB == 16) {
-        const float2 v23 = __fmul2_rn(__fmul2_rn(f2(d[2], d[3]), ti.sab), f2(e2g8, e2g8));
-        if (ti.oa) red_shared_off<8 * YS_STRIDE>(ti.aa, v23.x);
-        if (ti.ob) red_shared_off<8 * YS_STRIDE>(ti.ab, v23.y);
-    }
-}
-
-// Tiles k0 .. k1-1 of one (column, width W) bucket: items bs + 8k .. of the
-// bucket [bs, be); pay / scb / rwb: the width's payload, scales and row bytes.
-// Two tiles at a time, their loads, MMAs and stores interleaved (the MMA
-// chain of one tile alone leaves the warp waiting).
-template <int NB, int W>
-__device__ __forceinline__ void run_tiles(const uint32_t (&A4)[4][4], float e2g, float e2g8, uint32_t pay, uint32_t scb,
-                                          uint32_t rwb, int bs, int be, int k0, int k1, uint32_t ysg, int g, int t) {
-    int k = k0;
-    for (; k + 1 < k1; k += 2) {
-        const int i0 = bs + 8 * k, i1 = i0 + 8;                      // the first tile is whole
-        TileIn p, q;
-        tile_in<W>(p, pay, scb, rwb, i0, 8, ysg, g, t);
-        tile_in<W>(q, pay, scb, rwb, i1, min(8, be - i1), ysg, g, t);
-        float dp[4], dq[4];
-        tile_mma<NB>(A4, p, dp);
-        tile_mma<NB>(A4, q, dq);
-        tile_out<NB>(p, dp, e2g, e2g8);
-        tile_out<NB>(q, dq, e2g, e2g8);
-    }
-    if (k < k1) {
-        const int i0 = bs + 8 * k;
-        TileIn p;
-        tile_in<W>(p, pay, scb, rwb, i0, min(8, be - i0), ysg, g, t);
-        float dp[4];
-        tile_mma<NB>(A4, p, dp);
-        tile_out<NB>(p, dp, e2g, e2g8);
-    }
-}
-
 // ---------------------------------------------------------------------------
-// Up to 8 batch rows: the weights are the MMA's A operand (16 items of one
-// (column, width) bucket as its 16 rows) and the activations its B operand
-// (batch rows as its 8 columns). Lane (g, t) decodes items g and g + 8 of a
-// tile, and D gives it batch rows 2t and 2t + 1 of both, so a tile covers 16
-// items with 4 MMAs and 4 shared-memory additions per lane. The k order is the
-// one above: in k-step s, A register (row, h) holds weights 16t + 2s + h and
-// 16t + 8 + 2s + h, which is the activations' fragment register 2s + h of
-// the NB = 8 table, read here as B's two registers.
+// The weights as the MMA's A operand (16 items of one (column, width) bucket
+// as its 16 rows) and the activations as its B operand (8 batch rows as its
+// 8 columns; two such MMAs per k-step for NB = 16). Lane (g, t) decodes items
+// g and g + 8 of a tile, and D gives it batch rows 2t and 2t + 1 (and 8 + 2t,
+// 9 + 2t) of both, so a tile covers 16 items with 4 (8) MMAs and 4 (8)
+// shared-memory additions per lane. The k order is the one above: in k-step s,
+// A register (row, h) holds weights 16t + 2s + h and 16t + 8 + 2s + h, the
+// activation table's register for batch row g, k-step s and half h (NB = 8:
+// register 2s + h; NB = 16: 4s + 2h + n for the batch rows 8n + g), read here
+// as B's two registers.
 // ---------------------------------------------------------------------------
 struct Tile16In {
     uint32_t bg[8], bh[8];       // levels of the lane's items g and g + 8 (fp16x2, u * 2^-24)
@@ -357,23 +288,28 @@ __device__ __forceinline__ void tile16_in(Tile16In& ti, uint32_t pay, uint32_t s
     to_levels<W>(ti.bh);
 }
 
-__device__ __forceinline__ void tile16_mma(const uint32_t (&xb)[8], const Tile16In& ti, float (&d)[4]) {
-    {
-        const uint32_t a[4] = {ti.bg[0], ti.bh[0], ti.bg[1], ti.bh[1]};
-        mma16816_z(d, a, xb[0], xb[1]);
-    }
+template <int NB>
+__device__ __forceinline__ void tile16_mma(const uint32_t (&xb)[NB], const Tile16In& ti, float (&d)[NB / 2]) {
 #pragma unroll
-    for (int s2 = 1; s2 < 4; ++s2) {
+    for (int s2 = 0; s2 < 4; ++s2) {
         const uint32_t a[4] = {ti.bg[2 * s2], ti.bh[2 * s2], ti.bg[2 * s2 + 1], ti.bh[2 * s2 + 1]};
-        mma16816(d, a, xb[2 * s2], xb[2 * s2 + 1]);
+#pragma unroll
+        for (int n = 0; n < NB / 8; ++n) {
+            float (&dn)[4] = *reinterpret_cast<float (*)[4]>(&d[4 * n]);
+            const uint32_t b0 = NB == 8 ? xb[2 * s2] : xb[4 * s2 + n];
+            const uint32_t b1 = NB == 8 ? xb[2 * s2 + 1] : xb[4 * s2 + 2 + n];
+            if (s2 == 0) mma16816_z(dn, a, b0, b1);
+            else mma16816(dn, a, b0, b1);
+        }
     }
 }
 
-// D (items g, g + 8 x batch rows 2t, 2t + 1) times the items' scales and the
-// batch rows' 2^E, into the row partials.
-__device__ __forceinline__ void tile16_out(const Tile16In& ti, const float (&d)[4], float2 e2) {
-    const float2 vg = __fmul2_rn(__fmul2_rn(f2(d[0], d[1]), f2(ti.sg, ti.sg)), e2);
-    const float2 vh = __fmul2_rn(__fmul2_rn(f2(d[2], d[3]), f2(ti.sh, ti.sh)), e2);
+// D (items g, g + 8 x batch rows 2t, 2t + 1, and 8 + 2t, 9 + 2t) times the
+// items' scales and the batch rows' 2^E, into the row partials.
+template <int NB>
+__device__ __forceinline__ void tile16_out(const Tile16In& ti, const float (&d)[NB / 2], const float2 (&e2)[NB / 8]) {
+    const float2 vg = __fmul2_rn(__fmul2_rn(f2(d[0], d[1]), f2(ti.sg, ti.sg)), e2[0]);
+    const float2 vh = __fmul2_rn(__fmul2_rn(f2(d[2], d[3]), f2(ti.sh, ti.sh)), e2[0]);
     if (ti.og) {
         red_shared(ti.ag, vg.x);
         red_shared_off<YS_STRIDE>(ti.ag, vg.y);
@@ -382,26 +318,40 @@ __device__ __forceinline__ void tile16_out(const Tile16In& ti, const float (&d)[
         red_shared(ti.ah, vh.x);
         red_shared_off<YS_STRIDE>(ti.ah, vh.y);
     }
+    if constexpr (NB == 16) {
+        const float2 wg = __fmul2_rn(__fmul2_rn(f2(d[4], d[5]), f2(ti.sg, ti.sg)), e2[1]);
+        const float2 wh = __fmul2_rn(__fmul2_rn(f2(d[6], d[7]), f2(ti.sh, ti.sh)), e2[1]);
+        if (ti.og) {
+            red_shared_off<8 * YS_STRIDE>(ti.ag, wg.x);
+            red_shared_off<9 * YS_STRIDE>(ti.ag, wg.y);
+        }
+        if (ti.oh) {
+            red_shared_off<8 * YS_STRIDE>(ti.ah, wh.x);
+            red_shared_off<9 * YS_STRIDE>(ti.ah, wh.y);
+        }
+    }
 }
 
 // Tiles k0 .. k1-1 (16 items each) of one (column, width W) bucket [bs, be).
-template <int W>
-__device__ __forceinline__ void run_tiles16(const uint32_t (&xb)[8], float2 e2, uint32_t pay, uint32_t scb, uint32_t rwb,
-                                            int bs, int be, int k0, int k1, uint32_t yst, int g, int t) {
+template <int NB, int W>
+__device__ __forceinline__ void run_tiles16(const uint32_t (&xb)[NB], const float2 (&e2)[NB / 8], uint32_t pay,
+                                            uint32_t scb, uint32_t rwb, int bs, int be, int k0, int k1, uint32_t yst,
+                                            int g, int t) {
     for (int k = k0; k < k1; ++k) {
         const int i0 = bs + 16 * k;
         Tile16In ti;
         tile16_in<W>(ti, pay, scb, rwb, i0, min(16, be - i0), yst, g, t);
-        float d[4];
-        tile16_mma(xb, ti, d);
-        tile16_out(ti, d, e2);
+        float d[NB / 2];
+        tile16_mma<NB>(xb, ti, d);
+        tile16_out<NB>(ti, d, e2);
     }
 }
 
-// One consumer warp's share of a unit at up to 8 batch rows: tiles of 16 items
-// of one (column, width) bucket, in (column, width) order; warp wt of a team
-// of tw warps takes a contiguous run of them.
-__device__ __forceinline__ void consume_unit_b16(const TablesB<8>& T, uint32_t sblob, int C, int cols, uint32_t ys,
+// One consumer warp's share of a unit: tiles of 16 items of one (column,
+// width) bucket, in (column, width) order; warp wt of a team of tw warps takes
+// a contiguous run of them.
+template <int NB>
+__device__ __forceinline__ void consume_unit_b16(const TablesB<NB>& T, uint32_t sblob, int C, int cols, uint32_t ys,
                                                  int wt, int tw, int lane) {
     const int g = lane >> 2, t = lane & 3;
     const uint32_t yst = ys + 4u * (uint32_t)(2 * t * YS_STRIDE);   // the lane's batch row 2t
@@ -437,15 +387,16 @@ __device__ __forceinline__ void consume_unit_b16(const TablesB<8>& T, uint32_t s
     for (int c = __popc(__ballot_sync(0xffffffffu, incl <= ta)); c < cols; ++c) {
         const int c_end = __shfl_sync(0xffffffffu, incl, c), c_begin = c_end - __shfl_sync(0xffffffffu, nt_col, c);
         if (c_begin >= tb) break;
-        // the column's activation fragments (the NB = 8 table's 8 registers per lane)
-        uint32_t xb[8];
-        {
-            const uint4 v0 = *reinterpret_cast<const uint4*>(&T.afr[c][0][lane][0]);
-            const uint4 v1 = *reinterpret_cast<const uint4*>(&T.afr[c][1][lane][0]);
-            xb[0] = v0.x; xb[1] = v0.y; xb[2] = v0.z; xb[3] = v0.w;
-            xb[4] = v1.x; xb[5] = v1.y; xb[6] = v1.z; xb[7] = v1.w;
+        // the column's activation fragments (the table's NB registers per lane)
+        uint32_t xb[NB];
+#pragma unroll
+        for (int r = 0; r < NB; r += 4) {
+            const uint4 v = *reinterpret_cast<const uint4*>(&T.xfr[c][r >> 2][lane][0]);
+            xb[r] = v.x; xb[r + 1] = v.y; xb[r + 2] = v.z; xb[r + 3] = v.w;
         }
-        const float2 e2 = f2(T.e2[c][2 * t], T.e2[c][2 * t + 1]);
+        float2 e2[NB / 8];
+#pragma unroll
+        for (int n = 0; n < NB / 8; ++n) e2[n] = f2(T.e2[c][8 * n + 2 * t], T.e2[c][8 * n + 2 * t + 1]);
         int tile0 = c_begin;
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
@@ -453,86 +404,10 @@ __device__ __forceinline__ void consume_unit_b16(const TablesB<8>& T, uint32_t s
             const int k0 = max(ta - tile0, 0), k1 = min(tb - tile0, nt);
             if (k0 < k1) {
                 const int bs = __shfl_sync(0xffffffffu, start[w], c), be = __shfl_sync(0xffffffffu, end[w], c);
-                if (w == 0) run_tiles16<0>(xb, e2, pay[0], scb[0], rwb[0], bs, be, k0, k1, yst, g, t);
-                else if (w == 1) run_tiles16<1>(xb, e2, pay[1], scb[1], rwb[1], bs, be, k0, k1, yst, g, t);
-                else if (w == 2) run_tiles16<2>(xb, e2, pay[2], scb[2], rwb[2], bs, be, k0, k1, yst, g, t);
-                else run_tiles16<3>(xb, e2, pay[3], scb[3], rwb[3], bs, be, k0, k1, yst, g, t);
-            }
-            tile0 += nt;
-        }
-    }
-}
-
-// One consumer warp's share of a unit: tiles of 8 items of one (column, width)
-// bucket, in (column, width) order; warp wt of a team of tw warps takes a
-// contiguous run of them, so its A fragments change only with the column.
-template <int NB>
-__device__ __forceinline__ void consume_unit_b(const TablesB<NB>& T, uint32_t sblob, int C, int cols, uint32_t ys,
-                                               int wt, int tw, int lane) {
-    const int g = lane >> 2, t = lane & 3;
-    const uint32_t ysg = ys + 4u * (uint32_t)(g * YS_STRIDE);     // the lane's batch row g
-    const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
-    const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
-    // lane c (< cols) holds, per width, its bucket's first item and end, and tile counts
-    int start[4], end[4], ntile[4], nt_col = 0;
-#pragma unroll
-    for (int w = 0; w < 4; ++w) {
-        const int e = lane < cols ? (int)lds_u16(cc + 2 * (w * C + lane)) : 0;
-        int a = __shfl_up_sync(0xffffffffu, e, 1);
-        if (lane == 0) a = 0;
-        start[w] = a;
-        end[w] = e;
-        ntile[w] = lane < cols ? (e - a + 7) >> 3 : 0;
-        nt_col += ntile[w];
-    }
-    int incl = nt_col;                   // tiles of columns 0..lane
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int v = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += v;
-    }
-    const int total = __shfl_sync(0xffffffffu, incl, 31);
-    const int lg_tw = __popc(tw - 1);                  // tw is a power of two
-    const int ta = (total * wt) >> lg_tw, tb = (total * (wt + 1)) >> lg_tw;
-    if (ta >= tb) return;
-    const uint32_t pay[4] = {sblob + (h0.z & 0xFFFF) * 16, sblob + (h0.z >> 16) * 16, sblob + (h0.w & 0xFFFF) * 16,
-                             sblob + (h0.w >> 16) * 16};
-    const uint32_t scb[4] = {sblob + (h1.x & 0xFFFF) * 16, sblob + (h1.x >> 16) * 16, sblob + (h1.y & 0xFFFF) * 16,
-                             sblob + (h1.y >> 16) * 16};
-    const uint32_t rwb[4] = {sblob + (h1.z & 0xFFFF) * 16, sblob + (h1.z >> 16) * 16, sblob + (h1.w & 0xFFFF) * 16,
-                             sblob + (h1.w >> 16) * 16};
-    // walk the columns that hold tiles ta .. tb-1; per column, its four width buckets
-    for (int c = __popc(__ballot_sync(0xffffffffu, incl <= ta)); c < cols; ++c) {
-        const int c_end = __shfl_sync(0xffffffffu, incl, c), c_begin = c_end - __shfl_sync(0xffffffffu, nt_col, c);
-        if (c_begin >= tb) break;
-        uint32_t a[NB];
-        {
-#pragma unroll
-            for (int r = 0; r < NB; r += 4) {
-                const uint4 v = *reinterpret_cast<const uint4*>(&T.afr[c][r >> 2][lane][0]);
-                a[r] = v.x; a[r + 1] = v.y; a[r + 2] = v.z; a[r + 3] = v.w;
-            }
-        }
-        // the column's A operands, one register quad per k-step (NB = 8: rows
-        // 8..15 of the m16 shape are zero), set once for all of its tiles
-        uint32_t A4[4][4];
-#pragma unroll
-        for (int s2 = 0; s2 < 4; ++s2) {
-            if (NB == 16) { A4[s2][0] = a[4 * s2]; A4[s2][1] = a[4 * s2 + 1]; A4[s2][2] = a[4 * s2 + 2]; A4[s2][3] = a[4 * s2 + 3]; }
-            else { A4[s2][0] = a[2 * s2]; A4[s2][1] = 0u; A4[s2][2] = a[(2 * s2 + 1) % NB]; A4[s2][3] = 0u; }
-        }
-        const float e2g = T.e2[c][g], e2g8 = T.e2[c][g + 8];
-        int tile0 = c_begin;                            // global index of the bucket's first tile
-#pragma unroll
-        for (int w = 0; w < 4; ++w) {
-            const int nt = __shfl_sync(0xffffffffu, ntile[w], c);
-            const int k0 = max(ta - tile0, 0), k1 = min(tb - tile0, nt);
-            if (k0 < k1) {
-                const int bs = __shfl_sync(0xffffffffu, start[w], c), be = __shfl_sync(0xffffffffu, end[w], c);
-                if (w == 0) run_tiles<NB, 0>(A4, e2g, e2g8, pay[0], scb[0], rwb[0], bs, be, k0, k1, ysg, g, t);
-                else if (w == 1) run_tiles<NB, 1>(A4, e2g, e2g8, pay[1], scb[1], rwb[1], bs, be, k0, k1, ysg, g, t);
-                else if (w == 2) run_tiles<NB, 2>(A4, e2g, e2g8, pay[2], scb[2], rwb[2], bs, be, k0, k1, ysg, g, t);
-                else run_tiles<NB, 3>(A4, e2g, e2g8, pay[3], scb[3], rwb[3], bs, be, k0, k1, ysg, g, t);
+                if (w == 0) run_tiles16<NB, 0>(xb, e2, pay[0], scb[0], rwb[0], bs, be, k0, k1, yst, g, t);
+                else if (w == 1) run_tiles16<NB, 1>(xb, e2, pay[1], scb[1], rwb[1], bs, be, k0, k1, yst, g, t);
+                else if (w == 2) run_tiles16<NB, 2>(xb, e2, pay[2], scb[2], rwb[2], bs, be, k0, k1, yst, g, t);
+                else run_tiles16<NB, 3>(xb, e2, pay[3], scb[3], rwb[3], bs, be, k0, k1, yst, g, t);
             }
             tile0 += nt;
         }
@@ -678,12 +553,8 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             const uint32_t par = (uint32_t)(j / NST) & 1u;
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
-                if constexpr (NB == 8)
-                    consume_unit_b16(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
+                consume_unit_b16<NB>(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
                                      smem_u32(&T.ys[st][0][0]), wt, tw, lane);
-                else
-                    consume_unit_b<NB>(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
-                                       smem_u32(&T.ys[st][0][0]), wt, tw, lane);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty0 + 8 * st);
             }
