@@ -31,6 +31,12 @@ cudaError_t launch_quantize(const float* w, const uint8_t* widths, int64_t N, in
 cudaError_t launch_soft_quant(const float* w, const float* logits, const float* gumbel, float tau, int64_t N,
                               int64_t K, float* w_soft, float* exp_bits, uint8_t* hard, cudaStream_t s);
 
+// Batches of 2..GEMV1_MAX_B rows may run on the batch-1 table kernel, two
+// rows per launch; tables_for_batch (vbq_plan.cu) says whether the layout's
+// width mix makes that cheaper than the tensor-core kernel.
+constexpr int GEMV1_MAX_B = 4;
+bool tables_for_batch(const LayoutView& L, int B);
+
 // Products (vbq_gemv.cu). Y is B x N, overwritten (no zeroing needed).
 cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s);
 
