@@ -184,7 +184,7 @@ __device__ __noinline__ void build_tables_b(TablesB<NB>& T, const LayoutView& L,
     consumer_sync_b();
 }
 
-// B fragments (8 registers, u * 2^-24 per half) of lane t's 16 weights of one item.
+// Weight fragments (8 registers, u * 2^-24 per half) of lane t's 16 weights of one item.
 __device__ __forceinline__ void bfrag_1(uint2 w, int t, uint32_t (&b)[8]) {
     const uint32_t word = t < 2 ? w.x : w.y;
     const uint32_t lo = 2u * (t & 1), sel = lo | (lo << 4) | ((lo + 1) << 8) | ((lo + 1) << 12);
@@ -239,12 +239,9 @@ __device__ __forceinline__ void to_levels(uint32_t (&b)[8]) {
     }
 }
 
-// Tiles k0 .. k1-1 of one (column, width W) bucket: items bs + 8k .. of the
-// bucket [bs, be); pay / scb / rwb: the width's payload, scales and row bytes.
-// One tile's operands: the lane's B fragments (levels, fp16) and where its
-// two output items go.
 // The lane's 16 weights of item ig (positions 16t .. 16t + 15) as 8 fp16x2
-// registers of u * 2^-24 (register rho: weights 16t + rho and 16t + 8 + rho).
+// registers of u * 2^-24 (register rho: weights 16t + rho and 16t + 8 + rho);
+// pay is the item's width's payload.
 template <int W>
 __device__ __forceinline__ void item_frag(uint32_t pay, int ig, int t, uint32_t (&b)[8]) {
     if (W == 0) bfrag_1(lds_u32x2(pay + ig * 8), t, b);
@@ -332,7 +329,8 @@ __device__ __forceinline__ void tile16_out(const Tile16In& ti, const float (&d)[
     }
 }
 
-// Tiles k0 .. k1-1 (16 items each) of one (column, width W) bucket [bs, be).
+// Tiles k0 .. k1-1 (16 items each) of one (column, width W) bucket [bs, be);
+// pay / scb / rwb: the width's payload, scales and row bytes.
 template <int NB, int W>
 __device__ __forceinline__ void run_tiles16(const uint32_t (&xb)[NB], const float2 (&e2)[NB / 8], uint32_t pay,
                                             uint32_t scb, uint32_t rwb, int bs, int be, int k0, int k1, uint32_t yst,
