@@ -253,6 +253,10 @@ vbq_status_t vbq_pack(const uint8_t* codes, const uint8_t* bitwidths, const uint
     V.units = (int)units;
     for (int w = 0; w < 4; ++w) V.items[w] = (int64_t)real_items[w];
     V.max_blob16 = (int)max16;
+    V.single_w = -1;
+    for (int w = 0, present = 0; w < 4; ++w)
+        if (real_items[w]) V.single_w = present++ ? -2 : w;
+    if (V.single_w < 0) V.single_w = -1;
 
     if ((e = cudaMemsetAsync(L->base, 0, alloc_bytes, s)) != cudaSuccess) return bail(VBQ_ERR_CUDA, "memset", e);
     if ((e = cudaMemcpyAsync(base + off_at, blob_off.data(), blob_off.size() * 4, cudaMemcpyHostToDevice, s)) !=

@@ -152,6 +152,8 @@ struct LayoutView {
     int G, C, S, nrb, units;
     int max_blob16;             // largest blob, in 16-byte units
     int64_t items[4];           // groups per width index (1, 2, 4, 8 bits): host-side launch choices
+    int single_w;               // the width index of every group when the matrix has one width (the
+                                // fixed recipe's projections, §3.4), else -1
 };
 
 // One product of a chain (a sequence of batch-1 products run by one
@@ -185,6 +187,14 @@ __host__ __device__ inline int unit_cols(const LayoutView& L, int s) {
 
 // Sizes of the blob parts, given the item counts of a unit.
 __host__ __device__ inline uint32_t pad16(uint32_t bytes) { return (bytes + 15u) / 16u; }
+
+// A unit of a single-width matrix (every group at width index w, n = rows x
+// cols items in (column, row) order) starts with its header, payload and
+// scales; this is that prefix's length in 16-byte units (make_header lays the
+// blob out so).
+__host__ __device__ inline uint32_t single_prefix16(uint32_t n, int w) {
+    return (uint32_t)(sizeof(UnitHeader) / 16) + pad16(n * 8u * (1u << w)) + pad16(n * 2u);
+}
 
 __host__ __device__ inline UnitHeader make_header(const uint32_t n[4], int C, int ntask) {
     UnitHeader h{};

@@ -465,7 +465,8 @@ __device__ void build_tables(TablesT<NX>& T, const LayoutView& L, const uint16_t
 // redo its first item (always present) and store nothing, so every body is
 // branch-free.
 struct Task {
-    uint32_t pay, sc, row;      // shared addresses of the lane's (first) item: payload, scale, row byte
+    uint32_t pay, sc;           // shared addresses of the lane's (first) item: payload, scale
+    uint32_t r, r2;             // the rows of its item(s) within the unit
     bool on, on2;               // the lane's item (1 bit: its first and second item) is stored
     int c, c2;                  // their columns
 };
@@ -480,7 +481,8 @@ __device__ __forceinline__ Task task32(uint32_t sblob, uint4 d, int lane, int by
     t.c = (int)((d.x >> 16) & 15u) + __popc(d.y & le) + 2 * __popc(d.z & le);
     t.pay = sblob + (d.w & 0xFFFFu) + ii * bytes_per_item;
     t.sc = sblob + (d.x & 0xFFFFu) + 2 * ii;
-    t.row = sblob + (d.w >> 16) + ii;
+    t.r = lds_u8(sblob + (d.w >> 16) + ii);
+    t.r2 = t.r;
     t.on2 = false;
     t.c2 = t.c;
     return t;
@@ -501,7 +503,9 @@ __device__ __forceinline__ Task task64(uint32_t sblob, uint4 d, int lane) {
     t.c2 = t.c + (int)((d.z >> lane) & 1u);
     t.pay = sblob + (d.w & 0xFFFFu) + ii * 8;
     t.sc = sblob + (d.x & 0xFFFFu) + 2 * ii;
-    t.row = sblob + (d.w >> 16) + ii;
+    const uint32_t rows2 = lds_u16(sblob + (d.w >> 16) + ii);
+    t.r = rows2 & 0xffu;
+    t.r2 = rows2 >> 8;
     return t;
 }
 
@@ -516,7 +520,7 @@ __device__ __forceinline__ void body4(const TablesT<NX>& T, const Task& t, uint3
     const int h0 = (lane >> 2) & 1;
     const uint4 va = lds_u32x4(t.pay + h0 * 16), vb = lds_u32x4(t.pay + (h0 ^ 1) * 16);
     const uint32_t xa = smem_u32(T.x4s) + (c * 2 + h0) * XH * 4, xb = smem_u32(T.x4s) + (c * 2 + (h0 ^ 1)) * XH * 4;
-    const uint32_t sa = slot_addr(slots, lds_u8(t.row), c);
+    const uint32_t sa = slot_addr(slots, t.r, c);
     const float scl = half_bits(lds_u16(t.sc)) * 0x1p100f;
     if constexpr (NX == 1) {
         const float2 aa = dot4_half(va, xa), ab = dot4_half(vb, xb);
@@ -541,7 +545,7 @@ __device__ __forceinline__ void body8(const TablesT<NX>& T, const Task& t, uint3
     // quarter (k + (lane >> 1)) & 3 in step k: conflict-free 16-byte loads
     const int c = t.c;
     const int q0 = lane >> 1;
-    const uint32_t sa = slot_addr(slots, lds_u8(t.row), c);
+    const uint32_t sa = slot_addr(slots, t.r, c);
     const float scl = half_bits(lds_u16(t.sc));
     if constexpr (NX == 1) {
         float part = 0.f;
@@ -573,7 +577,7 @@ __device__ __forceinline__ void body2(const TablesT<NX>& T, const Task& t, uint3
     const int c = t.c;
     const uint4 pl = lds_u32x4(t.pay);
     const uint32_t tb = smem_u32(T.lut) + c * LUT_COL_BYTES;
-    const uint32_t sa = slot_addr(slots, lds_u8(t.row), c);
+    const uint32_t sa = slot_addr(slots, t.r, c);
     const float scl = half_bits(lds_u16(t.sc));
     // T0 / 2 + T1 - X / 2: for an all-zero-level group (b0 = 0, b1 = 1) T0 = -X
     // and T1 = X exactly, and X - X / 2 is exact, so the result is exactly 0
@@ -600,9 +604,8 @@ __device__ __forceinline__ void body1(const TablesT<NX>& T, const Task& t, uint3
     constexpr uint32_t SLOT_V = SLOT_FLOATS * 4;
     const int ca = t.c, cb = t.c2;
     const uint4 v = lds_u32x4(t.pay);
-    const uint32_t rows2 = lds_u16(t.row);
     const uint32_t sc2 = lds_u32(t.sc);
-    const uint32_t sb = slot_addr(slots, rows2 >> 8, cb), sa = slot_addr(slots, rows2 & 0xff, ca);
+    const uint32_t sb = slot_addr(slots, t.r2, cb), sa = slot_addr(slots, t.r, ca);
     const float scb = half_bits(sc2 >> 16), sca = half_bits(sc2);
     if constexpr (NX == 1) {
         float va[16], vb[16];
