@@ -647,6 +647,85 @@ __device__ __forceinline__ void consume_unit(const TablesT<NX>& T, uint32_t sblo
     }
 }
 
+// Single-width units (every group of the matrix at width index W, items in
+// (column, row) order, n = rows x cols of them): warp task k covers items
+// SPAN k .. SPAN k + SPAN - 1 (64 at one bit, two per lane; 32 otherwise),
+// and every item's column and row follow from its index, so the unit's task
+// table, row bytes and column ends are neither read nor copied.
+__device__ __forceinline__ void item_pos(int i, int rows, int& c, uint32_t& r) {
+    if (rows == RB) {
+        c = i >> 7;
+        r = (uint32_t)(i & (RB - 1));
+    } else {
+        c = i / rows;
+        r = (uint32_t)(i - c * rows);
+    }
+}
+static_assert(RB == 128, "item_pos shifts by log2(RB)");
+
+template <int NX, int W>
+__device__ __forceinline__ void consume_single_w(const TablesT<NX>& T, uint32_t sblob, uint32_t slots, int t0,
+                                                 int tstep, int lane, int rows) {
+    const int n = (int)lds_u16(sblob + offsetof(UnitHeader, n) + 2 * W);
+    const uint32_t pay = sblob + lds_u16(sblob + offsetof(UnitHeader, pay16) + 2 * W) * 16;
+    const uint32_t sc = sblob + lds_u16(sblob + offsetof(UnitHeader, sc16) + 2 * W) * 16;
+    constexpr int SPAN = W == 0 ? TASK_SPAN1 : TASK_SPAN, BPI = 8 << W;
+    const int ntask = (n + SPAN - 1) / SPAN;
+    for (int k = t0; k < ntask; k += tstep) {
+        const int cnt = min(SPAN, n - SPAN * k);
+        Task t;
+        if (W == 0) {
+            // lane l: items 2l and 2l + 1 (an even first item: one 16-byte payload
+            // load, one 4-byte scale load); past the end, the task's first pair
+            const int j = 2 * lane;
+            t.on = j < cnt;
+            t.on2 = j + 1 < cnt;
+            const int ii = SPAN * k + (t.on ? j : 0);
+            item_pos(ii, rows, t.c, t.r);
+            if (t.on2 && (int)t.r + 1 == rows) { t.c2 = t.c + 1; t.r2 = 0; }
+            else { t.c2 = t.c; t.r2 = t.on2 ? t.r + 1 : t.r; }
+            t.pay = pay + ii * 8;
+            t.sc = sc + 2 * ii;
+            body1<NX>(T, t, slots);
+        } else {
+            t.on = lane < cnt;
+            t.on2 = false;
+            const int ii = SPAN * k + (t.on ? lane : 0);
+            item_pos(ii, rows, t.c, t.r);
+            t.c2 = t.c;
+            t.r2 = t.r;
+            t.pay = pay + ii * BPI;
+            t.sc = sc + 2 * ii;
+            if (W == 1) body2<NX>(T, t, slots);
+            else if (W == 2) body4<NX>(T, t, slots, lane);
+            else body8<NX>(T, t, slots, lane);
+        }
+    }
+}
+
+template <int NX>
+__device__ __forceinline__ void consume_single(const TablesT<NX>& T, uint32_t sblob, uint32_t slots, int t0, int tstep,
+                                               int lane, int rows, int w) {
+    if (w == 0) consume_single_w<NX, 0>(T, sblob, slots, t0, tstep, lane, rows);
+    else if (w == 1) consume_single_w<NX, 1>(T, sblob, slots, t0, tstep, lane, rows);
+    else if (w == 2) consume_single_w<NX, 2>(T, sblob, slots, t0, tstep, lane, rows);
+    else consume_single_w<NX, 3>(T, sblob, slots, t0, tstep, lane, rows);
+}
+
+// A unit's copy: the whole blob, or for a single-width matrix (SW) only the
+// header, payload and scales at its start.
+template <bool SW>
+__device__ __forceinline__ void issue_unit_g1(const LayoutView& L, int u, uint32_t dst, uint32_t bar) {
+    if constexpr (SW) {
+        const int rb = u % L.nrb, sl = u / L.nrb;
+        const int rows = min(RB, (int)(L.N - (int64_t)rb * RB)), cols = min(L.C, L.G - sl * L.C);
+        bulk_load(dst, L.blobs + (int64_t)L.blob_off[u] * 16, single_prefix16((uint32_t)(rows * cols), L.single_w) * 16u,
+                  bar);
+    } else {
+        issue_unit(L, u, dst, bar);
+    }
+}
+
 // SwiGLU epilogue of a gate-up product whose rows alternate (row 2i the gate
 // of feature i, row 2i + 1 its up projection): h_i = silu(g_i) * u_i, rounded
 // to BF16 (to nearest even), the input format of the down projection.
@@ -728,8 +807,9 @@ __device__ __forceinline__ void team_flush(const TablesT<NX>& T, const LayoutVie
     }
 }
 
-// NX activation vectors x (NX x K, row-major) and outputs y (NX x N).
-template <int NX, int MODE>
+// NX activation vectors x (NX x K, row-major) and outputs y (NX x N). SW: the
+// matrix has a single width (L.single_w >= 0; see consume_single).
+template <int NX, int MODE, bool SW = false>
 __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, const uint16_t* __restrict__ x,
                                                               float* __restrict__ y, int dep,
                                                               uint16_t* __restrict__ h,
@@ -777,7 +857,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
     __syncthreads();
     if (tid == 0) {
         const int first = n_units < NSTAGE ? n_units : NSTAGE;
-        for (int j = 0; j < first; ++j) issue_unit(L, u_begin + j, stage0 + j * STAGE_BYTES, full0 + 8 * j);
+        for (int j = 0; j < first; ++j) issue_unit_g1<SW>(L, u_begin + j, stage0 + j * STAGE_BYTES, full0 + 8 * j);
     }
     // Weights never depend on earlier work in the stream, so the first copies
     // are in flight before this grid waits for its predecessor (programmatic
@@ -897,7 +977,7 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
                 }
                 __syncwarp();
                 if (j + NSTAGE < n_units && lane == 0)
-                    issue_unit(L, u_begin + j + NSTAGE, stage0 + st * STAGE_BYTES, full0 + 8 * st);
+                    issue_unit_g1<SW>(L, u_begin + j + NSTAGE, stage0 + st * STAGE_BYTES, full0 + 8 * st);
                 jdone = j;
                 if (MODE == MODE_SWIGLU_EPI && L.S > 1) {
                     // SwiGLU: count this unit's slab, then act on the previous unit's count
@@ -954,7 +1034,11 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             if (!dead) {
                 // tasks rotate over the team's warps from unit to unit, so no warp always draws the costly ones
                 const int t0 = (wt - (j >> lg_teams)) & (tw - 1);
-                consume_unit<NX>(T, stage0 + st * STAGE_BYTES, smem_u32(T.slots[st][0]), t0, tw, lane);
+                if constexpr (SW)
+                    consume_single<NX>(T, stage0 + st * STAGE_BYTES, smem_u32(T.slots[st][0]), t0, tw, lane,
+                                       min(RB, (int)(L.N - (int64_t)rbj * RB)), L.single_w);
+                else
+                    consume_unit<NX>(T, stage0 + st * STAGE_BYTES, smem_u32(T.slots[st][0]), t0, tw, lane);
                 __syncwarp();
                 if (!(COOP && j >= n_units - teams) && lane == 0) mbar_arrive(empty0 + 8 * st);
             }
@@ -1234,12 +1318,12 @@ __global__ void __launch_bounds__(CH_THREADS, 1) gemv_chain_kernel(const ChainIt
     }
 }
 
-template <int NX, int MODE = MODE_PLAIN>
+template <int NX, int MODE = MODE_PLAIN, bool SW = false>
 cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaStream_t s, int dep,
                          uint16_t* h = nullptr, const float* gu = nullptr) {
     static LaunchPrep prep;
     int sms = 0;
-    cudaError_t e = prep.get(gemv1_kernel<NX, MODE>, gemv1_smem<NX>(), &sms);
+    cudaError_t e = prep.get(gemv1_kernel<NX, MODE, SW>, gemv1_smem<NX>(), &sms);
     if (e != cudaSuccess) return e;
     const int grid = L.units < sms ? L.units : sms;
     cudaLaunchConfig_t cfg = {};
@@ -1252,7 +1336,7 @@ cudaError_t launch_gemv1(const LayoutView& L, const uint16_t* x, float* y, cudaS
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, gemv1_kernel<NX, MODE>, L, x, y, dep, h, gu);
+    e = cudaLaunchKernelEx(&cfg, gemv1_kernel<NX, MODE, SW>, L, x, y, dep, h, gu);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -1389,6 +1473,7 @@ cudaError_t launch_gemv(const LayoutView& L, const uint16_t* X, float* Y, int B,
         const cudaError_t e = launch_gemv1<2>(L, X + (int64_t)b * L.K, Y + (int64_t)b * L.N, s, DEP_BEFORE);
         if (e != cudaSuccess) return e;
     }
+    if (B == 1 && L.single_w >= 0) return launch_gemv1<1, MODE_PLAIN, true>(L, X, Y, s, DEP_BEFORE);
     if (b < B) return launch_gemv1<1>(L, X + (int64_t)b * L.K, Y + (int64_t)b * L.N, s, DEP_BEFORE);
     return cudaSuccess;
 }

@@ -107,6 +107,23 @@ def test_single_width(b):
     _assert_bound(_gemv(layout, m, 4), m, 4)
 
 
+@pytest.mark.parametrize("b", [1, 2, 4, 8])
+@pytest.mark.parametrize("shape", [(301, 64 * 37), (129, 832), (1, 64 * 20), (45, 64)], ids=lambda s: f"{s[0]}x{s[1]}")
+def test_single_width_ragged(b, shape):
+    # a matrix of one width takes the single-width path at batch 1 (tasks and
+    # row positions from item indices, only header, payload and scales
+    # copied): ragged last row blocks (odd row counts, so one-bit pairs cross
+    # columns), ragged last slabs, one row, one column; batch 3 runs the
+    # general path on the same layout
+    n, k = shape
+    d = tuple(1.0 if w == b else 0.0 for w in (1, 2, 4, 8))
+    m = Matrix(n, k, dist=d, seed_path=(92, b, n), batch=3)
+    layout = _pack(m)
+    for _ in range(2):
+        _assert_bound(_gemv(layout, m), m)
+    _assert_bound(_gemv(layout, m, 3), m, 3)
+
+
 def test_integer_all8_exact():
     rng = np.random.default_rng(5)
     n, k = 200, 1024
