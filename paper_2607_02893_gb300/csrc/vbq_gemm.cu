@@ -26,7 +26,10 @@
 //       level gives exactly 0.
 //
 // The epilogue scales D by the item's FP16 scale and 2^E and adds it to the
-// stage's row partials of that batch row. The kernel around it is the batch-1
+// stage's row partials of that batch row; for up to 8 batch rows on layouts
+// of 16-column units it stores it instead into the item's own (row, column)
+// slot, which the consumers sum per row after the unit (no shared-memory float
+// additions, which this GPU runs as compare-and-swap loops). The kernel around it is the batch-1
 // pipeline: one persistent block per SM, a copier warp streaming unit blobs by
 // TMA bulk copies into shared-memory stages and writing row partials to Y,
 // consumer warps in teams, two mbarriers per stage, split-K y zeroing by
@@ -49,31 +52,56 @@ constexpr int STAGE_BYTES_B = MAX_BLOB_BYTES;
 // banks 4 apart.
 constexpr int YS_STRIDE = RB + 4;
 static_assert(YS_STRIDE % 4 == 0 && RB == 32 * 4, "a warp flushes a batch row's 128 partials 4 per lane");
-// Stages and consumer teams: with NB = 8 A rows the tables leave room for four
-// stages, so up to two teams of two stages each (a team's next blob lands
-// while it works on the current one); NB = 16 fits three stages and one team.
-template <int NB> struct Pipe { static constexpr int stages = NB == 8 ? 4 : 3, max_teams = NB == 8 ? 2 : 1; };
-static_assert(Pipe<8>::stages % Pipe<8>::max_teams == 0 && Pipe<16>::stages % Pipe<16>::max_teams == 0,
+// Stages and consumer teams: three stages and one team. With NB = 8 the
+// epilogue stores into slots (one per row, group column and batch row: each
+// row of a unit has exactly one group per column) instead of adding into row
+// partials: shared-memory float additions are compare-and-swap loops on this
+// GPU (about 7 instructions and 2.6 times a plain store each, measured), and
+// they were a third of the kernel's time. The slots take 64 KB, the room of a
+// fourth stage; NB = 16 would need 128 KB and keeps the row partials.
+constexpr int SLOT_MIN_C = 16;          // the slot form for units of at least this many columns
+template <int NB, bool SL> struct Pipe {
+    static_assert(!SL || NB == 8, "slots for 8 batch rows only");
+    static constexpr int stages = NB == 8 && !SL ? 4 : 3, max_teams = NB == 8 && !SL ? 2 : 1;
+};
+static_assert(Pipe<8, false>::stages % Pipe<8, false>::max_teams == 0 && Pipe<16, false>::stages % Pipe<16, false>::max_teams == 0,
               "each team's units use stages no other team uses");
 static_assert(STAGE_BYTES_B % 256 == 0, "stage alignment");
 
-// Shared-memory tables of the batched kernel; NB = 8 or 16 A rows.
+// Shared-memory tables of the batched kernel; NB = 8 or 16 A rows: the
+// slab's activation tables, then the pipeline's state (SL: the slot form).
 template <int NB>
-struct __align__(16) TablesB {
+struct __align__(16) ActTables {
     uint32_t xfr[MAX_C][NB / 4][32][4];  // activation (B) fragments (fp16x2) per column, register quad and lane: a warp's
                                          // 16-byte loads of one quad read 512 contiguous bytes
     uint16_t xb[NB][MAX_C * GROUP];      // the slab's activations (BF16 bits), rows >= B zero
     float e2[MAX_C][16];                 // per column and batch row: 2^E (0 for absent rows)
     float fx[MAX_C][16];                 // per column and batch row: 2^(24 - E), the activations' prescale
-    float ys[Pipe<NB>::stages][NB][YS_STRIDE];     // row partials of each stage, per batch row
-    unsigned long long full[Pipe<NB>::stages];     // blob landed
-    unsigned long long empty[Pipe<NB>::stages];    // the unit's team is done
+};
+template <int NB, bool SL>
+struct __align__(16) TablesB : ActTables<NB> {
+    float ys[SL ? 1 : Pipe<NB, SL>::stages][NB][YS_STRIDE];   // row partials of each stage, per batch row
+    float sl[SL ? RB * MAX_C * 8 : 4];                        // SL: the current unit's slots (slot_index)
+    unsigned long long full[Pipe<NB, SL>::stages];            // blob landed
+    unsigned long long empty[Pipe<NB, SL>::stages];           // the unit's team is done
     int abort;
+    uint32_t sk_ok;                                           // SL: the copier's split-K flag check, passed on
 };
 
-template <int NB>
-constexpr size_t gemmb_smem() { return 256 + (size_t)Pipe<NB>::stages * STAGE_BYTES_B + sizeof(TablesB<NB>); }
-static_assert(gemmb_smem<16>() <= 227 * 1024 && gemmb_smem<8>() <= 227 * 1024, "one block per SM");
+template <int NB, bool SL>
+constexpr size_t gemmb_smem() { return 256 + (size_t)Pipe<NB, SL>::stages * STAGE_BYTES_B + sizeof(TablesB<NB, SL>); }
+static_assert(gemmb_smem<16, false>() <= 227 * 1024 && gemmb_smem<8, false>() <= 227 * 1024 &&
+              gemmb_smem<8, true>() <= 227 * 1024, "one block per SM");
+
+// Slot of row r, group column c and batch row b (NB = 8): a row's 16 columns x
+// 8 batch rows are 128 contiguous floats, its columns XOR-swizzled by the row's
+// low bits, so the 8-byte stores of four items of one column (a half-warp of
+// the epilogue) fall in four distinct groups of 8 banks when their rows differ
+// in their low two bits.
+__host__ __device__ constexpr uint32_t slot_index(uint32_t r, uint32_t c, uint32_t b) {
+    return r * (MAX_C * 8) + ((c ^ (r & (MAX_C - 1))) << 3) + b;
+}
+
 
 __device__ __forceinline__ void consumer_sync_b() {
     asm volatile("bar.sync 1, %0;" :: "n"(NCTB) : "memory");
@@ -114,7 +142,7 @@ __device__ __forceinline__ void red_shared_off(uint32_t addr, float v) {
 // 16-byte loads in flight at once (the table build is on the path of every
 // unit of the slab, so its latency counts, not its instructions).
 template <int NB>
-__device__ __noinline__ void build_tables_b(TablesB<NB>& T, const LayoutView& L, const uint16_t* __restrict__ X, int B, int s,
+__device__ __noinline__ void build_tables_b(ActTables<NB>& T, const LayoutView& L, const uint16_t* __restrict__ X, int B, int s,
                                int ct) {
     constexpr int ROW_CHUNKS = MAX_C * GROUP / 8;                 // 16-byte chunks of one staged row
     constexpr int PER = NB * ROW_CHUNKS / NCTB;
@@ -269,16 +297,22 @@ struct Tile16In {
     bool og, oh;                 // the items exist
 };
 
-template <int W>
+template <int W, bool SL>
 __device__ __forceinline__ void tile16_in(Tile16In& ti, uint32_t pay, uint32_t scb, uint32_t rwb, int i0, int nv,
-                                          uint32_t yst, int g, int t) {
+                                          uint32_t yst, int c, int g, int t) {
     const int ig = i0 + min(g, nv - 1), ih = i0 + min(g + 8, nv - 1);    // valid items past the end
     item_frag<W>(pay, ig, t, ti.bg);
     item_frag<W>(pay, ih, t, ti.bh);
     ti.sg = half_bits(lds_u16(scb + 2 * ig));
     ti.sh = half_bits(lds_u16(scb + 2 * ih));
-    ti.ag = yst + 4 * lds_u8(rwb + ig);
-    ti.ah = yst + 4 * lds_u8(rwb + ih);
+    const uint32_t rg = lds_u8(rwb + ig), rh = lds_u8(rwb + ih);
+    if constexpr (SL) {             // yst: the slots plus the lane's batch rows 2t, 2t + 1
+        ti.ag = yst + 4 * slot_index(rg, (uint32_t)c, 0);
+        ti.ah = yst + 4 * slot_index(rh, (uint32_t)c, 0);
+    } else {
+        ti.ag = yst + 4 * rg;
+        ti.ah = yst + 4 * rh;
+    }
     ti.og = g < nv;
     ti.oh = g + 8 < nv;
     to_levels<W>(ti.bg);
@@ -303,10 +337,15 @@ __device__ __forceinline__ void tile16_mma(const uint32_t (&xb)[NB], const Tile1
 
 // D (items g, g + 8 x batch rows 2t, 2t + 1, and 8 + 2t, 9 + 2t) times the
 // items' scales and the batch rows' 2^E, into the row partials.
-template <int NB>
+template <int NB, bool SL>
 __device__ __forceinline__ void tile16_out(const Tile16In& ti, const float (&d)[NB / 2], const float2 (&e2)[NB / 8]) {
     const float2 vg = __fmul2_rn(__fmul2_rn(f2(d[0], d[1]), f2(ti.sg, ti.sg)), e2[0]);
     const float2 vh = __fmul2_rn(__fmul2_rn(f2(d[2], d[3]), f2(ti.sh, ti.sh)), e2[0]);
+    if constexpr (SL) {                     // each (row, column) once per unit: stored, not added
+        if (ti.og) sts_f32x2(ti.ag, vg);
+        if (ti.oh) sts_f32x2(ti.ah, vh);
+        return;
+    }
     if (ti.og) {
         red_shared(ti.ag, vg.x);
         red_shared_off<YS_STRIDE>(ti.ag, vg.y);
@@ -331,28 +370,29 @@ __device__ __forceinline__ void tile16_out(const Tile16In& ti, const float (&d)[
 
 // Tiles k0 .. k1-1 (16 items each) of one (column, width W) bucket [bs, be);
 // pay / scb / rwb: the width's payload, scales and row bytes.
-template <int NB, int W>
+template <int NB, int W, bool SL>
 __device__ __forceinline__ void run_tiles16(const uint32_t (&xb)[NB], const float2 (&e2)[NB / 8], uint32_t pay,
                                             uint32_t scb, uint32_t rwb, int bs, int be, int k0, int k1, uint32_t yst,
-                                            int g, int t) {
+                                            int c, int g, int t) {
     for (int k = k0; k < k1; ++k) {
         const int i0 = bs + 16 * k;
         Tile16In ti;
-        tile16_in<W>(ti, pay, scb, rwb, i0, min(16, be - i0), yst, g, t);
+        tile16_in<W, SL>(ti, pay, scb, rwb, i0, min(16, be - i0), yst, c, g, t);
         float d[NB / 2];
         tile16_mma<NB>(xb, ti, d);
-        tile16_out<NB>(ti, d, e2);
+        tile16_out<NB, SL>(ti, d, e2);
     }
 }
 
 // One consumer warp's share of a unit: tiles of 16 items of one (column,
 // width) bucket, in (column, width) order; warp wt of a team of tw warps takes
 // a contiguous run of them.
-template <int NB>
-__device__ __forceinline__ void consume_unit_b16(const TablesB<NB>& T, uint32_t sblob, int C, int cols, uint32_t ys,
+template <int NB, bool SL>
+__device__ __forceinline__ void consume_unit_b16(const ActTables<NB>& T, uint32_t sblob, int C, int cols, uint32_t ys,
                                                  int wt, int tw, int lane) {
     const int g = lane >> 2, t = lane & 3;
-    const uint32_t yst = ys + 4u * (uint32_t)(2 * t * YS_STRIDE);   // the lane's batch row 2t
+    // the lane's batch row 2t: in the row partials, or (NB = 8) in the slots
+    const uint32_t yst = SL ? ys + 8u * (uint32_t)t : ys + 4u * (uint32_t)(2 * t * YS_STRIDE);
     const uint4 h0 = lds_u32x4(sblob), h1 = lds_u32x4(sblob + 16), h2 = lds_u32x4(sblob + 32);
     const uint32_t cc = sblob + (h2.x & 0xFFFF) * 16;
     int start[4], end[4], ntile[4], nt_col = 0;
@@ -402,23 +442,48 @@ __device__ __forceinline__ void consume_unit_b16(const TablesB<NB>& T, uint32_t 
             const int k0 = max(ta - tile0, 0), k1 = min(tb - tile0, nt);
             if (k0 < k1) {
                 const int bs = __shfl_sync(0xffffffffu, start[w], c), be = __shfl_sync(0xffffffffu, end[w], c);
-                if (w == 0) run_tiles16<NB, 0>(xb, e2, pay[0], scb[0], rwb[0], bs, be, k0, k1, yst, g, t);
-                else if (w == 1) run_tiles16<NB, 1>(xb, e2, pay[1], scb[1], rwb[1], bs, be, k0, k1, yst, g, t);
-                else if (w == 2) run_tiles16<NB, 2>(xb, e2, pay[2], scb[2], rwb[2], bs, be, k0, k1, yst, g, t);
-                else run_tiles16<NB, 3>(xb, e2, pay[3], scb[3], rwb[3], bs, be, k0, k1, yst, g, t);
+                if (w == 0) run_tiles16<NB, 0, SL>(xb, e2, pay[0], scb[0], rwb[0], bs, be, k0, k1, yst, c, g, t);
+                else if (w == 1) run_tiles16<NB, 1, SL>(xb, e2, pay[1], scb[1], rwb[1], bs, be, k0, k1, yst, c, g, t);
+                else if (w == 2) run_tiles16<NB, 2, SL>(xb, e2, pay[2], scb[2], rwb[2], bs, be, k0, k1, yst, c, g, t);
+                else run_tiles16<NB, 3, SL>(xb, e2, pay[3], scb[3], rwb[3], bs, be, k0, k1, yst, c, g, t);
             }
             tile0 += nt;
         }
     }
 }
 
-template <int NB>
+// NB = 8: the team's flush of a finished unit from its slots. Thread ct takes
+// row r = ct / 4 and batch rows 2q, 2q + 1 (q = ct % 4), sums the row's slots
+// over the unit's columns in column order, and stores the sums into Y (one
+// slab) or adds them (split-K). A half-warp's 8-byte loads (four rows, four
+// batch-row pairs) fall in distinct banks when the rows differ in their low
+// two bits, which four consecutive rows do.
+__device__ __forceinline__ void flush_slots(const float* sl, const LayoutView& L, float* __restrict__ Y, int B,
+                                            int rb, int cols, int ct) {
+    const int r = ct >> 2, q = ct & 3;
+    const int rows = min(RB, (int)(L.N - (int64_t)rb * RB));
+    if (r >= rows || 2 * q >= B) return;
+    const uint32_t row = smem_u32(sl) + 4u * ((uint32_t)r * (MAX_C * 8) + 2u * q);
+    const uint32_t sw = (uint32_t)r & (MAX_C - 1);            // column c sits at (c ^ sw) * 8 floats (slot_index)
+    float2 acc = lds_f32x2(row + ((0u ^ sw) << 5));
+    for (int c = 1; c < cols; ++c) acc = __fadd2_rn(acc, lds_f32x2(row + (((uint32_t)c ^ sw) << 5)));
+    float* y0 = Y + (int64_t)(2 * q) * L.N + (int64_t)rb * RB + r;
+    if (L.S == 1) {
+        y0[0] = acc.x;
+        if (2 * q + 1 < B) y0[L.N] = acc.y;
+    } else {
+        red_global(y0, acc.x);
+        if (2 * q + 1 < B) red_global(y0 + L.N, acc.y);
+    }
+}
+
+template <int NB, bool SL>
 __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, const uint16_t* __restrict__ X,
                                                               float* __restrict__ Y, int B) {
-    constexpr int NST = Pipe<NB>::stages;
+    constexpr int NST = Pipe<NB, SL>::stages;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     unsigned char* base = smem_raw + ((256u - (smem_u32(smem_raw) & 255u)) & 255u);
-    TablesB<NB>& T = *reinterpret_cast<TablesB<NB>*>(base + (size_t)NST * STAGE_BYTES_B);
+    TablesB<NB, SL>& T = *reinterpret_cast<TablesB<NB, SL>*>(base + (size_t)NST * STAGE_BYTES_B);
     const uint32_t stage0 = smem_u32(base);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int P = gridDim.x, p = blockIdx.x;
@@ -427,11 +492,11 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
     const int n_units = u_end - u_begin;
     if (n_units <= 0) return;
     const int s0 = u_begin / L.nrb, rb0 = u_begin - s0 * L.nrb;
-    // Teams as in the batch-1 kernel, at most Pipe<NB>::max_teams: unit j uses
+    // Teams as in the batch-1 kernel, at most Pipe<NB, SL>::max_teams: unit j uses
     // stage j % stages and goes to team j % teams, and teams divides stages, so
     // each team waits the phases of its own stages in order (a parity wait that
     // skipped a phase could match an older completed one).
-    const int lg_teams = Pipe<NB>::max_teams == 2 && n_units >= 4 ? 1 : 0;
+    const int lg_teams = Pipe<NB, SL>::max_teams == 2 && n_units >= 4 ? 1 : 0;
     const int teams = 1 << lg_teams, tw = NCWB >> lg_teams;
 
     const uint32_t full0 = smem_u32(&T.full[0]), empty0 = smem_u32(&T.empty[0]);
@@ -442,9 +507,11 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             mbar_init(empty0 + 8 * i, tw);
         }
         T.abort = 0;
+        T.sk_ok = 0;
         fence_barrier_init();
     }
-    for (int i = tid; i < NST * NB * YS_STRIDE; i += GB_THREADS) (&T.ys[0][0][0])[i] = 0.f;
+    if constexpr (!SL)
+        for (int i = tid; i < NST * NB * YS_STRIDE; i += GB_THREADS) (&T.ys[0][0][0])[i] = 0.f;
     __syncthreads();
     if (tid == 0) {
         const int first = n_units < NST ? n_units : NST;
@@ -491,6 +558,9 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             dead = true;
             if (lane == 0) raise_abort(&T.abort);
         }
+        // NB = 8: the consumers write Y; they add only after these flags (and
+        // this warp's own zeroing), passed on by a release
+        if (SL && L.S > 1 && lane == 0) red_release_cta_shared_add(smem_u32(&T.sk_ok), dead ? 0x10000u : 1u);
         int st = 0, rbw = rb0, issued = n_units < NST ? n_units : NST;
         uint32_t par = 0;
         for (int j = 0; j < n_units; ++j) {
@@ -500,7 +570,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
                 dead = true;
                 if (lane == 0) raise_abort(&T.abort);
             }
-            if (!dead) {
+            if (!dead && !SL) {
                 const int rows = min(RB, (int)(L.N - (int64_t)rbw * RB));
                 for (int b = 0; b < B; ++b) {
                     const uint32_t ysb = smem_u32(&T.ys[st][b][0]) + 16u * lane;
@@ -522,10 +592,10 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
                     }
                 }
                 __syncwarp();
-                if (j + NST < n_units) {
-                    if (lane == 0) issue_unit(L, u_begin + j + NST, stage0 + st * STAGE_BYTES_B, full0 + 8 * st);
-                    ++issued;
-                }
+            }
+            if (!dead && j + NST < n_units) {
+                if (lane == 0) issue_unit(L, u_begin + j + NST, stage0 + st * STAGE_BYTES_B, full0 + 8 * st);
+                ++issued;
             }
             if (++st == NST) { st = 0; par ^= 1; }
             if (++rbw == L.nrb) rbw = 0;
@@ -541,7 +611,7 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
         // ---- consumers: team `team` takes units j = team, team + teams, ... ----
         const int cw = warp - 1, ct = tid - 32, team = cw / tw, wt = cw - team * tw;
         const int s_last = (u_end - 1) / L.nrb;
-        bool dead = false;
+        bool dead = false, sk_seen = L.S == 1;
         int cur = s0, rbj = rb0 + team, sj = s0;
         while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
         build_tables_b(T, L, X, B, s0, ct);
@@ -549,12 +619,33 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
             while (cur < sj) build_tables_b(T, L, X, B, ++cur, ct);
             const int st = j % NST;                      // NST is a compile-time constant
             const uint32_t par = (uint32_t)(j / NST) & 1u;
+            const int cols = min(L.C, L.G - sj * L.C);
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
-                consume_unit_b16<NB>(T, stage0 + st * STAGE_BYTES_B, L.C, min(L.C, L.G - sj * L.C),
-                                     smem_u32(&T.ys[st][0][0]), wt, tw, lane);
+                consume_unit_b16<NB, SL>(T, stage0 + st * STAGE_BYTES_B, L.C, cols,
+                                         SL ? smem_u32(&T.sl[0]) : smem_u32(&T.ys[st][0][0]), wt, tw, lane);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty0 + 8 * st);
+            }
+            if constexpr (SL) {
+                // every warp's slot stores, then the unit's rows out; the next
+                // unit's stores only after every thread's reads
+                consumer_sync_b();
+                if (!sk_seen && !dead) {
+                    // split-K: after the copier's flag check (bounded wait)
+                    uint32_t g = 0;
+                    const unsigned long long w0 = global_ns();
+                    while ((g = ld_acquire_cta_shared(smem_u32(&T.sk_ok))) == 0u && !lds_volatile(abort_addr) &&
+                           global_ns() - w0 < WAIT_LIMIT_NS)
+                        __nanosleep(32);
+                    if (g != 1u) {
+                        dead = true;
+                        if (lane == 0) raise_abort(&T.abort);
+                    }
+                    sk_seen = true;
+                }
+                if (!dead) flush_slots(T.sl, L, Y, B, rbj, cols, ct);
+                consumer_sync_b();
             }
             rbj += teams;
             while (rbj >= L.nrb) { rbj -= L.nrb; ++sj; }
@@ -563,24 +654,24 @@ __global__ void __launch_bounds__(GB_THREADS, 1) gemmb_kernel(LayoutView L, cons
     }
 }
 
-template <int NB>
+template <int NB, bool SL>
 cudaError_t launch_gemmb(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
     static LaunchPrep prep;
     int sms = 0;
-    cudaError_t e = prep.get(gemmb_kernel<NB>, gemmb_smem<NB>(), &sms);
+    cudaError_t e = prep.get(gemmb_kernel<NB, SL>, gemmb_smem<NB, SL>(), &sms);
     if (e != cudaSuccess) return e;
     const int grid = L.units < sms ? L.units : sms;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(GB_THREADS);
-    cfg.dynamicSmemBytes = gemmb_smem<NB>();
+    cfg.dynamicSmemBytes = gemmb_smem<NB, SL>();
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, gemmb_kernel<NB>, L, X, Y, B);
+    e = cudaLaunchKernelEx(&cfg, gemmb_kernel<NB, SL>, L, X, Y, B);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -588,7 +679,10 @@ cudaError_t launch_gemmb(const LayoutView& L, const uint16_t* X, float* Y, int B
 }  // namespace
 
 cudaError_t launch_gemm_small(const LayoutView& L, const uint16_t* X, float* Y, int B, cudaStream_t s) {
-    return B <= 8 ? launch_gemmb<8>(L, X, Y, B, s) : launch_gemmb<16>(L, X, Y, B, s);
+    if (B > 8) return launch_gemmb<16, false>(L, X, Y, B, s);
+    // slots where units are wide: their per-unit flush and barriers are then
+    // small against a unit's tiles; narrow units keep two teams and four stages
+    return L.C >= SLOT_MIN_C ? launch_gemmb<8, true>(L, X, Y, B, s) : launch_gemmb<8, false>(L, X, Y, B, s);
 }
 
 cudaError_t read_device_status_gemm(uint32_t* status) {

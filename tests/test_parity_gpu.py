@@ -98,6 +98,22 @@ def test_gemm_small_parity(batch):
     _assert_bound(_gemv(layout, m, batch), m, batch)
 
 
+@pytest.mark.parametrize("shape,dist", [((4827, 64 * 40), "main"), ((4827, 64 * 40), "mlp0"), ((9700, 1024), "main")],
+                         ids=["4827x2560-main", "4827x2560-mlp0", "9700x1024-main"])
+@pytest.mark.parametrize("batch", [5, 8])
+def test_gemm_small_wide_units(shape, dist, batch):
+    # wide enough for 16-column units (at least 76 of them), so batches of 5..8
+    # take the per-slot epilogue: a ragged last row block (91 rows), a ragged
+    # last slab (8 of 16 columns) with split-K over three slabs, and one slab
+    # (no split-K); every output row against the oracle
+    n, k = shape
+    d = {"main": synth.DIST_MAIN, "mlp0": synth.DIST_MLP0}[dist]
+    m = Matrix(n, k, dist=d, seed_path=(91, n, batch), batch=batch)
+    layout = _pack(m)
+    for _ in range(2):
+        _assert_bound(_gemv(layout, m, batch), m, batch)
+
+
 @pytest.mark.parametrize("b", [1, 2, 4, 8])
 def test_single_width(b):
     d = tuple(1.0 if w == b else 0.0 for w in (1, 2, 4, 8))
