@@ -63,9 +63,6 @@ __device__ __forceinline__ void sts_f32_if(uint32_t addr, float v, bool pred) {
     asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %2, 0;\n\t@p st.shared.f32 [%0], %1;\n\t}"
                  :: "r"(addr), "f"(v), "r"((uint32_t)pred) : "memory");
 }
-__device__ __forceinline__ void sts_f32x2(uint32_t addr, float2 v) {
-    asm volatile("st.shared.v2.f32 [%0], {%1, %2};" :: "r"(addr), "f"(v.x), "f"(v.y) : "memory");
-}
 __device__ __forceinline__ void sts_zero4(uint32_t addr) {
     asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" :: "r"(addr), "r"(0u) : "memory");
 }

@@ -128,6 +128,10 @@ __device__ __forceinline__ void red_global_v4(float* p, float4 v) {
                  : "memory");
 }
 
+__device__ __forceinline__ void sts_f32x2(uint32_t addr, float2 v) {
+    asm volatile("st.shared.v2.f32 [%0], {%1, %2};" :: "r"(addr), "f"(v.x), "f"(v.y) : "memory");
+}
+
 // red_shared at a constant offset of OFF floats from addr.
 template <int OFF>
 __device__ __forceinline__ void red_shared_off(uint32_t addr, float v) {
