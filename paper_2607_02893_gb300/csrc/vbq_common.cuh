@@ -17,7 +17,8 @@
 //         column ends: uint16 cend[w][c] = index (within width w) of the
 //         first item after column c
 //         task table: one 16-byte TaskDesc per warp task of the batch-1
-//         product (see TaskDesc), 8-bit tasks first, then 4, 2 and 1 bit
+//         product (see TaskDesc), in the balanced order of balance_tasks
+//         (vbq_pack.cu)
 //     Blob u starts at byte 16 * blob_off[u] of the layout's blob area.
 //   * When a row has several slabs, the batch-1 product adds every slab's row
 //     partials into y with atomics, and y needs no zeroing by the caller: the

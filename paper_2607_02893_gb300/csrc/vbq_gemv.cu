@@ -628,9 +628,9 @@ __device__ __forceinline__ void body1(const TablesT<NX>& T, const Task& t, uint3
 }
 
 // One consumer warp's share of a unit (blob at shared address sblob): tasks
-// t0, t0 + tstep, ... of the unit's task table (8-bit tasks first, costliest
-// first). Each group's result goes to its slot in the stage's slot array at
-// shared address slots.
+// t0, t0 + tstep, ... of the unit's task table (written at pack time in an
+// order that balances the warps of this deal). Each group's result goes to its
+// slot in the stage's slot array at shared address slots.
 template <int NX>
 __device__ __forceinline__ void consume_unit(const TablesT<NX>& T, uint32_t sblob, uint32_t slots, int t0, int tstep,
                                              int lane) {
@@ -1032,8 +1032,9 @@ __global__ void __launch_bounds__(G1_THREADS, 1) gemv1_kernel(LayoutView L, cons
             const uint32_t par = (uint32_t)(j / NSTAGE) & 1u;
             if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
             if (!dead) {
-                // tasks rotate over the team's warps from unit to unit, so no warp always draws the costly ones
-                const int t0 = (wt - (j >> lg_teams)) & (tw - 1);
+                // the deal rotates by 5 warps from unit to unit (coprime with tw), so a
+                // warp's bins differ from unit to unit
+                const int t0 = (wt - 5 * (j >> lg_teams)) & (tw - 1);
                 if constexpr (SW)
                     consume_single<NX>(T, stage0 + st * STAGE_BYTES, smem_u32(T.slots[st][0]), t0, tw, lane,
                                        min(RB, (int)(L.N - (int64_t)rbj * RB)), L.single_w);
@@ -1307,8 +1308,8 @@ __global__ void __launch_bounds__(CH_THREADS, 1) gemv_chain_kernel(const ChainIt
                 const uint32_t par = (uint32_t)(j / NSTAGE) & 1u;
                 if (!dead && !warp_wait(full0 + 8 * st, par, abort_addr)) { dead = true; if (lane == 0) raise_abort(&T.abort); }
                 if (!dead) {
-                    // tasks rotate over the warps from unit to unit
-                    const int t0 = (wt - j) & (TW - 1);
+                    // the deal rotates by 5 warps from unit to unit
+                    const int t0 = (wt - 5 * j) & (TW - 1);
                     consume_unit<1>(T, stage0 + st * STAGE_BYTES, smem_u32(T.slots[st][0]), t0, TW, lane);
                     __syncwarp();
                     if (lane == 0) mbar_arrive(empty0 + 8 * st);

@@ -71,6 +71,42 @@ __global__ void __launch_bounds__(RB) count_kernel(const uint8_t* __restrict__ w
 // width (rows in increasing order) and written as the next item of that
 // width: payload, scale and row byte. Also writes the header (prepared on the
 // host) and the per-column counts.
+// The batch-1 kernel deals a unit's task k to warp (k + rotation) mod tw of its
+// team (tw = 16 or 8) and a block's warps meet at the end of its last unit, so
+// the table is written in an order that balances those warps: tasks by
+// decreasing cost, each to the least-loaded of 16 bins that still has a
+// position (bin b holds positions b, b + 16, ...; the first nt % 16 bins one
+// more than the rest, so the positions are exactly 0 .. nt - 1; bins b and
+// b + 8 together are a warp's share when tw = 8). The costs are the batch-1
+// kernel's measured time per group and width (COST_ONE in vbq_plan.cu: 5.33,
+// 7.02, 9.98, 14.0 units for 1, 2, 4, 8 bits) times a task's items: a task
+// costs its full span even when shorter, since idle lanes repeat its first
+// item. The order does not change any result: every group has its own slot.
+__device__ void balance_tasks(TaskDesc* t, int nt) {
+    if (nt <= 1 || nt > MAX_UNIT_TASKS) return;
+    constexpr int BINS = 16;
+    constexpr uint32_t cost_w[4] = {341, 225, 319, 448};     // 64 x 5.33, 32 x 7.02, 32 x 9.98, 32 x 14.0
+    constexpr int by_cost[4] = {3, 0, 2, 1};                  // 8, 1, 4, 2 bits
+    TaskDesc in[MAX_UNIT_TASKS];
+    for (int k = 0; k < nt; ++k) in[k] = t[k];
+    uint32_t load[BINS];
+    int cnt[BINS];
+    for (int b = 0; b < BINS; ++b) { load[b] = 0; cnt[b] = 0; }
+    const int base = nt / BINS, extra = nt % BINS;
+    for (int oi = 0; oi < 4; ++oi) {
+        const uint32_t w = (uint32_t)by_cost[oi];
+        for (int k = 0; k < nt; ++k) {
+            if (((in[k].x >> 26) & 3u) != w) continue;
+            int best = -1;
+            for (int b = 0; b < BINS; ++b)
+                if (cnt[b] < base + (b < extra ? 1 : 0) && (best < 0 || load[b] < load[best])) best = b;
+            t[best + BINS * cnt[best]] = in[k];
+            load[best] += cost_w[w];
+            ++cnt[best];
+        }
+    }
+}
+
 __global__ void __launch_bounds__(RB) scatter_kernel(const uint8_t* __restrict__ codes,
                                                      const uint8_t* __restrict__ widths,
                                                      const uint16_t* __restrict__ scales,
@@ -131,8 +167,12 @@ __global__ void __launch_bounds__(RB) scatter_kernel(const uint8_t* __restrict__
         __syncthreads();
     }
     // the batch-1 product's warp tasks (the count was planned on the host from
-    // the same column ends)
-    if (threadIdx.x == 0) unit_tasks(ce_s, cols, &h, reinterpret_cast<TaskDesc*>(blob + h.task16 * 16));
+    // the same column ends), in the dealing's balanced order
+    if (threadIdx.x == 0) {
+        TaskDesc* tasks = reinterpret_cast<TaskDesc*>(blob + h.task16 * 16);
+        const int nt = unit_tasks(ce_s, cols, &h, tasks);
+        balance_tasks(tasks, nt);
+    }
 }
 
 // Unpack one item of width B into codes_out (64 bytes) and/or w_out
