@@ -29,11 +29,12 @@
 // stage's row partials of that batch row; for up to 8 batch rows on layouts
 // of 16-column units it stores it instead into the item's own (row, column)
 // slot, which the consumers sum per row after the unit (no shared-memory float
-// additions, which this GPU runs as compare-and-swap loops). The kernel around it is the batch-1
-// pipeline: one persistent block per SM, a copier warp streaming unit blobs by
-// TMA bulk copies into shared-memory stages and writing row partials to Y,
-// consumer warps in teams, two mbarriers per stage, split-K y zeroing by
-// epoch-tagged flags (see vbq_gemv.cu).
+// additions, which this GPU runs as compare-and-swap loops). The kernel
+// around it is the batch-1 pipeline: one persistent block per SM, a copier
+// warp streaming unit blobs by TMA bulk copies into shared-memory stages and
+// writing row partials to Y (in the slot form the consumers write Y), consumer
+// warps in teams, two mbarriers per stage, split-K y zeroing by epoch-tagged
+// flags (see vbq_gemv.cu).
 #include <cstddef>
 
 #include "vbq_kernels.h"
@@ -52,13 +53,16 @@ constexpr int STAGE_BYTES_B = MAX_BLOB_BYTES;
 // banks 4 apart.
 constexpr int YS_STRIDE = RB + 4;
 static_assert(YS_STRIDE % 4 == 0 && RB == 32 * 4, "a warp flushes a batch row's 128 partials 4 per lane");
-// Stages and consumer teams: three stages and one team. With NB = 8 the
-// epilogue stores into slots (one per row, group column and batch row: each
-// row of a unit has exactly one group per column) instead of adding into row
+// Stages and consumer teams. With row partials, NB = 8 leaves room for four
+// stages and up to two teams (a team's next blob lands while it works on the
+// current one); NB = 16 for three stages and one team. The slot form (SL, NB =
+// 8 only) stores into slots (one per row, group column and batch row: each row
+// of a unit has exactly one group per column) instead of adding into row
 // partials: shared-memory float additions are compare-and-swap loops on this
 // GPU (about 7 instructions and 2.6 times a plain store each, measured), and
 // they were a third of the kernel's time. The slots take 64 KB, the room of a
-// fourth stage; NB = 16 would need 128 KB and keeps the row partials.
+// fourth stage, and one team flushes them after every unit, so the slot form
+// pays on wide units only; NB = 16 would need 128 KB and keeps the row partials.
 constexpr int SLOT_MIN_C = 16;          // the slot form for units of at least this many columns
 template <int NB, bool SL> struct Pipe {
     static_assert(!SL || NB == 8, "slots for 8 batch rows only");
