@@ -833,7 +833,7 @@ def run_ours(args, rank, world, local_rank):
         },
         "roofline": {
             "bound": "hbm",
-            "kernel": "gemv1_kernel (vbq_gemv)" if B == 1 else "gemm_kernel (vbq_gemm_small)",
+            "kernel": "gemv1_kernel (vbq_gemv)" if B == 1 else "vbq_gemm_small (gemmb_kernel, or gemv1_kernel<2> for B = 2..4 by layout)",
             "achieved": round(kernel_gbs, 1),
             "peak": peak,
             "peak_kind": peak_kind,
